@@ -1,0 +1,241 @@
+"""fp64 CPU oracle of the DBRX-style MoE layer (arxiv 2506.23635, Sec. 2.1,
+Table 1 notes (d),(e), Sec. 4.2).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` are the only code allowed to import this
+package.  It shares nothing with the CUDA path: the arithmetic lives in
+``moe_oracle.c`` (plain C, fp64, OpenMP over output rows) and this module only
+marshals numpy arrays into it.
+
+Stored arrays use the numpy representation of ``paper_2506_23635_gb300.inputs``:
+``"f32"`` = float32, ``"bf16"`` = uint16 bit patterns.  All functions return
+float64 (values) or int32 (indices).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "moe_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libmoe_oracle.so")
+_DT = {"f32": 0, "bf16": 1}
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ``moe_oracle.c`` with gcc (no -ffast-math) into ``_build/``."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared",
+                           "-std=c11", "-o", tmp, _SRC, "-lm"])
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _bind(path: str) -> ctypes.CDLL:
+    lib = ctypes.CDLL(path)
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.orc_router_logits.argtypes = [I, I, I, P, I, P, I, P]
+    lib.orc_topk_gates.argtypes = [I, I, I, P, P, P]
+    lib.orc_dispatch.argtypes = [I, I, I, P, P, P, P, P]
+    lib.orc_expert_ffn.argtypes = [I, I, P, P, P, P, I, P, P]
+    lib.orc_layer_tokens.argtypes = [I, I, I, I, I, I, P, P, I, P, P, P, P, I,
+                                     P, P, P, P]
+    lib.orc_layer_tokens.restype = I
+    lib.orc_layer_dense_masked.argtypes = [I, I, I, I, I, P, I, P, P, P, P, I, P]
+    lib.orc_layer_dense_masked.restype = I
+    lib.orc_num_threads.restype = I
+    return lib
+
+
+def _c(a: np.ndarray, dt=None) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=dt) if dt is not None else np.ascontiguousarray(a)
+
+
+def _p(a: np.ndarray):
+    return ctypes.c_void_p(a.ctypes.data) if a is not None else None
+
+
+def _storage(a: np.ndarray, dtype: str) -> np.ndarray:
+    return _c(a, np.uint16 if dtype == "bf16" else np.float32)
+
+
+class OracleLib:
+    """The oracle's functions bound to one compiled copy of ``moe_oracle.c``."""
+
+    def __init__(self, path: str):
+        self.path = path
+        self.lib = _bind(path)
+
+    def num_threads(self) -> int:
+        """Threads the oracle's parallel loops use."""
+        return int(self.lib.orc_num_threads())
+
+    def router_logits(self, x, w_r, dtype: str) -> np.ndarray:
+        """logits[t,e] = sum_d x[t,d] W_r[d,e] in fp64 (no bias)."""
+        x, w_r = _storage(x, dtype), _storage(w_r, dtype)
+        T, D = x.shape
+        E = w_r.shape[1]
+        out = np.empty((T, E), np.float64)
+        self.lib.orc_router_logits(T, D, E, _p(x), _DT[dtype], _p(w_r), _DT[dtype],
+                                   _p(out))
+        return out
+
+    def topk_gates(self, logits: np.ndarray, k: int):
+        """Softmax over all experts, K largest logits (descending, ties to the
+        lower index), gates renormalised to sum to 1.  Returns (idx, gate)."""
+        lg = _c(logits, np.float64)
+        T, E = lg.shape
+        idx = np.empty((T, k), np.int32)
+        gate = np.empty((T, k), np.float64)
+        self.lib.orc_topk_gates(T, E, k, _p(lg), _p(idx), _p(gate))
+        return idx, gate
+
+    def dispatch(self, topk_idx: np.ndarray, n_experts: int):
+        """Stable dispatch by (expert, slot).  Returns counts [E], offsets
+        [E+1], perm [S], inv_perm [S] (int32)."""
+        idx = _c(topk_idx, np.int32)
+        T, K = idx.shape
+        if idx.size and (idx.min() < 0 or idx.max() >= n_experts):
+            raise ValueError("expert index out of range")
+        S = T * K
+        counts = np.empty(n_experts, np.int32)
+        offsets = np.empty(n_experts + 1, np.int32)
+        perm = np.empty(S, np.int32)
+        inv = np.empty(S, np.int32)
+        self.lib.orc_dispatch(T, K, n_experts, _p(idx), _p(counts), _p(offsets),
+                              _p(perm), _p(inv))
+        return counts, offsets, perm, inv
+
+    def expert_ffn(self, x_row64: np.ndarray, w1e, v1e, w2e, dtype: str):
+        """One expert on one fp64 token vector: returns (h [F], y [D])."""
+        xt = _c(x_row64, np.float64)
+        w1e, v1e, w2e = (_storage(a, dtype) for a in (w1e, v1e, w2e))
+        F, D = w1e.shape
+        h = np.empty(F, np.float64)
+        y = np.empty(D, np.float64)
+        self.lib.orc_expert_ffn(D, F, _p(xt), _p(w1e), _p(v1e), _p(w2e), _DT[dtype],
+                                _p(h), _p(y))
+        return h, y
+
+    def layer_tokens(self, x, w_r, w1, v1, w2, dtype: str, top_k: int,
+                     tokens=None, residual=None):
+        """The sparse MoE layer for the listed tokens (default: all).
+
+        Returns (out [n,D] f64, idx [n,K] i32, gate [n,K] f64).  ``residual``
+        ([T,D] float64) is added to each output row when given.
+        """
+        x = _storage(x, dtype)
+        w_r, w1, v1, w2 = (_storage(a, dtype) for a in (w_r, w1, v1, w2))
+        T, D = x.shape
+        E, F, _ = w1.shape
+        tok = _c(np.arange(T) if tokens is None else tokens, np.int32)
+        n = tok.shape[0]
+        out = np.empty((n, D), np.float64)
+        idx = np.empty((n, top_k), np.int32)
+        gate = np.empty((n, top_k), np.float64)
+        res = None if residual is None else _c(residual, np.float64)
+        rc = self.lib.orc_layer_tokens(T, D, F, E, top_k, n, _p(tok), _p(x),
+                                       _DT[dtype], _p(w_r), _p(w1), _p(v1), _p(w2),
+                                       _DT[dtype], _p(res), _p(out), _p(idx), _p(gate))
+        if rc != 0:
+            raise ValueError("token index out of range")
+        return out, idx, gate
+
+    def layer_dense_masked(self, x, w_r, w1, v1, w2, dtype: str,
+                           top_k: int) -> np.ndarray:
+        """Busy full loading (Sec. 4.2): all experts on all tokens, unselected
+        outputs zeroed in the weighted sum.  Returns out [T,D] f64."""
+        x = _storage(x, dtype)
+        w_r, w1, v1, w2 = (_storage(a, dtype) for a in (w_r, w1, v1, w2))
+        T, D = x.shape
+        E, F, _ = w1.shape
+        out = np.empty((T, D), np.float64)
+        self.lib.orc_layer_dense_masked(T, D, F, E, top_k, _p(x), _DT[dtype],
+                                        _p(w_r), _p(w1), _p(v1), _p(w2), _DT[dtype],
+                                        _p(out))
+        return out
+
+    def layer_steps(self, x, w_r, w1, v1, w2, dtype: str, top_k: int):
+        """Every intermediate of the layer for all tokens, in the order of the
+        method: logits, (idx, gate), dispatch, per-sorted-slot GLU hidden
+        vectors and expert outputs (ungated), and the combined output."""
+        logits = self.router_logits(x, w_r, dtype)
+        idx, gate = self.topk_gates(logits, top_k)
+        E = w1.shape[0]
+        counts, offsets, perm, inv = self.dispatch(idx, E)
+        x64 = _to_f64(x, dtype)
+        S = perm.shape[0]
+        T, D = x64.shape
+        F = w1.shape[1]
+        h_sorted = np.empty((S, F), np.float64)
+        y_sorted = np.empty((S, D), np.float64)
+        for j in range(S):
+            t, k = divmod(int(perm[j]), top_k)
+            e = int(idx[t, k])
+            h_sorted[j], y_sorted[j] = self.expert_ffn(x64[t], w1[e], v1[e], w2[e], dtype)
+        out = np.zeros((T, D), np.float64)
+        for t in range(T):
+            for k in range(top_k):
+                out[t] += gate[t, k] * y_sorted[inv[t * top_k + k]]
+        return dict(logits=logits, idx=idx, gate=gate, counts=counts,
+                    offsets=offsets, perm=perm, inv_perm=inv, h_sorted=h_sorted,
+                    y_sorted=y_sorted, out=out)
+
+
+def default() -> OracleLib:
+    """The oracle built from this directory's ``moe_oracle.c``."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = OracleLib(build())
+        return _lib
+
+
+def num_threads():
+    return default().num_threads()
+
+
+def router_logits(*a, **k):
+    return default().router_logits(*a, **k)
+
+
+def topk_gates(*a, **k):
+    return default().topk_gates(*a, **k)
+
+
+def dispatch(*a, **k):
+    return default().dispatch(*a, **k)
+
+
+def expert_ffn(*a, **k):
+    return default().expert_ffn(*a, **k)
+
+
+def layer_tokens(*a, **k):
+    return default().layer_tokens(*a, **k)
+
+
+def layer_dense_masked(*a, **k):
+    return default().layer_dense_masked(*a, **k)
+
+
+def layer_steps(*a, **k):
+    return default().layer_steps(*a, **k)
+
+
+def _to_f64(a, dtype):
+    if dtype == "bf16":
+        u = _c(a, np.uint16).astype(np.uint32) << 16
+        return u.view(np.float32).astype(np.float64)
+    return _c(a, np.float32).astype(np.float64)

@@ -1,0 +1,299 @@
+"""Pins of the fp64 oracle against facts fixed outside the oracle itself.
+
+Each ``pin_*`` takes an ``oracle.OracleLib`` and raises ``AssertionError`` if
+the oracle disagrees with:
+
+* exact integer arithmetic (router logits of small integers);
+* brute force over every K-subset (top-k);
+* a closed form of the gates that is not the oracle's formula (pairwise
+  exponentials), the K=1 and K=E special cases (scipy softmax);
+* Python's stable ``sorted`` (dispatch);
+* closed forms of the SiLU-GLU expert on one-hot weights (sigma(ln 3) = 3/4),
+  its linear regime (a library matmul) and the odd-part identity
+  silu(z) - silu(-z) = z, which reduces the expert to a bilinear form;
+* invariants of the layer: identical experts, K = 1, token permutation, expert
+  relabelling, busy full loading (Sec. 4.2), linearity in W2 and V1.
+
+The same pins are run against deliberately broken copies of the oracle in
+``test_oracle_mutations.py``, so each plausible mistake is shown to fail one.
+"""
+from __future__ import annotations
+
+import itertools
+import math
+
+import numpy as np
+
+from paper_2506_23635_gb300 import inputs as gen
+
+LN3 = math.log(3.0)
+
+
+def _close(a, b, rtol, atol=0.0, msg=""):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    assert a.shape == b.shape, f"{msg}: shape {a.shape} vs {b.shape}"
+    err = np.abs(a - b)
+    lim = atol + rtol * np.abs(b)
+    assert np.all(err <= lim), f"{msg}: max err {err.max()} (limit {lim.max()})"
+
+
+# --------------------------------------------------------------------------
+# router
+# --------------------------------------------------------------------------
+
+
+def pin_router_exact_integers(orc):
+    """Small-integer x and W_r are exact in f32 and bf16; their dot products
+    are exact integers, computed here with Python ints."""
+    rng = np.random.default_rng(11)
+    T, D, E = 3, 7, 5
+    xi = rng.integers(-8, 9, size=(T, D))
+    wi = rng.integers(-8, 9, size=(D, E))
+    want = np.array([[sum(int(xi[t, d]) * int(wi[d, e]) for d in range(D))
+                      for e in range(E)] for t in range(T)], np.float64)
+    for dt in ("f32", "bf16"):
+        got = orc.router_logits(gen.store(xi, dt), gen.store(wi, dt), dt)
+        assert np.array_equal(got, want), f"router logits ({dt})"
+
+
+# --------------------------------------------------------------------------
+# softmax -> top-k -> renormalised gates
+# --------------------------------------------------------------------------
+
+
+def pin_topk_bruteforce(orc):
+    rng = np.random.default_rng(12)
+    for E in (2, 3, 5, 8):
+        for K in range(1, E + 1):
+            lg = rng.normal(size=(40, E)) * 2.0
+            idx, _ = orc.topk_gates(lg, K)
+            for t in range(lg.shape[0]):
+                best = max(itertools.combinations(range(E), K),
+                           key=lambda c: sum(lg[t, list(c)]))
+                assert set(idx[t].tolist()) == set(best), "top-k set"
+                vals = lg[t, idx[t]]
+                assert np.all(vals[:-1] > vals[1:]), "top-k order"
+
+
+def pin_topk_ties(orc):
+    idx, _ = orc.topk_gates(np.array([[1.0, 3.0, 3.0, 2.0]]), 2)
+    assert idx.tolist() == [[1, 2]], "tie keeps lower index first"
+    idx, _ = orc.topk_gates(np.array([[5.0, 5.0, 5.0, 5.0]]), 3)
+    assert idx.tolist() == [[0, 1, 2]], "all-equal logits"
+    idx, _ = orc.topk_gates(np.array([[0.0, 7.0, 7.0, 7.0, 1.0]]), 4)
+    assert idx.tolist() == [[1, 2, 3, 4]], "ties then smaller"
+
+
+def pin_gates_closed_form(orc):
+    """g_k = 1 / sum_j exp(l_j - l_k) over the selected j."""
+    rng = np.random.default_rng(13)
+    E, K = 16, 4
+    lg = rng.normal(size=(64, E)) * 3.0
+    idx, gate = orc.topk_gates(lg, K)
+    for t in range(lg.shape[0]):
+        sel = [lg[t, e] for e in idx[t]]
+        want = [1.0 / sum(math.exp(lj - lk) for lj in sel) for lk in sel]
+        _close(gate[t], want, 1e-13, msg="gate closed form")
+    _close(gate.sum(axis=1), np.ones(lg.shape[0]), 1e-14, msg="sum of gates")
+
+
+def pin_gates_special_cases(orc):
+    from scipy.special import softmax
+
+    rng = np.random.default_rng(14)
+    lg = rng.normal(size=(32, 6)) * 4.0
+    _, g1 = orc.topk_gates(lg, 1)
+    assert np.all(g1 == 1.0), "K=1 gate is exactly 1"
+    idx, gE = orc.topk_gates(lg, 6)
+    want = np.take_along_axis(softmax(lg, axis=1), idx.astype(np.int64), axis=1)
+    _close(gE, want, 1e-13, msg="K=E gates = softmax")
+
+
+# --------------------------------------------------------------------------
+# dispatch
+# --------------------------------------------------------------------------
+
+
+def pin_dispatch_stable_sort(orc):
+    rng = np.random.default_rng(15)
+    for (T, E, K) in ((1, 16, 4), (37, 16, 4), (64, 5, 2), (300, 7, 1), (9, 3, 3)):
+        idx = np.stack([rng.permutation(E)[:K] for _ in range(T)]).astype(np.int32)
+        flat = idx.reshape(-1)
+        S = flat.size
+        counts, offsets, perm, inv = orc.dispatch(idx, E)
+        assert np.array_equal(counts, np.bincount(flat, minlength=E)), "counts"
+        assert np.array_equal(offsets, np.concatenate([[0], np.cumsum(counts)])), "offsets"
+        want = sorted(range(S), key=lambda s: (int(flat[s]), s))
+        assert perm.tolist() == want, "perm = stable sort by expert"
+        assert np.array_equal(inv[perm], np.arange(S)), "inv_perm inverts perm"
+
+
+# --------------------------------------------------------------------------
+# SiLU-GLU expert
+# --------------------------------------------------------------------------
+
+
+def _silu(z):
+    return z / (1.0 + math.exp(-z))
+
+
+def pin_expert_one_hot_closed_form(orc):
+    """One-hot W1/V1 rows pick x entries; sigma(ln 3) = 3/4, sigma(-ln 3) = 1/4.
+
+    D=5, F=3 so a transposed operand cannot pass."""
+    D, F = 5, 3
+    x = np.array([LN3, -LN3, 2.0, 0.5, 0.0])
+    w1 = np.zeros((F, D)); v1 = np.zeros((F, D))
+    for f, (d1, d2, c2) in enumerate(((0, 2, 1.0), (1, 3, 2.0), (4, 2, -1.0))):
+        w1[f, d1] = 1.0
+        v1[f, d2] = c2
+    w2 = np.array([[1, 0, 0], [0, 1, 0], [1, 1, 0], [0, 0, 1], [2, 0, -1]], np.float64)
+    x32 = x.astype(np.float32).astype(np.float64)
+    h, y = orc.expert_ffn(x32, gen.store(w1, "f32"), gen.store(v1, "f32"),
+                          gen.store(w2, "f32"), "f32")
+    h_want = np.array([0.75 * LN3 * 2.0, -0.25 * LN3 * 1.0, 0.0])
+    y_want = np.array([h_want[0], h_want[1], h_want[0] + h_want[1], h_want[2],
+                       2.0 * h_want[0] - h_want[2]])
+    _close(h, h_want, 1e-7, 1e-12, msg="GLU hidden, closed form")
+    _close(y, y_want, 1e-7, 1e-12, msg="expert output, closed form")
+
+
+def pin_expert_linear_regime(orc):
+    """With b = 1 and a >= 50, SiLU(a) = a to 1e-21, so the expert is the
+    plain product W2 (W1 x); with a <= -50 it is 0."""
+    rng = np.random.default_rng(16)
+    D, F = 16, 24
+    x = rng.normal(size=D); x[0] = 1.0
+    w1 = rng.normal(size=(F, D)) * 0.01; w1[:, 0] = 60.0
+    v1 = np.zeros((F, D)); v1[:, 0] = 1.0
+    w2 = rng.normal(size=(D, F))
+    S = lambda a: gen.store(a, "f32")
+    xs = S(x).astype(np.float64)
+    w1s, v1s, w2s = (S(a).astype(np.float64) for a in (w1, v1, w2))
+    _, y = orc.expert_ffn(xs, S(w1), S(v1), S(w2), "f32")
+    _close(y, w2s @ (w1s @ xs), 1e-12, 1e-12, msg="linear regime")
+    _, yneg = orc.expert_ffn(xs, S(-w1), S(v1), S(w2), "f32")
+    assert np.max(np.abs(yneg)) < 1e-15, "negative regime is zero"
+
+
+def pin_expert_odd_part(orc):
+    """silu(z) - silu(-z) = z, so y(W1) - y(-W1) = W2 ((W1 x) * (V1 x))."""
+    rng = np.random.default_rng(17)
+    D, F = 24, 40
+    for dt in ("f32", "bf16"):
+        x = gen.store(rng.normal(size=D), dt)
+        w1 = gen.store(rng.normal(size=(F, D)) * 0.3, dt)
+        v1 = gen.store(rng.normal(size=(F, D)) * 0.3, dt)
+        w2 = gen.store(rng.normal(size=(D, F)) * 0.3, dt)
+        w1n = gen.store(-gen.to_f64(w1, dt), dt)  # exact negation
+        x64 = gen.to_f64(x, dt)
+        _, yp = orc.expert_ffn(x64, w1, v1, w2, dt)
+        _, yn = orc.expert_ffn(x64, w1n, v1, w2, dt)
+        W1, V1, W2 = (gen.to_f64(a, dt) for a in (w1, v1, w2))
+        want = W2 @ ((W1 @ x64) * (V1 @ x64))
+        _close(yp - yn, want, 1e-11, 1e-11, msg=f"odd part ({dt})")
+
+
+# --------------------------------------------------------------------------
+# whole-layer invariants
+# --------------------------------------------------------------------------
+
+
+def _small_layer(seed=21, T=12, E=5, K=2, D=32, F=48, dt="f32"):
+    shape = gen.LayerShape(D, F, E, K, dt)
+    L = gen.host_layer(shape, T, seed)
+    # larger weights than the DBRX recipe so that every term is visible
+    rng = np.random.default_rng(seed)
+    L.w1 = gen.store(rng.normal(size=(E, F, D)) * 0.2, dt)
+    L.v1 = gen.store(rng.normal(size=(E, F, D)) * 0.2, dt)
+    L.w2 = gen.store(rng.normal(size=(E, D, F)) * 0.2, dt)
+    L.w_r = gen.store(rng.normal(size=(D, E)) * 0.5, dt)
+    L.x = gen.gap_condition_tokens(L.x, L.w_r, shape, seed, 1e-3)
+    return L
+
+
+def pin_layer_identical_experts(orc):
+    """Identical experts: the layer is one expert, whatever the routing."""
+    L = _small_layer()
+    sh = L.shape
+    for a in (L.w1, L.v1, L.w2):
+        a[:] = a[0]
+    out, _, gate = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    x64 = gen.to_f64(L.x, sh.dtype)
+    for t in range(x64.shape[0]):
+        _, y = orc.expert_ffn(x64[t], L.w1[0], L.v1[0], L.w2[0], sh.dtype)
+        _close(out[t], y, 1e-12, 1e-12, msg="identical experts")
+
+
+def pin_layer_k1_one_expert(orc):
+    """K = 1: the output is exactly the arg-max expert's output."""
+    L = _small_layer(K=1)
+    sh = L.shape
+    out, idx, gate = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, 1)
+    lg = gen.to_f64(L.x, sh.dtype) @ gen.to_f64(L.w_r, sh.dtype)
+    assert np.array_equal(idx[:, 0], np.argmax(lg, axis=1)), "K=1 expert"
+    assert np.all(gate == 1.0)
+    x64 = gen.to_f64(L.x, sh.dtype)
+    for t in range(x64.shape[0]):
+        e = int(idx[t, 0])
+        _, y = orc.expert_ffn(x64[t], L.w1[e], L.v1[e], L.w2[e], sh.dtype)
+        assert np.array_equal(out[t], y), "K=1 output"
+
+
+def pin_layer_token_permutation(orc):
+    L = _small_layer()
+    sh = L.shape
+    out, idx, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    p = np.random.default_rng(5).permutation(L.x.shape[0])
+    out_p, idx_p, _ = orc.layer_tokens(L.x[p], L.w_r, L.w1, L.v1, L.w2, sh.dtype,
+                                       sh.top_k)
+    _close(out_p, out[p], 1e-13, 1e-13, msg="token permutation")
+    assert np.array_equal(idx_p, idx[p])
+
+
+def pin_layer_expert_relabel(orc):
+    L = _small_layer()
+    sh = L.shape
+    out, idx, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    s = np.random.default_rng(6).permutation(sh.n_experts)
+    out_s, idx_s, _ = orc.layer_tokens(L.x, L.w_r[:, s], L.w1[s], L.v1[s], L.w2[s],
+                                       sh.dtype, sh.top_k)
+    _close(out_s, out, 1e-13, 1e-13, msg="expert relabelling")
+    assert np.array_equal(s[idx_s], idx)
+
+
+def pin_layer_busy_full_loading(orc):
+    """Sec. 4.2: computing all experts and zeroing the unselected ones in the
+    weighted sum gives the same layer."""
+    L = _small_layer()
+    sh = L.shape
+    out, _, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    dense = orc.layer_dense_masked(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    _close(dense, out, 1e-13, 1e-13, msg="busy full loading")
+
+
+def pin_layer_linear_in_w2_v1(orc):
+    L = _small_layer()
+    sh = L.shape
+    out, _, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    out2, _, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2 * 2, sh.dtype, sh.top_k)
+    out3, _, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1 * 4, L.w2, sh.dtype, sh.top_k)
+    assert np.array_equal(out2, 2 * out), "linear in W2"
+    assert np.array_equal(out3, 4 * out), "linear in V1"
+
+
+def pin_layer_steps_agree(orc):
+    """The step-by-step route (dispatch, per-slot experts, combine) equals the
+    per-token route."""
+    L = _small_layer(T=9, E=4, K=3)
+    sh = L.shape
+    out, idx, gate = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    st = orc.layer_steps(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    assert np.array_equal(st["idx"], idx)
+    _close(st["gate"], gate, 1e-15, msg="gates")
+    _close(st["out"], out, 1e-13, 1e-13, msg="steps vs tokens")
+    assert st["counts"].sum() == idx.size
+
+
+ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

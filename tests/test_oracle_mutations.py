@@ -1,0 +1,56 @@
+"""Each plausible mistake planted in a copy of the oracle fails at least one
+pin.  The copies are compiled with gcc into a temporary directory; the oracle
+in the repository is never modified."""
+import os
+import subprocess
+
+import pytest
+
+import oracle
+from tests import oracle_pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "moe_oracle.c")
+
+# (name, original text, mutated text)
+MUTATIONS = [
+    ("silu_on_v1", "h[f] = a / (1.0 + exp(-a)) * b;", "h[f] = b / (1.0 + exp(-b)) * a;"),
+    ("sigmoid_sign", "h[f] = a / (1.0 + exp(-a)) * b;", "h[f] = a / (1.0 + exp(a)) * b;"),
+    ("no_silu", "h[f] = a / (1.0 + exp(-a)) * b;", "h[f] = a * b;"),
+    ("w2_transposed", "h[f] * orc_load(w2e, wdt, (size_t)d * F + f)",
+     "h[f] * orc_load(w2e, wdt, (size_t)f * D + d)"),
+    ("w1_dropped_term", "for (int d = 0; d < D; ++d) {\n            a +=",
+     "for (int d = 1; d < D; ++d) {\n            a +="),
+    ("router_transposed", "orc_load(wr, wdt, (size_t)d * E + e)",
+     "orc_load(wr, wdt, (size_t)e * D + d)"),
+    ("tie_to_higher_index", "if (best < 0 || l[e] > l[best]) best = e;",
+     "if (best < 0 || l[e] >= l[best]) best = e;"),
+    ("no_renormalisation", "gate[(size_t)t * K + k] = p[idx[(size_t)t * K + k]] / psel;",
+     "gate[(size_t)t * K + k] = p[idx[(size_t)t * K + k]];"),
+    ("softmax_sign", "p[e] = exp(l[e] - m);", "p[e] = exp(m - l[e]);"),
+    ("dispatch_reversed", "for (int s = 0; s < S; ++s)\n            if (idx[s] == e) {",
+     "for (int s = S - 1; s >= 0; --s)\n            if (idx[s] == e) {"),
+    ("offsets_not_scanned", "offsets[e + 1] = offsets[e] + counts[e];",
+     "offsets[e + 1] = counts[e];"),
+    ("combine_ungated", "for (int d = 0; d < D; ++d) o[d] += g[k] * y[d];",
+     "for (int d = 0; d < D; ++d) o[d] += y[d];"),
+    ("dense_mask_ungated", "mask[idx[k]] = g[k];", "mask[idx[k]] = 1.0;"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_mutation_is_caught(tmp_path, name, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation site for {name} not unique"
+    mutated = tmp_path / "moe_oracle_mut.c"
+    mutated.write_text(src.replace(old, new))
+    so = tmp_path / f"libmut_{name}.so"
+    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11",
+                           "-o", str(so), str(mutated), "-lm"])
+    orc = oracle.OracleLib(str(so))
+    failed = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(orc)
+        except AssertionError:
+            failed.append(pin.__name__)
+    assert failed, f"mutation {name} passed every pin"
