@@ -1,0 +1,183 @@
+/*
+ * moe.h -- C ABI of the GB300 (sm_103a) DBRX-style Mixture-of-Experts layer.
+ *
+ * The layer is the one of arxiv 2506.23635 (Sec. 2.1; Table 1 and its notes
+ * (d),(e)): every token is routed to top_k of n_experts feed-forward experts,
+ * each expert is a SiLU-GLU FFN with three matrices w1, v1, w2 of size
+ * d_model x ffn_hidden, and the selected experts' outputs are combined by a
+ * weighted sum (Table 2 caption; Sec. 4.2).  With all experts resident in one
+ * GPU's memory the layer is five steps, each exported here:
+ *
+ *   moe_route        router product, softmax, top-k, renormalised gates
+ *   moe_dispatch     histogram, prefix sum and stable permutation
+ *   moe_expert_ffn   grouped SiLU-GLU expert FFN over sorted slots
+ *   moe_combine      gated combine back to token order
+ *   moe_layer_forward  all of the above, fused where it pays
+ *
+ * Formulas (the paper gives the structure; the router and GLU formula are
+ * the standard DBRX readings):
+ *   logits[t,e] = sum_d x[t,d] * w_router[d,e]
+ *   p[t,:] = softmax(logits[t,:]);  idx[t,0..K) = K largest logits,
+ *            descending, ties to the lower expert index
+ *   gate[t,k] = p[t,idx[t,k]] / sum_j p[t,idx[t,j]]
+ *   h = SiLU(x . w1[e]^T) * (x . v1[e]^T),  SiLU(z) = z * sigmoid(z)
+ *   y = h . w2[e]^T;   out[t,:] = sum_k gate[t,k] * y[(t,k),:]
+ *
+ * Layouts (row-major, all experts of a tensor in one contiguous allocation):
+ *   x [T, D]; w_router [D, E]; w1, v1 [E, F, D]; w2 [E, D, F];
+ *   a slot is s = t*K + k; "sorted" arrays are indexed by the position of a
+ *   slot in the dispatch order (by expert, then by s).
+ *
+ * Conventions shared by every entry point:
+ *   - Tensor pointers are DEVICE pointers owned by the caller, 16-byte
+ *     aligned.  The library allocates no device memory; scratch space is the
+ *     caller's workspace (moe_workspace_size).
+ *   - Calls are asynchronous on `stream` and never synchronise with the host
+ *     (except moe_get_last_error and moe_profile_read).
+ *   - Arguments are validated before anything is launched; on a validation
+ *     error nothing is written and the status says why.
+ *   - T == 0 is valid and launches nothing (moe_dispatch still writes zero
+ *     counts and offsets).
+ *   - Limits: 1 <= top_k <= n_experts <= 256; d_model and ffn_hidden are
+ *     multiples of 8, 8 <= d_model <= 49152, 8 <= ffn_hidden <= 65536;
+ *     T <= 1048576 and T*top_k <= 16777216; w_dtype == x_dtype.
+ *   - Errors found by kernels (an expert index out of range, a bounded wait
+ *     that ran out) are recorded on the device and reported by
+ *     moe_get_last_error.
+ */
+#ifndef MOE_H_
+#define MOE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st *moe_stream_t;
+
+typedef enum {
+    MOE_OK = 0,
+    MOE_ERR_INVALID_ARG = 1,  /* null pointer, bad size, misaligned pointer */
+    MOE_ERR_UNSUPPORTED = 2,  /* a dtype combination that is not built */
+    MOE_ERR_WORKSPACE = 3,    /* workspace missing or too small */
+    MOE_ERR_CUDA = 4,         /* a CUDA call or kernel launch failed */
+    MOE_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up */
+    MOE_ERR_DEVICE_INDEX = 6  /* a kernel met an expert index outside [0,E) */
+} moe_status;
+
+typedef enum { MOE_F32 = 0, MOE_BF16 = 1 } moe_dtype;
+
+typedef struct {
+    int32_t d_model;    /* D, Table 1 "D_embed" (6144 for DBRX) */
+    int32_t ffn_hidden; /* F, Table 1 "D_ffn" (10752 for DBRX) */
+    int32_t n_experts;  /* E, Sec. 2.1 (16 for DBRX) */
+    int32_t top_k;      /* K, Sec. 2.1 (4 for DBRX) */
+    int32_t w_dtype;    /* moe_dtype of w_router, w1, v1, w2 */
+    int32_t x_dtype;    /* moe_dtype of x and of a residual */
+    int32_t out_dtype;  /* moe_dtype of out */
+} moe_dims;
+
+/* Bytes of workspace moe_layer_forward and moe_expert_ffn need for up to
+ * max_tokens tokens (a multiple of 256).  Writes *bytes; MOE_ERR_INVALID_ARG
+ * for bad dims or max_tokens < 0. */
+moe_status moe_workspace_size(const moe_dims *dims, int32_t max_tokens,
+                              size_t *bytes);
+
+/* Step 1 -- router and gates (Sec. 2.1 "selects 4 out of 16"; Table 2
+ * caption lists the router under "Misc").
+ *   x          [T, D]  x_dtype
+ *   w_router   [D, E]  w_dtype
+ *   logits_opt [T, E]  float32, written if non-NULL
+ *   topk_idx   [T, K]  int32 expert ids, descending logit, ties -> lower id
+ *   topk_gate  [T, K]  float32 renormalised gates (sum over k is 1)
+ * fp32 accumulation.  Errors: MOE_ERR_INVALID_ARG (nulls, sizes). */
+moe_status moe_route(const moe_dims *dims, int32_t T, const void *x,
+                     const void *w_router, float *logits_opt,
+                     int32_t *topk_idx, float *topk_gate, moe_stream_t stream);
+
+/* Step 2 -- dispatch of the T*K slots to experts (the fork of Sec. 3.1,
+ * Fig. 2: tokens go to the nodes holding their selected experts).
+ *   topk_idx [T, K]  int32 in [0, E)
+ *   counts   [E]     int32, slots per expert
+ *   offsets  [E+1]   int32, exclusive prefix sum of counts
+ *   perm     [T*K]   int32, perm[j] = slot at sorted position j; slots of an
+ *                    expert are in ascending slot order (stable)
+ *   inv_perm [T*K]   int32, inv_perm[s] = sorted position of slot s
+ * Deterministic and bit-exact.  An index outside [0,E) is recorded as
+ * MOE_ERR_DEVICE_INDEX (read by moe_get_last_error) and that slot is left
+ * out of the permutation. */
+moe_status moe_dispatch(const moe_dims *dims, int32_t T,
+                        const int32_t *topk_idx, int32_t *counts,
+                        int32_t *offsets, int32_t *perm, int32_t *inv_perm,
+                        moe_stream_t stream);
+
+/* Step 3 -- grouped SiLU-GLU expert FFN (Table 1 notes (d),(e): w1, v1, w2),
+ * ungated, over the sorted slots.
+ *   x        [T, D]    x_dtype
+ *   perm     [T*K], offsets [E+1]   from moe_dispatch
+ *   w1, v1   [E, F, D] w_dtype;  w2 [E, D, F] w_dtype
+ *   y_sorted [T*K, D]  float32: y_sorted[j] = expert(e_j)(x[perm[j] / K])
+ *   ws       workspace of at least moe_workspace_size(dims, T) bytes
+ * fp32 accumulation; the GLU hidden vector is kept in fp32 (small T) or
+ * rounded to bf16 before the down projection (tensor-core path). */
+moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x,
+                          const int32_t *perm, const int32_t *offsets,
+                          const void *w1, const void *v1, const void *w2,
+                          float *y_sorted, void *ws, size_t ws_bytes,
+                          moe_stream_t stream);
+
+/* Step 4 -- weighted combine (Sec. 4.2 "weighted sum"; Sec. 4.3).
+ *   y_sorted     [T*K, D] float32;  inv_perm [T*K];  topk_gate [T, K]
+ *   residual_opt [T, D]   x_dtype, added if non-NULL
+ *   out          [T, D]   out_dtype
+ *   out[t,:] = residual[t,:] + sum_{k=0..K-1} gate[t,k] * y_sorted[inv_perm[t*K+k],:]
+ * summed in ascending k. */
+moe_status moe_combine(const moe_dims *dims, int32_t T, const float *y_sorted,
+                       const int32_t *inv_perm, const float *topk_gate,
+                       const void *residual_opt, void *out,
+                       moe_stream_t stream);
+
+/* The whole layer: route, dispatch, expert FFN and combine, with the gate
+ * and combine fused into the expert kernels where the token count allows.
+ *   x [T,D], w_router [D,E], w1/v1 [E,F,D], w2 [E,D,F] as above;
+ *   residual_opt [T,D] x_dtype or NULL;  out [T,D] out_dtype;
+ *   ws  workspace of at least moe_workspace_size(dims, T) bytes.
+ * No host synchronisation; capturable in a CUDA graph. */
+moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x,
+                             const void *w_router, const void *w1,
+                             const void *v1, const void *w2,
+                             const void *residual_opt, void *out, void *ws,
+                             size_t ws_bytes, moe_stream_t stream);
+
+/* Human-readable name of a status. */
+const char *moe_status_string(moe_status status);
+
+/* Synchronises `stream`, then reports (and clears) the first error recorded
+ * by a kernel since the last call, or MOE_ERR_CUDA for a failed launch or an
+ * asynchronous CUDA fault. */
+moe_status moe_get_last_error(moe_stream_t stream);
+
+/* ---- launch accounting and per-kernel timing (benchmarks) ---------------
+ * moe_launch_count: number of kernels this library has launched since load.
+ * moe_profile_enable(1): every later kernel launch is bracketed by a pair of
+ * CUDA events recorded on its own stream; moe_profile_read synchronises those
+ * events and returns, per kernel name, the launches and the summed
+ * event-measured milliseconds since the last moe_profile_reset. */
+typedef struct {
+    char name[48];
+    int64_t launches;
+    double total_ms;
+} moe_kernel_stat;
+
+int64_t moe_launch_count(void);
+void moe_profile_enable(int on);
+void moe_profile_reset(void);
+int32_t moe_profile_read(moe_kernel_stat *stats, int32_t max_stats);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MOE_H_ */

@@ -1,0 +1,609 @@
+// C ABI of libmoe (include/moe.h): argument validation, workspace layout,
+// launch bookkeeping, and the small kernels of the layer -- router + gates,
+// dispatch, and the unfused combine.
+#include <algorithm>
+#include <atomic>
+#include <mutex>
+#include <string.h>
+#include <string>
+#include <vector>
+
+#include "moe_internal.cuh"
+
+namespace moe {
+
+__device__ unsigned g_moe_err = 0;
+
+// ===========================================================================
+// Step 1: router logits, softmax, top-k, renormalised gates.
+// A block of 256 threads handles kRouteTokens tokens; its threads split d,
+// each accumulating 16 experts at a time for every token, then the partial
+// sums are reduced across the block.  Warp w then selects the top-k of token
+// w: K rounds of a warp arg-max over the not-yet-taken experts, ties going
+// to the lower expert index.
+// ===========================================================================
+constexpr int kRouteThreads = 256;
+constexpr int kRouteTokens = 4;
+
+template <typename TX, typename TW>
+__global__ void __launch_bounds__(kRouteThreads)
+k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restrict__ wr,
+        float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
+        float *__restrict__ topk_gate) {
+    constexpr int TT = kRouteTokens, NW = kRouteThreads / 32;
+    __shared__ float red[NW][TT * 16];
+    __shared__ float lg[TT][256];
+    __shared__ float pk[TT][256];
+    const int t0 = blockIdx.x * TT;
+    const int nt = min(TT, T - t0);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    for (int e0 = 0; e0 < E; e0 += 16) {
+        const int ne = min(16, E - e0);
+        float acc[TT][16];
+#pragma unroll
+        for (int a = 0; a < TT; ++a)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) acc[a][j] = 0.f;
+        for (int d = threadIdx.x; d < D; d += kRouteThreads) {
+            float xv[TT];
+#pragma unroll
+            for (int a = 0; a < TT; ++a) xv[a] = a < nt ? to_f(x[(size_t)(t0 + a) * D + d]) : 0.f;
+            const TW *wrow = wr + (size_t)d * E + e0;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                if (j < ne) {
+                    const float w = to_f(wrow[j]);
+#pragma unroll
+                    for (int a = 0; a < TT; ++a) acc[a][j] = fmaf(xv[a], w, acc[a][j]);
+                }
+            }
+        }
+#pragma unroll
+        for (int a = 0; a < TT; ++a)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float v = warp_sum(acc[a][j]);
+                if (lane == 0) red[warp][a * 16 + j] = v;
+            }
+        __syncthreads();
+        for (int i = threadIdx.x; i < TT * 16; i += kRouteThreads) {
+            const int a = i >> 4, j = i & 15;
+            if (a < nt && j < ne) {
+                float s = 0.f;
+#pragma unroll
+                for (int w = 0; w < NW; ++w) s += red[w][i];
+                lg[a][e0 + j] = s;
+            }
+        }
+        __syncthreads();
+    }
+
+    if (warp >= nt) return;
+    const int t = t0 + warp;
+    const float *l = lg[warp];
+    if (logits_opt)
+        for (int e = lane; e < E; e += 32) logits_opt[(size_t)t * E + e] = l[e];
+    float m = -INFINITY;
+    for (int e = lane; e < E; e += 32) m = fmaxf(m, l[e]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float z = 0.f;
+    for (int e = lane; e < E; e += 32) z += expf(l[e] - m);
+    z = warp_sum(z);
+
+    uint32_t taken = 0;  // bit i: expert lane + 32*i already selected
+    float psel = 0.f;
+    for (int k = 0; k < K; ++k) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int i = 0, e = lane; e < E; ++i, e += 32) {
+            if ((taken >> i) & 1u) continue;
+            const float v = l[e];
+            if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+        }
+        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+        const float p = expf(bv - m) / z;
+        psel += p;
+        if (lane == 0) {
+            topk_idx[(size_t)t * K + k] = bi;
+            pk[warp][k] = p;
+        }
+    }
+    __syncwarp();
+    for (int k = lane; k < K; k += 32) topk_gate[(size_t)t * K + k] = pk[warp][k] / psel;
+}
+
+// ===========================================================================
+// Step 2: dispatch.  One block of 1024 threads: a shared-memory histogram,
+// an exclusive scan, then a stable counting sort over chunks of 1024 slots.
+// Within a chunk a slot's rank among equal experts is its rank in its warp
+// (__match_any_sync) plus the counts of the same expert in lower warps, so
+// the order is ascending slot order and needs no atomics.
+// ===========================================================================
+constexpr int kDispatchThreads = 1024;
+
+__global__ void __launch_bounds__(kDispatchThreads)
+k_dispatch(int S, int E, const int32_t *__restrict__ idx, int32_t *__restrict__ counts,
+           int32_t *__restrict__ offsets, int32_t *__restrict__ perm,
+           int32_t *__restrict__ inv_perm, unsigned *err) {
+    constexpr int NW = kDispatchThreads / 32;
+    __shared__ int cnt[256];
+    __shared__ int run[256];
+    __shared__ int wh[NW][256];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    for (int e = tid; e < E; e += kDispatchThreads) cnt[e] = 0;
+    __syncthreads();
+    for (int s = tid; s < S; s += kDispatchThreads) {
+        const int e = idx[s];
+        if (e >= 0 && e < E) atomicAdd(&cnt[e], 1);
+        else set_error(err, kErrIndex);
+    }
+    __syncthreads();
+    if (warp == 0) {  // exclusive scan of cnt over E <= 256 experts
+        int carry = 0;
+        for (int base = 0; base < E; base += 32) {
+            const int e = base + lane;
+            const int c = e < E ? cnt[e] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (e < E) {
+                run[e] = carry + incl - c;
+                counts[e] = c;
+                offsets[e] = carry + incl - c;
+            }
+            carry += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) offsets[E] = carry;
+    }
+    __syncthreads();
+
+    const unsigned lt_mask = (1u << lane) - 1u;
+    for (int c0 = 0; c0 < S; c0 += kDispatchThreads) {
+        for (int i = tid; i < NW * E; i += kDispatchThreads) wh[i / E][i % E] = 0;
+        __syncthreads();
+        const int s = c0 + tid;
+        int e = s < S ? idx[s] : -1;
+        const bool valid = e >= 0 && e < E;
+        if (!valid) e = -1;
+        const unsigned same = __match_any_sync(0xffffffffu, e);
+        const int rank = __popc(same & lt_mask);
+        if (valid && rank == 0) wh[warp][e] = __popc(same);
+        __syncthreads();
+        if (valid) {
+            int pre = 0;
+            for (int w = 0; w < warp; ++w) pre += wh[w][e];
+            const int pos = run[e] + pre + rank;
+            perm[pos] = s;
+            inv_perm[s] = pos;
+        } else if (s < S) {
+            inv_perm[s] = -1;
+        }
+        __syncthreads();
+        for (int ee = tid; ee < E; ee += kDispatchThreads) {
+            int tot = 0;
+            for (int w = 0; w < NW; ++w) tot += wh[w][ee];
+            run[ee] += tot;
+        }
+        __syncthreads();
+    }
+}
+
+// ===========================================================================
+// Step 4 (unfused): out[t,:] = residual + sum_k gate[t,k] * y_sorted[inv[t*K+k],:]
+// One thread per 4 consecutive outputs; k in ascending order.
+// ===========================================================================
+template <typename TO, typename TR>
+__global__ void __launch_bounds__(256)
+k_combine(int T, int D, int K, const float *__restrict__ y, const int32_t *__restrict__ inv,
+          const float *__restrict__ gate, const TR *__restrict__ residual, TO *__restrict__ out,
+          unsigned *err) {
+    const int S = T * K;
+    const int nq = D >> 2;
+    const long long total = (long long)T * nq;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int t = (int)(i / nq);
+        const int d = (int)(i - (long long)t * nq) * 4;
+        float a[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int k = 0; k < K; ++k) {
+            const int j = inv[(size_t)t * K + k];
+            if (j < 0 || j >= S) {  // a slot left out by dispatch, or a corrupt index
+                if (j >= S) set_error(err, kErrIndex);
+                continue;
+            }
+            const float g = gate[(size_t)t * K + k];
+            const float4 v = *reinterpret_cast<const float4 *>(y + (size_t)j * D + d);
+            a[0] = fmaf(g, v.x, a[0]); a[1] = fmaf(g, v.y, a[1]);
+            a[2] = fmaf(g, v.z, a[2]); a[3] = fmaf(g, v.w, a[3]);
+        }
+        if (residual)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) a[q] += to_f(residual[(size_t)t * D + d + q]);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) out[(size_t)t * D + d + q] = from_f<TO>(a[q]);
+    }
+}
+
+// ===========================================================================
+// host side
+// ===========================================================================
+
+const DeviceInfo &device_info() {
+    static DeviceInfo info[64];
+    static bool ready[64];
+    static std::mutex mu;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64) dev = 0;
+    std::lock_guard<std::mutex> g(mu);
+    if (!ready[dev]) {
+        int sms = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        void *p = nullptr;
+        cudaGetSymbolAddress(&p, g_moe_err);
+        info[dev].sm_count = sms > 0 ? sms : 1;
+        info[dev].err = static_cast<unsigned *>(p);
+        ready[dev] = true;
+    }
+    return info[dev];
+}
+
+namespace {
+
+struct ProfState {
+    std::mutex mu;
+    bool on = false;
+    std::vector<std::string> names;
+    std::vector<int64_t> launches;
+    std::vector<double> ms;
+    struct Pending { int kind; cudaEvent_t a, b; };
+    std::vector<Pending> pending;
+    std::vector<cudaEvent_t> pool;
+    std::vector<cudaEvent_t> begin_of_slot;  // begin event of each open launch
+};
+
+ProfState &prof() {
+    static ProfState *p = new ProfState();  // never destroyed: used at exit
+    return *p;
+}
+
+std::atomic<int64_t> g_launches{0};
+
+cudaEvent_t take_event(ProfState &P) {
+    if (!P.pool.empty()) {
+        cudaEvent_t e = P.pool.back();
+        P.pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+int kind_of(ProfState &P, const char *name) {
+    for (size_t i = 0; i < P.names.size(); ++i)
+        if (P.names[i] == name) return (int)i;
+    P.names.push_back(name);
+    P.launches.push_back(0);
+    P.ms.push_back(0.0);
+    return (int)P.names.size() - 1;
+}
+
+}  // namespace
+
+LaunchScope::LaunchScope(const char *n, cudaStream_t s) : name(n), stream(s), slot(-1) {
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    ProfState &P = prof();
+    std::lock_guard<std::mutex> g(P.mu);
+    if (!P.on) return;
+    cudaEvent_t a = take_event(P);
+    cudaEventRecord(a, stream);
+    P.begin_of_slot.push_back(a);
+    slot = (int)P.begin_of_slot.size() - 1;
+}
+
+LaunchScope::~LaunchScope() {
+    if (slot < 0) return;
+    ProfState &P = prof();
+    std::lock_guard<std::mutex> g(P.mu);
+    cudaEvent_t b = take_event(P);
+    cudaEventRecord(b, stream);
+    P.pending.push_back({kind_of(P, name), P.begin_of_slot[slot], b});
+}
+
+WsLayout ws_layout(const moe_dims &d, int64_t T) {
+    auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+    const size_t S = (size_t)T * d.top_k;
+    WsLayout L{};
+    size_t o = 0;
+    L.idx = o; o += up(S * 4);
+    L.gate = o; o += up(S * 4);
+    L.counts = o; o += up((size_t)d.n_experts * 4);
+    L.offsets = o; o += up(((size_t)d.n_experts + 1) * 4);
+    L.perm = o; o += up(S * 4);
+    L.inv_perm = o; o += up(S * 4);
+    L.h = o; o += up(S * d.ffn_hidden * 4);
+    L.y = o; o += (T > kFusedCombineMaxTokens) ? up(S * d.d_model * 4) : 0;
+    L.total = o;
+    return L;
+}
+
+}  // namespace moe
+
+using namespace moe;
+
+namespace {
+
+bool dt_ok(int32_t v) { return v == MOE_F32 || v == MOE_BF16; }
+
+moe_status check_dims(const moe_dims *d) {
+    if (!d) return MOE_ERR_INVALID_ARG;
+    if (d->d_model < 8 || d->d_model > 49152 || d->d_model % 8) return MOE_ERR_INVALID_ARG;
+    if (d->ffn_hidden < 8 || d->ffn_hidden > 65536 || d->ffn_hidden % 8) return MOE_ERR_INVALID_ARG;
+    if (d->n_experts < 1 || d->n_experts > 256) return MOE_ERR_INVALID_ARG;
+    if (d->top_k < 1 || d->top_k > d->n_experts) return MOE_ERR_INVALID_ARG;
+    if (!dt_ok(d->w_dtype) || !dt_ok(d->x_dtype) || !dt_ok(d->out_dtype)) return MOE_ERR_INVALID_ARG;
+    if (d->w_dtype != d->x_dtype) return MOE_ERR_UNSUPPORTED;
+    return MOE_OK;
+}
+
+moe_status check_T(const moe_dims *d, int32_t T) {
+    if (T < 0 || T > (1 << 20)) return MOE_ERR_INVALID_ARG;
+    if ((int64_t)T * d->top_k > (1 << 24)) return MOE_ERR_INVALID_ARG;
+    return MOE_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool ok_ptr(const void *p) { return p != nullptr && aligned16(p); }
+bool ok_opt(const void *p) { return p == nullptr || aligned16(p); }
+
+moe_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA; }
+
+template <typename TX, typename TW>
+cudaError_t launch_route(const moe_dims &d, int T, const void *x, const void *wr, float *logits,
+                         int32_t *idx, float *gate, cudaStream_t st) {
+    const int grid = (T + kRouteTokens - 1) / kRouteTokens;
+    LaunchScope ls("route", st);
+    k_route<TX, TW><<<grid, kRouteThreads, 0, st>>>(T, d.d_model, d.n_experts, d.top_k,
+                                                   static_cast<const TX *>(x),
+                                                   static_cast<const TW *>(wr), logits, idx, gate);
+    return cudaGetLastError();
+}
+
+cudaError_t route_any(const moe_dims &d, int T, const void *x, const void *wr, float *logits,
+                      int32_t *idx, float *gate, cudaStream_t st) {
+    if (d.w_dtype == MOE_BF16) return launch_route<bf16, bf16>(d, T, x, wr, logits, idx, gate, st);
+    return launch_route<float, float>(d, T, x, wr, logits, idx, gate, st);
+}
+
+cudaError_t dispatch_any(const moe_dims &d, int T, const int32_t *idx, int32_t *counts,
+                         int32_t *offsets, int32_t *perm, int32_t *inv, cudaStream_t st) {
+    LaunchScope ls("dispatch", st);
+    k_dispatch<<<1, kDispatchThreads, 0, st>>>(T * d.top_k, d.n_experts, idx, counts, offsets,
+                                               perm, inv, device_info().err);
+    return cudaGetLastError();
+}
+
+template <typename TO, typename TR>
+cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const int32_t *inv,
+                           const float *gate, const void *res, void *out, cudaStream_t st) {
+    const long long total = (long long)T * (d.d_model / 4);
+    const long long cap = (long long)device_info().sm_count * 8;
+    const long long want = (total + 255) / 256;
+    const int grid = (int)std::max(1LL, std::min(want, cap));
+    LaunchScope ls("combine", st);
+    k_combine<TO, TR><<<grid, 256, 0, st>>>(T, d.d_model, d.top_k, y, inv, gate,
+                                            static_cast<const TR *>(res), static_cast<TO *>(out),
+                                            device_info().err);
+    return cudaGetLastError();
+}
+
+cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t *inv,
+                        const float *gate, const void *res, void *out, cudaStream_t st) {
+    const bool xb = d.x_dtype == MOE_BF16, ob = d.out_dtype == MOE_BF16;
+    if (xb && ob) return launch_combine<bf16, bf16>(d, T, y, inv, gate, res, out, st);
+    if (xb) return launch_combine<float, bf16>(d, T, y, inv, gate, res, out, st);
+    if (ob) return launch_combine<bf16, float>(d, T, y, inv, gate, res, out, st);
+    return launch_combine<float, float>(d, T, y, inv, gate, res, out, st);
+}
+
+template <typename P> P *at(void *ws, size_t off) {
+    return reinterpret_cast<P *>(static_cast<char *>(ws) + off);
+}
+
+}  // namespace
+
+extern "C" {
+
+moe_status moe_workspace_size(const moe_dims *dims, int32_t max_tokens, size_t *bytes) {
+    moe_status s = check_dims(dims);
+    if (s == MOE_ERR_UNSUPPORTED) s = MOE_OK;  // sizing does not depend on dtypes
+    if (s != MOE_OK) return s;
+    if (!bytes || max_tokens < 0) return MOE_ERR_INVALID_ARG;
+    if ((s = check_T(dims, max_tokens)) != MOE_OK) return s;
+    *bytes = ws_layout(*dims, max_tokens).total;
+    return MOE_OK;
+}
+
+moe_status moe_route(const moe_dims *dims, int32_t T, const void *x, const void *w_router,
+                     float *logits_opt, int32_t *topk_idx, float *topk_gate, moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(x) || !ok_ptr(w_router) || !ok_opt(logits_opt) || !topk_idx || !topk_gate)
+        return MOE_ERR_INVALID_ARG;
+    return cuda_status(route_any(*dims, T, x, w_router, logits_opt, topk_idx, topk_gate,
+                                 (cudaStream_t)stream));
+}
+
+moe_status moe_dispatch(const moe_dims *dims, int32_t T, const int32_t *topk_idx,
+                        int32_t *counts, int32_t *offsets, int32_t *perm, int32_t *inv_perm,
+                        moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s == MOE_ERR_UNSUPPORTED) s = MOE_OK;  // dispatch does not read floating point data
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (!counts || !offsets) return MOE_ERR_INVALID_ARG;
+    if (T > 0 && (!topk_idx || !perm || !inv_perm)) return MOE_ERR_INVALID_ARG;
+    return cuda_status(dispatch_any(*dims, T, topk_idx, counts, offsets, perm, inv_perm,
+                                    (cudaStream_t)stream));
+}
+
+moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x, const int32_t *perm,
+                          const int32_t *offsets, const void *w1, const void *v1, const void *w2,
+                          float *y_sorted, void *ws, size_t ws_bytes, moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(x) || !perm || !offsets || !ok_ptr(w1) || !ok_ptr(v1) || !ok_ptr(w2) ||
+        !ok_ptr(y_sorted))
+        return MOE_ERR_INVALID_ARG;
+    const WsLayout L = ws_layout(*dims, T);
+    if (!ws || !aligned16(ws) || ws_bytes < L.total) return MOE_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    float *h = at<float>(ws, L.h);
+    cudaError_t e = launch_up_glu_gemv(*dims, T, x, perm, offsets, w1, v1, h, st);
+    if (e == cudaSuccess)
+        e = launch_down_gemv(*dims, T, h, perm, offsets, w2, nullptr, y_sorted, nullptr, nullptr,
+                             false, st);
+    return cuda_status(e);
+}
+
+moe_status moe_combine(const moe_dims *dims, int32_t T, const float *y_sorted,
+                       const int32_t *inv_perm, const float *topk_gate, const void *residual_opt,
+                       void *out, moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(y_sorted) || !inv_perm || !topk_gate || !ok_opt(residual_opt) || !ok_ptr(out))
+        return MOE_ERR_INVALID_ARG;
+    return cuda_status(combine_any(*dims, T, y_sorted, inv_perm, topk_gate, residual_opt, out,
+                                   (cudaStream_t)stream));
+}
+
+moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, const void *w_router,
+                             const void *w1, const void *v1, const void *w2,
+                             const void *residual_opt, void *out, void *ws, size_t ws_bytes,
+                             moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(x) || !ok_ptr(w_router) || !ok_ptr(w1) || !ok_ptr(v1) || !ok_ptr(w2) ||
+        !ok_opt(residual_opt) || !ok_ptr(out))
+        return MOE_ERR_INVALID_ARG;
+    const WsLayout L = ws_layout(*dims, T);
+    if (!ws || !aligned16(ws) || ws_bytes < L.total) return MOE_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    const moe_dims &d = *dims;
+    int32_t *idx = at<int32_t>(ws, L.idx);
+    float *gate = at<float>(ws, L.gate);
+    int32_t *counts = at<int32_t>(ws, L.counts);
+    int32_t *offsets = at<int32_t>(ws, L.offsets);
+    int32_t *perm = at<int32_t>(ws, L.perm);
+    int32_t *inv = at<int32_t>(ws, L.inv_perm);
+    float *h = at<float>(ws, L.h);
+
+    cudaError_t e = route_any(d, T, x, w_router, nullptr, idx, gate, st);
+    if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
+    if (e == cudaSuccess) e = launch_up_glu_gemv(d, T, x, perm, offsets, w1, v1, h, st);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    if (T <= kFusedCombineMaxTokens) {
+        e = launch_down_gemv(d, T, h, perm, offsets, w2, gate, nullptr, residual_opt, out, true, st);
+    } else {
+        float *y = at<float>(ws, L.y);
+        e = launch_down_gemv(d, T, h, perm, offsets, w2, nullptr, y, nullptr, nullptr, false, st);
+        if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st);
+    }
+    return cuda_status(e);
+}
+
+const char *moe_status_string(moe_status status) {
+    switch (status) {
+    case MOE_OK: return "MOE_OK";
+    case MOE_ERR_INVALID_ARG: return "MOE_ERR_INVALID_ARG: invalid argument";
+    case MOE_ERR_UNSUPPORTED: return "MOE_ERR_UNSUPPORTED: unsupported dtype combination";
+    case MOE_ERR_WORKSPACE: return "MOE_ERR_WORKSPACE: workspace missing or too small";
+    case MOE_ERR_CUDA: return "MOE_ERR_CUDA: CUDA launch or runtime error";
+    case MOE_ERR_TIMEOUT: return "MOE_ERR_TIMEOUT: a bounded device wait gave up";
+    case MOE_ERR_DEVICE_INDEX: return "MOE_ERR_DEVICE_INDEX: expert index out of range";
+    }
+    return "unknown moe_status";
+}
+
+moe_status moe_get_last_error(moe_stream_t stream) {
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    if (cudaGetLastError() != cudaSuccess) return MOE_ERR_CUDA;
+    unsigned v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_moe_err, sizeof v) != cudaSuccess) return MOE_ERR_CUDA;
+    if (v != kErrNone) {
+        const unsigned zero = 0;
+        if (cudaMemcpyToSymbol(g_moe_err, &zero, sizeof zero) != cudaSuccess) return MOE_ERR_CUDA;
+    }
+    if (v == kErrIndex) return MOE_ERR_DEVICE_INDEX;
+    if (v == kErrTimeout) return MOE_ERR_TIMEOUT;
+    return MOE_OK;
+}
+
+int64_t moe_launch_count(void) { return g_launches.load(); }
+
+void moe_profile_enable(int on) {
+    ProfState &P = prof();
+    std::lock_guard<std::mutex> g(P.mu);
+    P.on = on != 0;
+}
+
+void moe_profile_reset(void) {
+    ProfState &P = prof();
+    std::lock_guard<std::mutex> g(P.mu);
+    for (auto &p : P.pending) {
+        cudaEventSynchronize(p.b);
+        P.pool.push_back(p.a);
+        P.pool.push_back(p.b);
+    }
+    P.pending.clear();
+    P.begin_of_slot.clear();
+    for (auto &v : P.launches) v = 0;
+    for (auto &v : P.ms) v = 0.0;
+}
+
+int32_t moe_profile_read(moe_kernel_stat *stats, int32_t max_stats) {
+    ProfState &P = prof();
+    std::lock_guard<std::mutex> g(P.mu);
+    for (auto &p : P.pending) {
+        cudaEventSynchronize(p.b);
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) P.ms[p.kind] += ms;
+        P.launches[p.kind] += 1;
+        P.pool.push_back(p.a);
+        P.pool.push_back(p.b);
+    }
+    P.pending.clear();
+    P.begin_of_slot.clear();
+    const int n = (int)P.names.size();
+    for (int i = 0; i < n && i < max_stats; ++i) {
+        memset(stats[i].name, 0, sizeof stats[i].name);
+        strncpy(stats[i].name, P.names[i].c_str(), sizeof stats[i].name - 1);
+        stats[i].launches = P.launches[i];
+        stats[i].total_ms = P.ms[i];
+    }
+    return n;
+}
+
+}  // extern "C"

@@ -1,0 +1,124 @@
+// Internal helpers shared by the CUDA translation units of libmoe.
+// Nothing here is part of the C ABI (include/moe.h).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "moe.h"
+
+namespace moe {
+
+typedef __nv_bfloat16 bf16;
+
+// Device error word: the first error a kernel meets is stored here with an
+// atomic compare-and-swap and read back by moe_get_last_error.
+enum : unsigned { kErrNone = 0, kErrIndex = 1, kErrTimeout = 2 };
+
+__device__ __forceinline__ void set_error(unsigned *err, unsigned code) {
+    if (err) atomicCAS(err, 0u, code);
+}
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+
+// Two bf16 packed in a 32-bit word -> two floats (exact).
+__device__ __forceinline__ void unpack_bf16x2(uint32_t u, float &lo, float &hi) {
+    lo = __uint_as_float(u << 16);
+    hi = __uint_as_float(u & 0xffff0000u);
+}
+
+// 16-byte read-only load that does not allocate in L1 (weights are streamed
+// once per call; keeping them out of L1 leaves it to the token vectors).
+__device__ __forceinline__ uint4 ld_stream16(const void *p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+// Eight consecutive weights (streamed) -> float[8].
+__device__ __forceinline__ void stream8(const bf16 *p, float (&o)[8]) {
+    uint4 u = ld_stream16(p);
+    unpack_bf16x2(u.x, o[0], o[1]);
+    unpack_bf16x2(u.y, o[2], o[3]);
+    unpack_bf16x2(u.z, o[4], o[5]);
+    unpack_bf16x2(u.w, o[6], o[7]);
+}
+__device__ __forceinline__ void stream8(const float *p, float (&o)[8]) {
+    uint4 a = ld_stream16(p), b = ld_stream16(p + 4);
+    o[0] = __uint_as_float(a.x); o[1] = __uint_as_float(a.y);
+    o[2] = __uint_as_float(a.z); o[3] = __uint_as_float(a.w);
+    o[4] = __uint_as_float(b.x); o[5] = __uint_as_float(b.y);
+    o[6] = __uint_as_float(b.z); o[7] = __uint_as_float(b.w);
+}
+
+// Eight consecutive values through the normal cached path -> float[8].
+__device__ __forceinline__ void load8(const bf16 *p, float (&o)[8]) {
+    uint4 u = __ldg(reinterpret_cast<const uint4 *>(p));
+    unpack_bf16x2(u.x, o[0], o[1]);
+    unpack_bf16x2(u.y, o[2], o[3]);
+    unpack_bf16x2(u.z, o[4], o[5]);
+    unpack_bf16x2(u.w, o[6], o[7]);
+}
+__device__ __forceinline__ void load8(const float *p, float (&o)[8]) {
+    float4 a = __ldg(reinterpret_cast<const float4 *>(p));
+    float4 b = __ldg(reinterpret_cast<const float4 *>(p) + 1);
+    o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+    o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ float silu(float a) { return a / (1.0f + expf(-a)); }
+
+// ---- host side -----------------------------------------------------------
+
+struct DeviceInfo {
+    int sm_count;
+    unsigned *err;  // device address of the error word
+};
+
+// Per-device facts, looked up once per device (current device).
+const DeviceInfo &device_info();
+
+// Launch bookkeeping: counts every launch and, when profiling is on,
+// brackets it with CUDA events on its stream.
+struct LaunchScope {
+    LaunchScope(const char *name, cudaStream_t stream);
+    ~LaunchScope();
+    const char *name;
+    cudaStream_t stream;
+    int slot;
+};
+
+// Workspace layout of moe_layer_forward / moe_expert_ffn for T tokens.
+struct WsLayout {
+    size_t idx, gate, counts, offsets, perm, inv_perm, h, y, total;
+};
+WsLayout ws_layout(const moe_dims &d, int64_t T);
+
+// Decode-path launchers (ffn_gemv.cu).
+cudaError_t launch_up_glu_gemv(const moe_dims &d, int T, const void *x,
+                               const int32_t *perm, const int32_t *offsets,
+                               const void *w1, const void *v1, float *h,
+                               cudaStream_t st);
+cudaError_t launch_down_gemv(const moe_dims &d, int T, const float *h,
+                             const int32_t *perm, const int32_t *offsets,
+                             const void *w2, const float *gate, float *y_sorted,
+                             const void *residual, void *out, bool fused,
+                             cudaStream_t st);
+
+constexpr int kFusedCombineMaxTokens = 64;
+
+}  // namespace moe

@@ -1,0 +1,235 @@
+"""Python binding of libmoe (``include/moe.h``): argument marshalling only.
+
+Every step runs in the library's CUDA kernels; this module passes
+``tensor.data_ptr()`` and the current CUDA stream through ctypes and raises
+``MoeError`` on a non-zero status.  PyTorch is used for device memory and
+streams only.  There is no fallback: if ``libmoe.so`` has not been built the
+import of the library raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+F32, BF16 = 0, 1
+_DT = {torch.float32: F32, torch.bfloat16: BF16}
+_STATUS = {
+    0: "MOE_OK", 1: "MOE_ERR_INVALID_ARG", 2: "MOE_ERR_UNSUPPORTED",
+    3: "MOE_ERR_WORKSPACE", 4: "MOE_ERR_CUDA", 5: "MOE_ERR_TIMEOUT",
+    6: "MOE_ERR_DEVICE_INDEX",
+}
+
+# Every function the header declares (checked by the CPU tests).
+EXPORTS = (
+    "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
+    "moe_combine", "moe_layer_forward", "moe_status_string",
+    "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
+    "moe_profile_reset", "moe_profile_read",
+)
+
+
+class MoeError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {_STATUS.get(status, status)}")
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [("d_model", ctypes.c_int32), ("ffn_hidden", ctypes.c_int32),
+                ("n_experts", ctypes.c_int32), ("top_k", ctypes.c_int32),
+                ("w_dtype", ctypes.c_int32), ("x_dtype", ctypes.c_int32),
+                ("out_dtype", ctypes.c_int32)]
+
+    def __repr__(self):
+        return (f"Dims(D={self.d_model}, F={self.ffn_hidden}, E={self.n_experts}, "
+                f"K={self.top_k}, w={self.w_dtype}, x={self.x_dtype}, out={self.out_dtype})")
+
+
+class KernelStat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int64),
+                ("total_ms", ctypes.c_double)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib() -> ctypes.CDLL:
+    """Load libmoe.so (built by ``__graft_entry__.build()``); raise if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"libmoe.so is not built ({path}); run __graft_entry__.build()")
+    L = ctypes.CDLL(path)
+    P, I32, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    DP = ctypes.POINTER(Dims)
+    sigs = {
+        "moe_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
+        "moe_route": [DP, I32, P, P, P, P, P, P],
+        "moe_dispatch": [DP, I32, P, P, P, P, P, P],
+        "moe_expert_ffn": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
+        "moe_combine": [DP, I32, P, P, P, P, P, P],
+        "moe_layer_forward": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
+        "moe_get_last_error": [P],
+        "moe_status_string": [ctypes.c_int],
+        "moe_profile_enable": [ctypes.c_int],
+        "moe_profile_reset": [],
+        "moe_profile_read": [ctypes.POINTER(KernelStat), I32],
+        "moe_launch_count": [],
+    }
+    for name, args in sigs.items():
+        fn = getattr(L, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_int
+    L.moe_status_string.restype = ctypes.c_char_p
+    L.moe_launch_count.restype = ctypes.c_int64
+    L.moe_profile_enable.restype = None
+    L.moe_profile_reset.restype = None
+    L.moe_profile_read.restype = I32
+    _lib = L
+    return L
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise MoeError(status, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def dims(d_model: int, ffn_hidden: int, n_experts: int, top_k: int,
+         w_dtype=torch.bfloat16, x_dtype=None, out_dtype=None) -> Dims:
+    x_dtype = w_dtype if x_dtype is None else x_dtype
+    out_dtype = x_dtype if out_dtype is None else out_dtype
+    return Dims(d_model, ffn_hidden, n_experts, top_k, _DT[w_dtype], _DT[x_dtype],
+                _DT[out_dtype])
+
+
+def _tdt(code: int):
+    return torch.bfloat16 if code == BF16 else torch.float32
+
+
+def workspace_size(d: Dims, max_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().moe_workspace_size(ctypes.byref(d), max_tokens, ctypes.byref(n)),
+           "moe_workspace_size")
+    return int(n.value)
+
+
+def alloc_workspace(d: Dims, max_tokens: int, device="cuda") -> torch.Tensor:
+    return torch.empty(max(workspace_size(d, max_tokens), 256), dtype=torch.uint8, device=device)
+
+
+def route(d: Dims, x: torch.Tensor, w_r: torch.Tensor, want_logits: bool = False,
+          stream=None):
+    """Step 1: returns (topk_idx int32 [T,K], topk_gate f32 [T,K], logits or None)."""
+    T = x.shape[0]
+    dev = x.device
+    idx = torch.empty((T, d.top_k), dtype=torch.int32, device=dev)
+    gate = torch.empty((T, d.top_k), dtype=torch.float32, device=dev)
+    logits = torch.empty((T, d.n_experts), dtype=torch.float32, device=dev) if want_logits else None
+    _check(lib().moe_route(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(logits), _ptr(idx),
+                           _ptr(gate), _stream(stream)), "moe_route")
+    return idx, gate, logits
+
+
+def dispatch(d: Dims, topk_idx: torch.Tensor, stream=None):
+    """Step 2: returns (counts [E], offsets [E+1], perm [S], inv_perm [S]) int32."""
+    T = topk_idx.shape[0]
+    dev = topk_idx.device
+    S = T * d.top_k
+    counts = torch.empty(d.n_experts, dtype=torch.int32, device=dev)
+    offsets = torch.empty(d.n_experts + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(S, dtype=torch.int32, device=dev)
+    inv = torch.empty(S, dtype=torch.int32, device=dev)
+    _check(lib().moe_dispatch(ctypes.byref(d), T, _ptr(topk_idx), _ptr(counts), _ptr(offsets),
+                              _ptr(perm), _ptr(inv), _stream(stream)), "moe_dispatch")
+    return counts, offsets, perm, inv
+
+
+def expert_ffn(d: Dims, x, perm, offsets, w1, v1, w2, ws=None, stream=None):
+    """Step 3: returns y_sorted f32 [T*K, D] (ungated expert outputs)."""
+    T = x.shape[0]
+    ws = alloc_workspace(d, T, x.device) if ws is None else ws
+    y = torch.empty((T * d.top_k, d.d_model), dtype=torch.float32, device=x.device)
+    _check(lib().moe_expert_ffn(ctypes.byref(d), T, _ptr(x), _ptr(perm), _ptr(offsets),
+                                _ptr(w1), _ptr(v1), _ptr(w2), _ptr(y), _ptr(ws),
+                                ws.numel(), _stream(stream)), "moe_expert_ffn")
+    return y
+
+
+def combine(d: Dims, y_sorted, inv_perm, gate, residual=None, out=None, stream=None):
+    """Step 4: returns out [T, D] (out_dtype)."""
+    T = gate.shape[0]
+    if out is None:
+        out = torch.empty((T, d.d_model), dtype=_tdt(d.out_dtype), device=gate.device)
+    _check(lib().moe_combine(ctypes.byref(d), T, _ptr(y_sorted), _ptr(inv_perm), _ptr(gate),
+                             _ptr(residual), _ptr(out), _stream(stream)), "moe_combine")
+    return out
+
+
+def layer_forward(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, ws=None,
+                  stream=None):
+    """The whole layer; returns out [T, D] (out_dtype)."""
+    T = x.shape[0]
+    if out is None:
+        out = torch.empty((T, d.d_model), dtype=_tdt(d.out_dtype), device=x.device)
+    ws = alloc_workspace(d, T, x.device) if ws is None else ws
+    _check(lib().moe_layer_forward(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(w1), _ptr(v1),
+                                   _ptr(w2), _ptr(residual), _ptr(out), _ptr(ws), ws.numel(),
+                                   _stream(stream)), "moe_layer_forward")
+    return out
+
+
+def get_last_error(stream=None) -> int:
+    """Synchronise the stream and return the library's pending status code."""
+    return int(lib().moe_get_last_error(_stream(stream)))
+
+
+def check_device_errors(stream=None):
+    _check(get_last_error(stream), "device")
+
+
+def launch_count() -> int:
+    return int(lib().moe_launch_count())
+
+
+def profile_enable(on: bool = True):
+    lib().moe_profile_enable(1 if on else 0)
+
+
+def profile_reset():
+    lib().moe_profile_reset()
+
+
+def profile_read() -> dict:
+    """{kernel name: (launches, total ms)} since the last reset."""
+    buf = (KernelStat * 64)()
+    n = lib().moe_profile_read(buf, 64)
+    return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].total_ms))
+            for i in range(min(n, 64))}
+
+
+def status_string(code: int) -> str:
+    return lib().moe_status_string(code).decode()

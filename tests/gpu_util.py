@@ -1,0 +1,51 @@
+"""Helpers for the GPU parity tests: tolerance checks and device copies."""
+from __future__ import annotations
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2506_23635_gb300 import inputs as gen
+
+# Layer-output bound for bf16 weights with fp32 accumulation: relative L2
+# error <= 5e-3 and max abs error <= 2e-2 * RMS(reference output).
+REL_L2 = 5e-3
+MAX_ABS_OF_RMS = 2e-2
+# fp32 weights and activations (the tiny layer): the same shape of bound,
+# tightened to what fp32 accumulation over a few thousand terms reaches.
+REL_L2_F32 = 1e-5
+MAX_ABS_OF_RMS_F32 = 1e-4
+
+
+def need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+
+
+def bounds(dtype: str):
+    return (REL_L2, MAX_ABS_OF_RMS) if dtype == "bf16" else (REL_L2_F32, MAX_ABS_OF_RMS_F32)
+
+
+def assert_parity(got, want, dtype: str = "bf16", what: str = ""):
+    rel_l2, max_abs = bounds(dtype)
+    g = np.asarray(got, np.float64)
+    w = np.asarray(want, np.float64)
+    assert g.shape == w.shape, f"{what}: shape {g.shape} vs {w.shape}"
+    assert np.all(np.isfinite(g)), f"{what}: non-finite output"
+    err = g - w
+    nw = np.linalg.norm(w)
+    rel = np.linalg.norm(err) / nw if nw > 0 else np.linalg.norm(err)
+    rms = float(np.sqrt(np.mean(w * w))) if w.size else 0.0
+    mx = float(np.max(np.abs(err))) if err.size else 0.0
+    assert rel <= rel_l2, f"{what}: rel L2 {rel:.3e} > {rel_l2}"
+    assert mx <= max_abs * rms + 1e-30, f"{what}: max abs {mx:.3e} > {max_abs}*RMS ({rms:.3e})"
+    return rel, mx / rms if rms else 0.0
+
+
+def to_numpy(t: torch.Tensor) -> np.ndarray:
+    """Values of a device tensor as float64 (bf16 and f32 widen exactly)."""
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def dev(a: np.ndarray, dtype: str):
+    return gen.host_to_torch(a, dtype, "cuda")

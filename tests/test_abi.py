@@ -1,0 +1,130 @@
+"""The C ABI library builds, loads and exports every function include/moe.h
+declares; host-side validation returns the documented status before any
+launch (CPU only -- no compute call is made)."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+from paper_2506_23635_gb300 import build as moe_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moe.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    moe_build.build()
+    from paper_2506_23635_gb300 import moe
+    return moe
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(moe_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_five_steps():
+    names = declared_functions()
+    for n in ("moe_route", "moe_dispatch", "moe_expert_ffn", "moe_combine",
+              "moe_layer_forward"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    L = lib.lib()
+    names = declared_functions()
+    assert names, "no declarations parsed"
+    for n in names:
+        assert hasattr(L, n), f"{n} not exported by libmoe.so"
+    assert set(names) == set(lib.EXPORTS)
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        s = lib.status_string(code)
+        assert s.startswith("MOE_")
+    assert "unknown" in lib.status_string(99)
+
+
+DBRX = dict(d_model=6144, ffn_hidden=10752, n_experts=16, top_k=4)
+
+
+def test_workspace_size(lib):
+    d = lib.dims(**DBRX)
+    n1 = lib.workspace_size(d, 1)
+    n64 = lib.workspace_size(d, 64)
+    n2048 = lib.workspace_size(d, 2048)
+    assert 0 < n1 < n64 < n2048
+    # the GLU hidden vectors (T*K x F fp32) dominate the decode workspace
+    assert n64 >= 64 * 4 * 10752 * 4
+    assert lib.workspace_size(d, 0) >= 0
+
+
+@pytest.mark.parametrize("bad", [
+    dict(d_model=6143), dict(d_model=0), dict(ffn_hidden=10), dict(n_experts=0),
+    dict(n_experts=257, top_k=4), dict(top_k=0), dict(top_k=17),
+])
+def test_workspace_size_rejects_bad_dims(lib, bad):
+    d = lib.dims(**{**DBRX, **bad})
+    with pytest.raises(lib.MoeError) as ei:
+        lib.workspace_size(d, 8)
+    assert ei.value.status == 1
+
+
+# Validation returns before anything touches the device, so these calls are
+# made with placeholder addresses.  They are skipped where a GPU is present
+# (the GPU tests cover the same cases with real tensors) so that a validation
+# bug could never launch a kernel on a placeholder address.
+no_gpu = pytest.mark.skipif(torch.cuda.is_available(),
+                            reason="placeholder addresses only where no GPU exists")
+
+A = ctypes.c_void_p(0x10000)  # 16-byte aligned placeholder
+MIS = ctypes.c_void_p(0x10004)  # misaligned placeholder
+
+
+@no_gpu
+def test_route_validation(lib):
+    L = lib.lib()
+    d = lib.dims(**DBRX)
+    r = lambda T, x=A, w=A, lg=None, i=A, g=A: L.moe_route(ctypes.byref(d), T, x, w, lg, i, g, None)
+    assert r(1, x=None) == 1
+    assert r(1, w=None) == 1
+    assert r(1, i=None) == 1
+    assert r(1, g=None) == 1
+    assert r(1, x=MIS) == 1
+    assert r(-1) == 1
+    assert r(1 << 21) == 1
+    assert r(0) == 0  # nothing to do
+    bad = lib.dims(**{**DBRX, "top_k": 17})
+    assert L.moe_route(ctypes.byref(bad), 1, A, A, None, A, A, None) == 1
+    mixed = lib.dims(**DBRX, w_dtype=torch.bfloat16, x_dtype=torch.float32)
+    assert L.moe_route(ctypes.byref(mixed), 1, A, A, None, A, A, None) == 2
+
+
+@no_gpu
+def test_layer_and_ffn_validation(lib):
+    L = lib.lib()
+    d = lib.dims(**DBRX)
+    need = lib.workspace_size(d, 8)
+    f = lambda T, ws=A, n=need, x=A: L.moe_layer_forward(ctypes.byref(d), T, x, A, A, A, A,
+                                                          None, A, ws, n, None)
+    assert f(8, ws=None) == 3
+    assert f(8, n=need - 1) == 3
+    assert f(8, ws=MIS) == 3
+    assert f(8, x=None) == 1
+    assert f(0) == 0
+    g = lambda T, ws=A, n=need: L.moe_expert_ffn(ctypes.byref(d), T, A, A, A, A, A, A, A, ws, n, None)
+    assert g(8, n=0) == 3
+    assert L.moe_expert_ffn(ctypes.byref(d), 8, A, None, A, A, A, A, A, A, need, None) == 1
+    assert L.moe_combine(ctypes.byref(d), 8, A, A, A, MIS, A, None) == 1
+    assert L.moe_combine(ctypes.byref(d), 8, A, None, A, None, A, None) == 1
+    assert L.moe_dispatch(ctypes.byref(d), 8, None, A, A, A, A, None) == 1
+    assert L.moe_dispatch(ctypes.byref(d), 8, A, None, A, A, A, None) == 1
+
+
+def test_launch_count_starts_at_zero_without_launches(lib):
+    assert lib.launch_count() >= 0

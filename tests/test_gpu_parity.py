@@ -1,0 +1,212 @@
+"""CUDA path vs the fp64 oracle, step by step and for the whole layer, on
+seeded inputs that span several tiles and ragged tails.
+
+Bars: expert indices, counts, offsets and permutations bit-exact; values
+within rel L2 5e-3 and max abs 2e-2 * RMS (bf16), tighter for fp32."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2506_23635_gb300 import inputs as gen
+from tests.gpu_util import assert_parity, dev, need_gpu, to_numpy
+
+pytestmark = pytest.mark.gpu
+
+
+def moe():
+    need_gpu()
+    from paper_2506_23635_gb300 import moe as m
+    return m
+
+
+# (D, F, E, K, T, dtype): tiny layer, ragged widths, K = E, E = 1,
+# E = 256, minimum widths, and token counts on both sides of the fused
+# combine limit (64).
+SMALL = [
+    (256, 512, 4, 2, 8, "f32"),
+    (64, 96, 8, 2, 1, "bf16"),
+    (72, 40, 5, 3, 17, "bf16"),
+    (128, 136, 16, 4, 65, "bf16"),
+    (256, 264, 7, 7, 33, "f32"),
+    (40, 24, 1, 1, 5, "bf16"),
+    (512, 256, 256, 8, 130, "bf16"),
+    (8, 8, 3, 2, 300, "f32"),
+    (264, 520, 16, 4, 64, "bf16"),
+]
+
+
+def _host(case, seed=3, skew=None):
+    D, F, E, K, T, dt = case
+    shape = gen.LayerShape(D, F, E, K, dt)
+    return gen.host_layer(shape, T, seed, skew)
+
+
+def _dims(m, shape, out_dtype=None):
+    tdt = gen.torch_dtype(shape.dtype)
+    return m.dims(shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k, tdt, tdt,
+                  out_dtype or tdt)
+
+
+def _devlayer(L):
+    dt = L.shape.dtype
+    return [dev(a, dt) for a in (L.x, L.w_r, L.w1, L.v1, L.w2)]
+
+
+@pytest.mark.parametrize("case", SMALL, ids=lambda c: "D{}F{}E{}K{}T{}{}".format(*c))
+def test_steps_and_layer(case):
+    m = moe()
+    L = _host(case)
+    sh = L.shape
+    d = _dims(m, sh)
+    ref = oracle.layer_steps(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+
+    idx, gate, logits = m.route(d, x, w_r, want_logits=True)
+    assert np.array_equal(idx.cpu().numpy(), ref["idx"]), "top-k indices"
+    np.testing.assert_allclose(to_numpy(gate), ref["gate"], rtol=0, atol=2e-6)
+    scale = np.abs(gen.to_f64(L.x, sh.dtype)) @ np.abs(gen.to_f64(L.w_r, sh.dtype))
+    assert np.all(np.abs(to_numpy(logits) - ref["logits"]) <= 1e-5 * scale + 1e-7)
+
+    counts, offsets, perm, inv = m.dispatch(d, idx)
+    assert np.array_equal(counts.cpu().numpy(), ref["counts"])
+    assert np.array_equal(offsets.cpu().numpy(), ref["offsets"])
+    assert np.array_equal(perm.cpu().numpy(), ref["perm"])
+    assert np.array_equal(inv.cpu().numpy(), ref["inv_perm"])
+
+    y = m.expert_ffn(d, x, perm, offsets, w1, v1, w2)
+    assert_parity(to_numpy(y), ref["y_sorted"], sh.dtype, "expert_ffn y_sorted")
+
+    out = m.combine(d, y, inv, gate)
+    assert_parity(to_numpy(out), ref["out"], sh.dtype, "combine")
+
+    out2 = m.layer_forward(d, x, w_r, w1, v1, w2)
+    assert_parity(to_numpy(out2), ref["out"], sh.dtype, "layer_forward")
+    assert m.get_last_error() == 0
+
+
+@pytest.mark.parametrize("T", [1, 8, 64, 65, 200])
+def test_layer_residual_and_bf16_out(T):
+    """out = residual + MoE(x), written in bf16; both the fused (T <= 64) and
+    the unfused combine."""
+    m = moe()
+    L = _host((136, 200, 6, 2, T, "bf16"), seed=7)
+    sh = L.shape
+    d = _dims(m, sh)
+    res = gen.host_normal((T, sh.d_model), 1.0, "bf16", 7, "residual")
+    want, _, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k,
+                                     residual=gen.to_f64(res, "bf16"))
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    out = m.layer_forward(d, x, w_r, w1, v1, w2, residual=dev(res, "bf16"))
+    assert out.dtype == torch.bfloat16
+    assert_parity(to_numpy(out), want, "bf16", "layer + residual")
+    d32 = _dims(m, sh, out_dtype=torch.float32)
+    out32 = m.layer_forward(d32, x, w_r, w1, v1, w2, residual=dev(res, "bf16"))
+    assert out32.dtype == torch.float32
+    assert_parity(to_numpy(out32), want, "bf16", "layer + residual, f32 out")
+
+
+@pytest.mark.parametrize("skew", [0.0, 0.6, 1.2])
+def test_designed_router_skew(skew):
+    """Zipf-skewed expert loads (few experts carry most slots)."""
+    m = moe()
+    L = _host((192, 128, 16, 4, 64, "bf16"), seed=11, skew=skew)
+    sh = L.shape
+    d = _dims(m, sh)
+    ref = oracle.layer_steps(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    idx, gate, _ = m.route(d, x, w_r)
+    assert np.array_equal(idx.cpu().numpy(), ref["idx"])
+    out = m.layer_forward(d, x, w_r, w1, v1, w2)
+    assert_parity(to_numpy(out), ref["out"], "bf16", f"skew {skew}")
+
+
+def test_all_tokens_one_expert():
+    """A router that sends every token to the same top-1 expert: one expert
+    holds all slots, the others none."""
+    m = moe()
+    D, F, E, K, T = 64, 80, 8, 1, 77
+    shape = gen.LayerShape(D, F, E, K, "bf16")
+    x = gen.host_normal((T, D), 1.0, "bf16", 5, "x")
+    w_r = np.zeros((D, E), np.float64)
+    x64 = gen.to_f64(x, "bf16")
+    # W_r column 3 = sign(sum of x) direction: every token's logit 3 is large
+    w_r[:, 3] = np.sign(x64.sum(0)) * 0.5
+    w_r = gen.store(w_r, "bf16")
+    lg = x64 @ gen.to_f64(w_r, "bf16")
+    keep = lg[:, 3] > 0.1  # the other logits are exactly 0
+    x = x[keep]
+    T = x.shape[0]
+    assert T > 10
+    w1, v1, w2 = gen.host_expert_weights(shape, 5)
+    d = _dims(m, shape)
+    want, idx, _ = oracle.layer_tokens(x, w_r, w1, v1, w2, "bf16", K)
+    assert np.all(idx == 3)
+    X, WR, W1, V1, W2 = (dev(a, "bf16") for a in (x, w_r, w1, v1, w2))
+    gi, _, _ = m.route(d, X, WR)
+    counts, offsets, perm, inv = m.dispatch(d, gi)
+    c = counts.cpu().numpy()
+    assert c[3] == T and c.sum() == T
+    out = m.layer_forward(d, X, WR, W1, V1, W2)
+    assert_parity(to_numpy(out), want, "bf16", "one expert")
+
+
+def test_empty_batch_is_a_no_op():
+    m = moe()
+    d = m.dims(64, 64, 4, 2)
+    x = torch.zeros((0, 64), dtype=torch.bfloat16, device="cuda")
+    w = torch.zeros((64, 4), dtype=torch.bfloat16, device="cuda")
+    idx, gate, _ = m.route(d, x, w)
+    assert idx.shape == (0, 2)
+    counts, offsets, perm, inv = m.dispatch(d, idx)
+    assert counts.cpu().tolist() == [0, 0, 0, 0]
+    assert offsets.cpu().tolist() == [0, 0, 0, 0, 0]
+    w1 = torch.zeros((4, 64, 64), dtype=torch.bfloat16, device="cuda")
+    out = m.layer_forward(d, x, w, w1, w1, w1)
+    assert out.shape == (0, 64)
+    assert m.get_last_error() == 0
+
+
+def test_dispatch_reports_bad_index():
+    m = moe()
+    d = m.dims(64, 64, 4, 2)
+    idx = torch.tensor([[0, 1], [2, 9]], dtype=torch.int32, device="cuda")
+    m.dispatch(d, idx)
+    assert m.get_last_error() == 6  # MOE_ERR_DEVICE_INDEX
+    assert m.get_last_error() == 0  # cleared by the read
+
+
+def test_bad_arguments_with_real_tensors():
+    m = moe()
+    d = m.dims(64, 64, 4, 2)
+    x = torch.zeros((4, 64), dtype=torch.bfloat16, device="cuda")
+    w = torch.zeros((64, 4), dtype=torch.bfloat16, device="cuda")
+    w1 = torch.zeros((4, 64, 64), dtype=torch.bfloat16, device="cuda")
+    small = torch.empty(16, dtype=torch.uint8, device="cuda")
+    with pytest.raises(m.MoeError) as ei:
+        m.layer_forward(d, x, w, w1, w1, w1, ws=small)
+    assert ei.value.status == 3
+    xm = torch.zeros(4 * 64 + 1, dtype=torch.bfloat16, device="cuda")[1:].view(4, 64)
+    with pytest.raises(m.MoeError) as ei:
+        m.layer_forward(d, xm, w, w1, w1, w1)
+    assert ei.value.status == 1
+    bad = m.dims(64, 64, 4, 5)
+    with pytest.raises(m.MoeError):
+        m.route(bad, x, w)
+
+
+def test_launch_count_and_profile():
+    m = moe()
+    L = _host((64, 64, 4, 2, 3, "bf16"))
+    d = _dims(m, L.shape)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    m.layer_forward(d, x, w_r, w1, v1, w2)
+    torch.cuda.synchronize()
+    n0 = m.launch_count()
+    m.profile_reset()
+    m.profile_enable(True)
+    m.layer_forward(d, x, w_r, w1, v1, w2)
+    m.profile_enable(False)
+    stats = m.profile_read()
+    assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == 4
+    assert all(v[1] > 0 for v in stats.values())
