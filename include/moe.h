@@ -152,6 +152,35 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x,
                              const void *residual_opt, void *out, void *ws,
                              size_t ws_bytes, moe_stream_t stream);
 
+/* ---- layer without a caller workspace ----------------------------------
+ * The paper has no counterpart of this entry point; it serves callers that
+ * cannot allocate device memory themselves (a framework that owns every
+ * device buffer through its own pool, a plugin handed only its inputs and
+ * outputs, a runtime that forbids allocation after start-up).
+ *
+ * Same arguments and result as moe_layer_forward, minus the workspace: the
+ * scratch space is a fixed array of MOE_NOALLOC_SCRATCH_BYTES bytes in device
+ * memory owned by the library.  Every GPU that loads this part of the
+ * library holds that array until the process exits.
+ *   - Limit: a call is accepted when moe_workspace_size(dims, T) is at most
+ *     MOE_NOALLOC_SCRATCH_BYTES (16 MiB: e.g. the DBRX-shaped layer up to
+ *     64 tokens); larger T returns MOE_ERR_WORKSPACE and launches nothing.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before
+ *     any stream capture on the device.
+ *   - Allocates nothing (no cudaMalloc, cudaFree or allocating library call).
+ *   - Every call uses the same array, which keeps the last call's contents;
+ *     nothing in it has to start at zero.  Calls whose executions overlap on
+ *     the GPU (different streams, or different host threads on one device)
+ *     race on the array: serialise them. */
+#define MOE_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+
+moe_status moe_layer_forward_noalloc(const moe_dims *dims, int32_t T,
+                                     const void *x, const void *w_router,
+                                     const void *w1, const void *v1,
+                                     const void *w2, const void *residual_opt,
+                                     void *out, moe_stream_t stream);
+
 /* Human-readable name of a status. */
 const char *moe_status_string(moe_status status);
 

@@ -27,7 +27,7 @@ _STATUS = {
 # Every function the header declares (checked by the CPU tests).
 EXPORTS = (
     "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
-    "moe_combine", "moe_layer_forward", "moe_status_string",
+    "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc", "moe_status_string",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
     "moe_profile_reset", "moe_profile_read",
 )
@@ -80,6 +80,7 @@ def lib() -> ctypes.CDLL:
         "moe_expert_ffn": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
         "moe_combine": [DP, I32, P, P, P, P, P, P],
         "moe_layer_forward": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
+        "moe_layer_forward_noalloc": [DP, I32, P, P, P, P, P, P, P, P],
         "moe_get_last_error": [P],
         "moe_status_string": [ctypes.c_int],
         "moe_profile_enable": [ctypes.c_int],
@@ -199,6 +200,22 @@ def layer_forward(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, ws=None,
     _check(lib().moe_layer_forward(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(w1), _ptr(v1),
                                    _ptr(w2), _ptr(residual), _ptr(out), _ptr(ws), ws.numel(),
                                    _stream(stream)), "moe_layer_forward")
+    return out
+
+
+NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024  # MOE_NOALLOC_SCRATCH_BYTES
+
+
+def layer_forward_noalloc(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, stream=None):
+    """The whole layer with the library's fixed device scratch array instead
+    of a workspace (for callers that cannot allocate; T limited so that the
+    workspace fits in 16 MiB).  Returns out [T, D] (out_dtype)."""
+    T = x.shape[0]
+    if out is None:
+        out = torch.empty((T, d.d_model), dtype=_tdt(d.out_dtype), device=x.device)
+    _check(lib().moe_layer_forward_noalloc(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(w1),
+                                           _ptr(v1), _ptr(w2), _ptr(residual), _ptr(out),
+                                           _stream(stream)), "moe_layer_forward_noalloc")
     return out
 
 

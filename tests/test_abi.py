@@ -126,5 +126,16 @@ def test_layer_and_ffn_validation(lib):
     assert L.moe_dispatch(ctypes.byref(d), 8, A, None, A, A, A, None) == 1
 
 
+@no_gpu
+def test_noalloc_validation(lib):
+    L = lib.lib()
+    d = lib.dims(**DBRX)
+    call = lambda T, x=A: L.moe_layer_forward_noalloc(ctypes.byref(d), T, x, A, A, A, A, None, A, None)
+    assert call(100000) == 3  # beyond the fixed scratch array
+    assert call(-1) == 1
+    assert call(0) == 0
+    assert call(1, x=None) == 1
+
+
 def test_launch_count_starts_at_zero_without_launches(lib):
     assert lib.launch_count() >= 0
