@@ -211,11 +211,15 @@ def algorithmic_bytes(kernel: str, shape: gen.LayerShape, T: int, U: float) -> f
     selected experts it streams, plus its activations."""
     D, F, E, K = shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k
     S = T * K
-    if kernel == "up_glu_gemv":
+    if kernel == "up_glu_gemv":  # fp32 h
         return U * 2 * F * D * 2 + T * D * 2 + S * F * 4
     if kernel == "down_combine_gemv":
         return U * D * F * 2 + S * F * 4 + T * D * 2
-    if kernel == "route":
+    if kernel == "up_glu_stream":  # bf16 h
+        return U * 2 * F * D * 2 + T * D * 2 + S * F * 2
+    if kernel == "down_combine_stream":
+        return U * D * F * 2 + S * F * 2 + T * D * 2
+    if kernel in ("route", "route_dispatch_small"):
         return D * E * 2 + T * D * 2 + S * 8
     return 0.0
 

@@ -27,34 +27,6 @@ constexpr int kRowsPerUnit = kWarps * kRowsPerWarp;  // up kernel: rows per work
 
 // Exclusive scan over experts of ceil(n_e / NS), written to prefix[0..E].
 // Executed by warp 0 of the block; E <= 256.
-// An expert whose slot range is not inside [0, S] is recorded as an index
-// error and given no work, so a corrupt offsets array cannot move an access
-// out of bounds.
-template <int NS>
-__device__ void chunk_prefix(const int32_t *offsets, int E, int S, int *prefix,
-                             unsigned *err) {
-    const int lane = threadIdx.x & 31;
-    int run = 0;
-    for (int base = 0; base < E; base += 32) {
-        int e = base + lane;
-        int c = 0;
-        if (e < E) {
-            const int lo = offsets[e], hi = offsets[e + 1];
-            if (lo < 0 || hi < lo || hi > S) set_error(err, kErrIndex);
-            else c = (hi - lo + NS - 1) / NS;
-        }
-        int incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            int v = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += v;
-        }
-        if (e < E) prefix[e] = run + incl - c;
-        run += __shfl_sync(0xffffffffu, incl, 31);
-    }
-    if (lane == 0) prefix[E] = run;
-}
-
 template <typename TX, typename TW, int NS>
 __global__ void __launch_bounds__(kThreads)
 k_up_glu_gemv(int D, int F, int E, int K, int T, const TX *__restrict__ x,

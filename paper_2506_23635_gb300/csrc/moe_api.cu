@@ -9,6 +9,7 @@
 #include <vector>
 
 #include "moe_internal.cuh"
+#include "ptx.cuh"
 
 namespace moe {
 
@@ -16,28 +17,45 @@ __device__ unsigned g_moe_err = 0;
 
 // ===========================================================================
 // Step 1: router logits, softmax, top-k, renormalised gates.
-// A block of 256 threads handles kRouteTokens tokens; its threads split d,
-// each accumulating 16 experts at a time for every token, then the partial
-// sums are reduced across the block.  Warp w then selects the top-k of token
-// w: K rounds of a warp arg-max over the not-yet-taken experts, ties going
-// to the lower expert index.
+// block_logits: a block of NT threads computes the logits of up to 4 tokens;
+// its threads split d, each accumulating 16 experts at a time for every
+// token (16-byte loads of a router row when E is a multiple of 8), then the
+// partial sums are reduced across the block into shared memory.
+// select_topk: one warp per token, K rounds of a warp arg-max over the
+// not-yet-taken experts, ties going to the lower expert index.
 // ===========================================================================
 constexpr int kRouteThreads = 256;
 constexpr int kRouteTokens = 4;
+constexpr int kSmallThreads = 512;
+constexpr int kSmallMaxSlots = 32;  // fused route + dispatch: T*K <= 32, T <= 4
 
-template <typename TX, typename TW>
-__global__ void __launch_bounds__(kRouteThreads)
-k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restrict__ wr,
-        float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
-        float *__restrict__ topk_gate) {
-    constexpr int TT = kRouteTokens, NW = kRouteThreads / 32;
-    __shared__ float red[NW][TT * 16];
-    __shared__ float lg[TT][256];
-    __shared__ float pk[TT][256];
-    const int t0 = blockIdx.x * TT;
-    const int nt = min(TT, T - t0);
+template <typename TW>
+__device__ __forceinline__ void router_row16(const TW *wrow, int ne, bool vec, float (&w)[16]) {
+    if (vec) {  // E % 8 == 0: whole 8-wide groups, 16-byte aligned
+        float t8[8];
+        load8(wrow, t8);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[j] = t8[j];
+        if (ne > 8) {
+            load8(wrow + 8, t8);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) w[8 + j] = t8[j];
+        } else {
+#pragma unroll
+            for (int j = 8; j < 16; ++j) w[j] = 0.f;
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) w[j] = j < ne ? to_f(wrow[j]) : 0.f;
+    }
+}
+
+template <typename TX, typename TW, int NT>
+__device__ void block_logits(int D, int E, const TX *__restrict__ x, const TW *__restrict__ wr,
+                             int t0, int nt, float (*lg)[256], float (*red)[kRouteTokens * 16]) {
+    constexpr int TT = kRouteTokens, NW = NT / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
+    const bool vec = (E % 8) == 0;
     for (int e0 = 0; e0 < E; e0 += 16) {
         const int ne = min(16, E - e0);
         float acc[TT][16];
@@ -45,19 +63,17 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
         for (int a = 0; a < TT; ++a)
 #pragma unroll
             for (int j = 0; j < 16; ++j) acc[a][j] = 0.f;
-        for (int d = threadIdx.x; d < D; d += kRouteThreads) {
+#pragma unroll 4
+        for (int d = threadIdx.x; d < D; d += NT) {
             float xv[TT];
 #pragma unroll
             for (int a = 0; a < TT; ++a) xv[a] = a < nt ? to_f(x[(size_t)(t0 + a) * D + d]) : 0.f;
-            const TW *wrow = wr + (size_t)d * E + e0;
+            float w[16];
+            router_row16(wr + (size_t)d * E + e0, ne, vec, w);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                if (j < ne) {
-                    const float w = to_f(wrow[j]);
+            for (int j = 0; j < 16; ++j)
 #pragma unroll
-                    for (int a = 0; a < TT; ++a) acc[a][j] = fmaf(xv[a], w, acc[a][j]);
-                }
-            }
+                for (int a = 0; a < TT; ++a) acc[a][j] = fmaf(xv[a], w[j], acc[a][j]);
         }
 #pragma unroll
         for (int a = 0; a < TT; ++a)
@@ -67,7 +83,7 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
                 if (lane == 0) red[warp][a * 16 + j] = v;
             }
         __syncthreads();
-        for (int i = threadIdx.x; i < TT * 16; i += kRouteThreads) {
+        for (int i = threadIdx.x; i < TT * 16; i += NT) {
             const int a = i >> 4, j = i & 15;
             if (a < nt && j < ne) {
                 float s = 0.f;
@@ -78,10 +94,14 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
         }
         __syncthreads();
     }
+}
 
-    if (warp >= nt) return;
-    const int t = t0 + warp;
-    const float *l = lg[warp];
+// Warp-level softmax + top-k of one token's logits l[0..E); writes
+// topk_idx/topk_gate[t*K + k] (and sidx[k] if non-null).
+__device__ void select_topk(int E, int K, int t, const float *l, float *pk,
+                            float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
+                            float *__restrict__ topk_gate, int *sidx) {
+    const int lane = threadIdx.x & 31;
     if (logits_opt)
         for (int e = lane; e < E; e += 32) logits_opt[(size_t)t * E + e] = l[e];
     float m = -INFINITY;
@@ -113,11 +133,84 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
         psel += p;
         if (lane == 0) {
             topk_idx[(size_t)t * K + k] = bi;
-            pk[warp][k] = p;
+            pk[k] = p;
+            if (sidx) sidx[k] = bi;
         }
     }
     __syncwarp();
-    for (int k = lane; k < K; k += 32) topk_gate[(size_t)t * K + k] = pk[warp][k] / psel;
+    for (int k = lane; k < K; k += 32) topk_gate[(size_t)t * K + k] = pk[k] / psel;
+}
+
+template <typename TX, typename TW>
+__global__ void __launch_bounds__(kRouteThreads)
+k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restrict__ wr,
+        float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
+        float *__restrict__ topk_gate) {
+    __shared__ float red[kRouteThreads / 32][kRouteTokens * 16];
+    __shared__ float lg[kRouteTokens][256];
+    __shared__ float pk[kRouteTokens][256];
+    const int t0 = blockIdx.x * kRouteTokens;
+    const int nt = min(kRouteTokens, T - t0);
+    const int warp = threadIdx.x >> 5;
+    block_logits<TX, TW, kRouteThreads>(D, E, x, wr, t0, nt, lg, red);
+    if (warp >= nt) return;
+    select_topk(E, K, t0 + warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate, nullptr);
+}
+
+// Route and dispatch of a tiny batch (T <= 4, T*K <= 32) in one block: the
+// top-k indices stay in shared memory and warp 0 ranks the slots (ranks of
+// equal experts from __match_any_sync, so the order is the stable one).
+template <typename TX, typename TW>
+__global__ void __launch_bounds__(kSmallThreads)
+k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
+                       const TW *__restrict__ wr, float *__restrict__ logits_opt,
+                       int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
+                       int32_t *__restrict__ counts, int32_t *__restrict__ offsets,
+                       int32_t *__restrict__ perm, int32_t *__restrict__ inv_perm) {
+    __shared__ float red[kSmallThreads / 32][kRouteTokens * 16];
+    __shared__ float lg[kRouteTokens][256];
+    __shared__ float pk[kRouteTokens][256];
+    __shared__ int sidx[kSmallMaxSlots];
+    __shared__ int cnt[256];
+    __shared__ int offs[257];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    ptx::grid_dependency_wait();
+    for (int e = threadIdx.x; e < E; e += kSmallThreads) cnt[e] = 0;
+    block_logits<TX, TW, kSmallThreads>(D, E, x, wr, 0, T, lg, red);
+    if (warp < T)
+        select_topk(E, K, warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
+                    sidx + warp * K);
+    __syncthreads();
+    if (warp != 0) return;
+    const int S = T * K;
+    const int e = lane < S ? sidx[lane] : -1;
+    if (e >= 0) atomicAdd(&cnt[e], 1);
+    __syncwarp();
+    int carry = 0;
+    for (int base = 0; base < E; base += 32) {
+        const int ee = base + lane;
+        const int c = ee < E ? cnt[ee] : 0;
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (ee < E) {
+            offs[ee] = carry + incl - c;
+            counts[ee] = c;
+            offsets[ee] = carry + incl - c;
+        }
+        carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) offsets[E] = carry;
+    __syncwarp();
+    const unsigned same = __match_any_sync(0xffffffffu, e);
+    if (e >= 0) {
+        const int pos = offs[e] + __popc(same & ((1u << lane) - 1u));
+        perm[pos] = lane;
+        inv_perm[lane] = pos;
+    }
 }
 
 // ===========================================================================
@@ -382,6 +475,35 @@ cudaError_t launch_route(const moe_dims &d, int T, const void *x, const void *wr
     return cudaGetLastError();
 }
 
+template <typename TX, typename TW>
+cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x, const void *wr,
+                                        int32_t *idx, float *gate, int32_t *counts,
+                                        int32_t *offsets, int32_t *perm, int32_t *inv,
+                                        cudaStream_t st) {
+    int Tv = T, D = d.d_model, E = d.n_experts, K = d.top_k;
+    const TX *xp = static_cast<const TX *>(x);
+    const TW *wp = static_cast<const TW *>(wr);
+    float *logits = nullptr;
+    void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &logits, &idx, &gate, &counts, &offsets, &perm, &inv};
+    LaunchScope ls("route_dispatch_small", st);
+    return launch_pdl((const void *)k_route_dispatch_small<TX, TW>, dim3(1), dim3(kSmallThreads), 0,
+                      st, args);
+}
+
+bool small_route_ok(const moe_dims &d, int T) {
+    return T <= kRouteTokens && T * d.top_k <= kSmallMaxSlots;
+}
+
+cudaError_t route_dispatch_small_any(const moe_dims &d, int T, const void *x, const void *wr,
+                                     int32_t *idx, float *gate, int32_t *counts, int32_t *offsets,
+                                     int32_t *perm, int32_t *inv, cudaStream_t st) {
+    if (d.w_dtype == MOE_BF16)
+        return launch_route_dispatch_small<bf16, bf16>(d, T, x, wr, idx, gate, counts, offsets,
+                                                       perm, inv, st);
+    return launch_route_dispatch_small<float, float>(d, T, x, wr, idx, gate, counts, offsets, perm,
+                                                     inv, st);
+}
+
 cudaError_t route_any(const moe_dims &d, int T, const void *x, const void *wr, float *logits,
                       int32_t *idx, float *gate, cudaStream_t st) {
     if (d.w_dtype == MOE_BF16) return launch_route<bf16, bf16>(d, T, x, wr, logits, idx, gate, st);
@@ -476,7 +598,16 @@ moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x, const 
     if (!ws || !aligned16(ws) || ws_bytes < L.total) return MOE_ERR_WORKSPACE;
     cudaStream_t st = (cudaStream_t)stream;
     float *h = at<float>(ws, L.h);
-    cudaError_t e = launch_up_glu_gemv(*dims, T, x, perm, offsets, w1, v1, h, st);
+    cudaError_t e;
+    if (stream_path_ok(*dims, T)) {
+        // bf16 weights, few slots: bulk-copy pipelined kernels, bf16 h
+        e = launch_up_glu_stream(*dims, T, x, perm, offsets, w1, v1, h, st);
+        if (e == cudaSuccess)
+            e = launch_down_stream(*dims, T, h, offsets, nullptr, w2, nullptr, nullptr, nullptr,
+                                   y_sorted, false, st);
+        return cuda_status(e);
+    }
+    e = launch_up_glu_gemv(*dims, T, x, perm, offsets, w1, v1, h, st);
     if (e == cudaSuccess)
         e = launch_down_gemv(*dims, T, h, perm, offsets, w2, nullptr, y_sorted, nullptr, nullptr,
                              false, st);
@@ -519,9 +650,24 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
     int32_t *inv = at<int32_t>(ws, L.inv_perm);
     float *h = at<float>(ws, L.h);
 
-    cudaError_t e = route_any(d, T, x, w_router, nullptr, idx, gate, st);
-    if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
-    if (e == cudaSuccess) e = launch_up_glu_gemv(d, T, x, perm, offsets, w1, v1, h, st);
+    cudaError_t e;
+    if (small_route_ok(d, T)) {
+        e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
+    } else {
+        e = route_any(d, T, x, w_router, nullptr, idx, gate, st);
+        if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
+    }
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    if (stream_path_ok(d, T)) {
+        // decode, bf16: bulk-copy pipelined kernels, combine fused into the
+        // down projection (T*K <= 64 slots, so T <= 64)
+        e = launch_up_glu_stream(d, T, x, perm, offsets, w1, v1, h, st);
+        if (e == cudaSuccess)
+            e = launch_down_stream(d, T, h, offsets, inv, w2, gate, residual_opt, out, nullptr,
+                                   true, st);
+        return cuda_status(e);
+    }
+    e = launch_up_glu_gemv(d, T, x, perm, offsets, w1, v1, h, st);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     if (T <= kFusedCombineMaxTokens) {
         e = launch_down_gemv(d, T, h, perm, offsets, w2, gate, nullptr, residual_opt, out, true, st);

@@ -2,6 +2,8 @@
 // Nothing here is part of the C ABI (include/moe.h).
 #pragma once
 
+#include <algorithm>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -82,6 +84,46 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 __device__ __forceinline__ float silu(float a) { return a / (1.0f + expf(-a)); }
 
+// An expert whose slot range is not inside [0, S] is recorded as an index
+// error and given no work, so a corrupt offsets array cannot move an access
+// out of bounds.
+template <int NS>
+__device__ __forceinline__ void chunk_prefix(const int32_t *offsets, int E, int S, int *prefix,
+                             unsigned *err) {
+    const int lane = threadIdx.x & 31;
+    int run = 0;
+    for (int base = 0; base < E; base += 32) {
+        int e = base + lane;
+        int c = 0;
+        if (e < E) {
+            const int lo = offsets[e], hi = offsets[e + 1];
+            if (lo < 0 || hi < lo || hi > S) set_error(err, kErrIndex);
+            else c = (hi - lo + NS - 1) / NS;
+        }
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (e < E) prefix[e] = run + incl - c;
+        run += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) prefix[E] = run;
+}
+
+
+// Expert e of chunk q: the largest e with prefix[e] <= q (prefix from
+// chunk_prefix; experts without chunks have prefix[e] == prefix[e+1]).
+__device__ __forceinline__ int chunk_expert(const int *prefix, int E, int q) {
+    int lo = 0, hi = E - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (prefix[mid] <= q) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
 // ---- host side -----------------------------------------------------------
 
 struct DeviceInfo {
@@ -119,6 +161,36 @@ cudaError_t launch_down_gemv(const moe_dims &d, int T, const float *h,
                              const void *residual, void *out, bool fused,
                              cudaStream_t st);
 
+// Launch with programmatic stream serialisation: the kernel may begin while
+// the previous kernel in the stream finishes, and must execute
+// griddepcontrol.wait before touching memory that kernel writes or reads.
+inline cudaError_t launch_pdl(const void *func, dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, void **args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelExC(&cfg, func, args);
+}
+
 constexpr int kFusedCombineMaxTokens = 64;
+
+// Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
+// kStreamMaxSlots slots; the GLU hidden vectors h are bf16.
+constexpr int kStreamMaxSlots = 64;
+bool stream_path_ok(const moe_dims &d, int T);
+cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
+                                 const int32_t *offsets, const void *w1, const void *v1, void *h,
+                                 cudaStream_t st);
+cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const int32_t *offsets,
+                               const int32_t *inv_perm, const void *w2, const float *gate,
+                               const void *residual, void *out, float *y_sorted, bool fused,
+                               cudaStream_t st);
 
 }  // namespace moe

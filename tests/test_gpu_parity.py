@@ -208,5 +208,7 @@ def test_launch_count_and_profile():
     m.layer_forward(d, x, w_r, w1, v1, w2)
     m.profile_enable(False)
     stats = m.profile_read()
-    assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == 4
+    # tiny batch: fused route+dispatch, up projection, down projection + combine
+    assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == 3
+    assert set(stats) == {"route_dispatch_small", "up_glu_stream", "down_combine_stream"}
     assert all(v[1] > 0 for v in stats.values())
