@@ -28,6 +28,9 @@ constexpr int kRouteThreads = 256;
 constexpr int kRouteTokens = 4;
 constexpr int kSmallThreads = 512;
 constexpr int kSmallMaxSlots = 32;  // fused route + dispatch: T*K <= 32, T <= 4
+// dynamic shared memory the fused kernel may use for the staged router and
+// tokens (static arrays of the kernel: ~15 KB)
+constexpr size_t kSmallStageBytes = 208 * 1024;
 
 template <typename TW>
 __device__ __forceinline__ void router_row16(const TW *wrow, int ne, bool vec, float (&w)[16]) {
@@ -160,23 +163,116 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
 // Route and dispatch of a tiny batch (T <= 4, T*K <= 32) in one block: the
 // top-k indices stay in shared memory and warp 0 ranks the slots (ranks of
 // equal experts from __match_any_sync, so the order is the stable one).
+// When the router matrix and the tokens fit in shared memory (STAGED), they
+// are brought in first by bulk copies on one mbarrier, so the block waits for
+// memory once instead of once per loop trip.
+template <typename TX, typename TW>
+__device__ void smem_logits(int D, int E, const TX *xs, const TW *wrs, int nt, float (*lg)[256],
+                            float (*red)[kRouteTokens * 16]) {
+    constexpr int TT = kRouteTokens, NT = kSmallThreads, NW = NT / 32;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool vec = (E % 8) == 0;
+    for (int e0 = 0; e0 < E; e0 += 16) {
+        const int ne = min(16, E - e0);
+        float acc[TT][16];
+#pragma unroll
+        for (int a = 0; a < TT; ++a)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) acc[a][j] = 0.f;
+        for (int d = threadIdx.x; d < D; d += NT) {
+            float xv[TT];
+#pragma unroll
+            for (int a = 0; a < TT; ++a) xv[a] = a < nt ? to_f(xs[(size_t)a * D + d]) : 0.f;
+            const TW *wrow = wrs + (size_t)d * E + e0;
+            float w[16];
+            if (vec && sizeof(TW) == 2) {
+                const uint4 u0 = *reinterpret_cast<const uint4 *>(wrow);
+                unpack_bf16x2(u0.x, w[0], w[1]); unpack_bf16x2(u0.y, w[2], w[3]);
+                unpack_bf16x2(u0.z, w[4], w[5]); unpack_bf16x2(u0.w, w[6], w[7]);
+                if (ne > 8) {
+                    const uint4 u1 = *reinterpret_cast<const uint4 *>(wrow + 8);
+                    unpack_bf16x2(u1.x, w[8], w[9]); unpack_bf16x2(u1.y, w[10], w[11]);
+                    unpack_bf16x2(u1.z, w[12], w[13]); unpack_bf16x2(u1.w, w[14], w[15]);
+                } else {
+#pragma unroll
+                    for (int j = 8; j < 16; ++j) w[j] = 0.f;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) w[j] = j < ne ? to_f(wrow[j]) : 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+#pragma unroll
+                for (int a = 0; a < TT; ++a) acc[a][j] = fmaf(xv[a], w[j], acc[a][j]);
+        }
+#pragma unroll
+        for (int a = 0; a < TT; ++a) {
+            if (a >= nt) break;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float v = warp_sum(acc[a][j]);
+                if (lane == 0) red[warp][a * 16 + j] = v;
+            }
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < TT * 16; i += NT) {
+            const int a = i >> 4, j = i & 15;
+            if (a < nt && j < ne) {
+                float s = 0.f;
+#pragma unroll
+                for (int w = 0; w < NW; ++w) s += red[w][i];
+                lg[a][e0 + j] = s;
+            }
+        }
+        __syncthreads();
+    }
+}
+
 template <typename TX, typename TW>
 __global__ void __launch_bounds__(kSmallThreads)
 k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
                        const TW *__restrict__ wr, float *__restrict__ logits_opt,
                        int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
                        int32_t *__restrict__ counts, int32_t *__restrict__ offsets,
-                       int32_t *__restrict__ perm, int32_t *__restrict__ inv_perm) {
+                       int32_t *__restrict__ perm, int32_t *__restrict__ inv_perm, int staged,
+                       unsigned *err) {
+    extern __shared__ __align__(128) unsigned char dsm[];  // staged: W_r, then x
     __shared__ float red[kSmallThreads / 32][kRouteTokens * 16];
     __shared__ float lg[kRouteTokens][256];
     __shared__ float pk[kRouteTokens][256];
     __shared__ int sidx[kSmallMaxSlots];
     __shared__ int cnt[256];
     __shared__ int offs[257];
+    __shared__ uint64_t bar;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    ptx::grid_dependency_wait();
     for (int e = threadIdx.x; e < E; e += kSmallThreads) cnt[e] = 0;
-    block_logits<TX, TW, kSmallThreads>(D, E, x, wr, 0, T, lg, red);
+    if (staged) {
+        const uint32_t wr_bytes = (uint32_t)D * E * sizeof(TW);
+        const uint32_t x_off = (wr_bytes + 127u) & ~127u;
+        const uint32_t x_bytes = (uint32_t)T * D * sizeof(TX);
+        if (threadIdx.x == 0) {
+            ptx::mbar_init(&bar, 1);
+            ptx::fence_barrier_init();
+        }
+        __syncthreads();
+        ptx::grid_dependency_wait();  // x may come from the previous kernel
+        if (threadIdx.x == 0) {
+            const uint64_t pol = ptx::policy_evict_last();
+            ptx::mbar_arrive_expect_tx(&bar, wr_bytes + x_bytes);
+            constexpr uint32_t kChunk = 32768;
+            for (uint32_t o = 0; o < wr_bytes; o += kChunk)
+                ptx::bulk_g2s(dsm + o, reinterpret_cast<const unsigned char *>(wr) + o,
+                              min(kChunk, wr_bytes - o), &bar, pol);
+            ptx::bulk_g2s(dsm + x_off, x, x_bytes, &bar, pol);
+        }
+        if (!ptx::mbar_wait(&bar, 0, err)) return;  // every thread waits; none has synced since
+        smem_logits<TX, TW>(D, E, reinterpret_cast<const TX *>(dsm + x_off),
+                            reinterpret_cast<const TW *>(dsm), T, lg, red);
+    } else {
+        ptx::grid_dependency_wait();
+        block_logits<TX, TW, kSmallThreads>(D, E, x, wr, 0, T, lg, red);
+    }
     if (warp < T)
         select_topk(E, K, warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
                     sidx + warp * K);
@@ -484,10 +580,22 @@ cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x,
     const TX *xp = static_cast<const TX *>(x);
     const TW *wp = static_cast<const TW *>(wr);
     float *logits = nullptr;
-    void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &logits, &idx, &gate, &counts, &offsets, &perm, &inv};
+    unsigned *err = device_info().err;
+    // stage W_r and x in shared memory when they fit next to the static arrays
+    const size_t wr_bytes = (size_t)D * E * sizeof(TW);
+    const size_t dyn = ((wr_bytes + 127) & ~size_t(127)) + (size_t)T * D * sizeof(TX);
+    int staged = dyn <= kSmallStageBytes ? 1 : 0;
+    const void *kern = (const void *)k_route_dispatch_small<TX, TW>;
+    const size_t smem = staged ? dyn : 0;
+    if (staged) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kSmallStageBytes);
+        if (e != cudaSuccess) return e;
+    }
+    void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &logits, &idx, &gate, &counts, &offsets, &perm, &inv,
+                    &staged, &err};
     LaunchScope ls("route_dispatch_small", st);
-    return launch_pdl((const void *)k_route_dispatch_small<TX, TW>, dim3(1), dim3(kSmallThreads), 0,
-                      st, args);
+    return launch_pdl(kern, dim3(1), dim3(kSmallThreads), smem, st, args);
 }
 
 bool small_route_ok(const moe_dims &d, int T) {
