@@ -36,20 +36,24 @@ import numpy as np  # noqa: E402
 from paper_2506_23635_gb300 import inputs as gen  # noqa: E402
 
 METRIC = "MoE-layer us/token-step (DBRX-shaped layer, decode)"
+METRIC_PREFILL = "MoE-layer prefill TFLOP/s (DBRX-shaped layer)"
 UNIT = "us/token-step"
 SEED = 1234
 POOL = 64  # distinct token inputs cycled through by the timed steps
 HBM_FALLBACK_GBS = 6800.0
 
+# name: (shape, tokens per step)
 WORKLOADS = {
-    # name: (shape, tokens per step)
-    "dbrx-decode-t1": (gen.DBRX, 1),
-    "dbrx-decode-t8": (gen.DBRX, 8),
-    "dbrx-decode-t64": (gen.DBRX, 64),
+    **{f"dbrx-decode-t{T}": (gen.DBRX, T) for T in (1, 2, 4, 8, 16, 32, 64)},
+    "dbrx-prefill-t2048": (gen.DBRX, 2048),
     # the same per-launch work as dbrx-decode-t1 (4 experts streamed) with
     # only 4 experts resident (1.6 GB): the small case for ncu captures
     "dbrx4-decode-t1": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 1),
+    # a 512-token prefill of the same 4-expert layer: the small case for
+    # captures of the tensor-core GEMMs
+    "dbrx4-prefill-t512": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 512),
 }
+PREFILL_MIN_TOKENS = 512
 
 
 def parse():
@@ -60,6 +64,8 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", choices=sorted(WORKLOADS), default="dbrx-decode-t1")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the prefill and decode-sweep side measurements")
     p.add_argument("--cpu-seconds", type=float, default=12.0,
                    help="time budget of the oracle sample")
     return p.parse_args()
@@ -229,15 +235,160 @@ def algorithmic_bytes(kernel: str, shape: gen.LayerShape, T: int, U: float) -> f
 # --------------------------------------------------------------------------
 
 
-def token_pool(shape, T, seed):
-    """POOL gap-conditioned token batches [POOL, T, D] sharing one router."""
+def token_pool(shape, T, seed, pool=POOL):
+    """`pool` gap-conditioned token batches [pool, T, D] sharing one router."""
     D, E = shape.d_model, shape.n_experts
     w_r = gen.host_normal((D, E), gen.W_STD, shape.dtype, seed, "w_r")
     xs = []
-    for i in range(POOL):
+    for i in range(pool):
         x = gen.host_normal((T, D), gen.X_STD, shape.dtype, seed, "x", i)
         xs.append(gen.gap_condition_tokens(x, w_r, shape, seed + i))
     return np.stack(xs), w_r
+
+
+def algorithmic_flops(kernel: str, shape: gen.LayerShape, T: int) -> float:
+    """Multiply-adds x 2 a GEMM kernel must do per launch."""
+    D, F, K = shape.d_model, shape.ffn_hidden, shape.top_k
+    S = T * K
+    if kernel == "gemm_up_glu_tc":
+        return 2.0 * S * 2 * F * D
+    if kernel == "gemm_down_tc":
+        return 2.0 * S * D * F
+    return 0.0
+
+
+class Layer:
+    """One DBRX-shaped layer resident on the device, and a timer for its steps."""
+
+    def __init__(self, moe, shape, dev, dist):
+        import torch
+
+        self.moe, self.shape, self.dev, self.dist = moe, shape, dev, dist
+        self.w = gen.device_expert_weights(shape, SEED, dev)
+        self.d = moe.dims(shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k,
+                          torch.bfloat16)
+        self.stream = torch.cuda.current_stream(dev)
+
+    def inputs(self, T, pool):
+        import torch
+
+        xs_host, w_r_host = token_pool(self.shape, T, SEED, pool)
+        xs = gen.host_to_torch(xs_host, self.shape.dtype, self.dev)
+        w_r = gen.host_to_torch(w_r_host, self.shape.dtype, self.dev)
+        ws = self.moe.alloc_workspace(self.d, T, self.dev)
+        out = torch.empty((T, self.shape.d_model), dtype=torch.bfloat16, device=self.dev)
+        return xs_host, w_r_host, xs, w_r, ws, out
+
+    def distinct_experts(self, xs, w_r):
+        U = []
+        for i in range(xs.shape[0]):
+            idx, _, _ = self.moe.route(self.d, xs[i], w_r)
+            U.append(len(set(idx.cpu().numpy().reshape(-1).tolist())))
+        return float(np.mean(U))
+
+    def time_steps(self, step, steps, clocks=None):
+        """ms per step over `steps` steps (CUDA events on the stream, max over
+        ranks), then the same steps again with per-kernel events."""
+        import torch
+
+        moe = self.moe
+        barrier(self.dist)
+        torch.cuda.synchronize()
+        n0 = moe.launch_count()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        wall0 = time.time()
+        ev0.record(self.stream)
+        for i in range(steps):
+            step(i)
+        ev1.record(self.stream)
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.mark(wall0, time.time())
+        barrier(self.dist)
+        launches = moe.launch_count() - n0
+        ms = max_over_ranks(ev0.elapsed_time(ev1) / steps, self.dist, self.dev)
+        moe.profile_reset()
+        moe.profile_enable(True)
+        for i in range(steps):
+            step(i)
+        torch.cuda.synchronize()
+        moe.profile_enable(False)
+        kstats = {k: v for k, v in moe.profile_read().items() if v[0] > 0}
+        moe.check_device_errors(self.stream)
+        return ms, launches, kstats
+
+
+def kernel_table(kstats):
+    tot = sum(v[1] for v in kstats.values())
+    return {k: {"launches": v[0], "avg_us": round(v[1] / v[0] * 1e3, 2),
+                "share": round(v[1] / tot, 4)} for k, v in kstats.items()}
+
+
+def hbm_roofline(kstats, shape, T, U, workload):
+    dominant = max(kstats, key=lambda k: kstats[k][1])
+    n_dom, ms_dom = kstats[dominant]
+    avg_s = ms_dom / n_dom / 1e3
+    alg = algorithmic_bytes(dominant, shape, T, U)
+    peaks, src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
+    achieved = alg / avg_s / 1e9
+    return {"kernel": dominant, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+            "unit": "GB/s", "frac": round(achieved / peak, 4),
+            "peak_source": f"{src} hbm_gbs" + (" (burst copy)" if src == "measured" else ""),
+            "traffic": committed_traffic(dominant, workload),
+            "algorithmic_bytes_per_launch": alg, "avg_launch_us": round(avg_s * 1e6, 2),
+            "timing": "CUDA events around each launch on its stream, over a second pass "
+                      "of the same K steps"}
+
+
+def tensor_roofline(kstats, shape, T, workload):
+    gemms = {k: v for k, v in kstats.items() if algorithmic_flops(k, shape, T) > 0}
+    dominant = max(gemms, key=lambda k: gemms[k][1])
+    n_dom, ms_dom = gemms[dominant]
+    avg_s = ms_dom / n_dom / 1e3
+    flops = algorithmic_flops(dominant, shape, T)
+    peaks, src = measured_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
+    achieved = flops / avg_s / 1e12
+    return {"kernel": dominant, "bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
+            "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+            "peak_source": f"{src} bf16_tflops_sustained (cuBLAS bf16 GEMM, seconds-long loop)",
+            "frac_of_burst_peak": round(achieved / float(peaks.get("bf16_tflops", 1910.6)), 4),
+            "traffic": committed_traffic(dominant, workload),
+            "algorithmic_flops_per_launch": flops, "avg_launch_us": round(avg_s * 1e6, 2),
+            "timing": "CUDA events around each launch on its stream, over a second pass "
+                      "of the same K steps"}
+
+
+def measure_extra(layer, workload, steps, warmup):
+    """A secondary workload of the same layer: a few timed steps."""
+    shape, T = WORKLOADS[workload]
+    pool = 4 if T >= PREFILL_MIN_TOKENS else 16
+    _, _, xs, w_r, ws, out = layer.inputs(T, pool)
+    w1, v1, w2 = layer.w
+    d, moe = layer.d, layer.moe
+
+    def step(i):
+        moe.layer_forward(d, xs[i % pool], w_r, w1, v1, w2, out=out, ws=ws, stream=layer.stream)
+
+    for i in range(warmup):
+        step(i)
+    ms, launches, kstats = layer.time_steps(step, steps)
+    r = {"workload": workload, "tokens_per_step": T, "steps": steps,
+         "ms_per_step": round(ms, 4), "us_per_token_step": round(ms * 1e3 / T, 3),
+         "kernels": kernel_table(kstats)}
+    if T >= PREFILL_MIN_TOKENS:
+        flops = 2.0 * T * shape.top_k * 3 * shape.d_model * shape.ffn_hidden
+        r["tflops"] = round(flops / (ms / 1e3) / 1e12, 1)
+        r["roofline"] = tensor_roofline(kstats, shape, T, workload)
+    else:
+        U = layer.distinct_experts(xs, w_r)
+        step_bytes = U * 3 * shape.d_model * shape.ffn_hidden * 2
+        r["distinct_experts_per_step"] = U
+        r["achieved_hbm_gbs_step"] = round(step_bytes / (ms / 1e3) / 1e9, 1)
+        peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
+        r["frac_of_hbm_step"] = round(step_bytes / (ms / 1e3) / 1e9 / peak, 4)
+    return r
 
 
 def run_ours(args):
@@ -251,25 +402,17 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     shape, T = WORKLOADS[args.workload]
     D, F, E, K = shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k
+    prefill = T >= PREFILL_MIN_TOKENS
 
-    w1, v1, w2 = gen.device_expert_weights(shape, SEED, dev)
-    xs_host, w_r_host = token_pool(shape, T, SEED)
-    xs = gen.host_to_torch(xs_host, shape.dtype, dev)  # [POOL, T, D]
-    w_r = gen.host_to_torch(w_r_host, shape.dtype, dev)
-    d = moe.dims(D, F, E, K, torch.bfloat16)
-    ws = moe.alloc_workspace(d, T, dev)
-    out = torch.empty((T, D), dtype=torch.bfloat16, device=dev)
-    stream = torch.cuda.current_stream(dev)
-
-    # distinct experts per step (algorithmic bytes), from the path's own routing
-    U = []
-    for i in range(POOL):
-        idx, _, _ = moe.route(d, xs[i], w_r)
-        U.append(len(set(idx.cpu().numpy().reshape(-1).tolist())))
-    U_mean = float(np.mean(U))
+    layer = Layer(moe, shape, dev, dist)
+    w1, v1, w2 = layer.w
+    pool = 4 if prefill else POOL
+    xs_host, w_r_host, xs, w_r, ws, out = layer.inputs(T, pool)
+    d, stream = layer.d, layer.stream
+    U_mean = layer.distinct_experts(xs, w_r)
 
     def step(i):
-        moe.layer_forward(d, xs[i % POOL], w_r, w1, v1, w2, out=out, ws=ws, stream=stream)
+        moe.layer_forward(d, xs[i % pool], w_r, w1, v1, w2, out=out, ws=ws, stream=stream)
 
     for i in range(args.warmup):
         step(i)
@@ -283,36 +426,10 @@ def run_ours(args):
     while time.time() - t_warm < 0.5:  # keep the GPU busy while nvidia-smi starts
         step(i)
         i += 1
-        if i % 64 == 0:
+        if i % 16 == 0:
             torch.cuda.synchronize()
-    barrier(dist)
-    torch.cuda.synchronize()
-    n_launch0 = moe.launch_count()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    wall0 = time.time()
-    ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    clocks.mark(wall0, time.time())
-    barrier(dist)
-    launches = moe.launch_count() - n_launch0
-    ms = ev0.elapsed_time(ev1) / args.steps
-    ms_max = max_over_ranks(ms, dist, dev)
-
-    # ---- the same K steps again with every kernel launch bracketed by CUDA
-    # events on its own stream: per-kernel durations for the roofline (the
-    # events cut the overlap between launches, so this pass is not `value`) ----
-    moe.profile_reset()
-    moe.profile_enable(True)
-    for i in range(args.steps):
-        step(i)
-    torch.cuda.synchronize()
-    moe.profile_enable(False)
-    kstats = moe.profile_read()
+    ms_max, launches, kstats = layer.time_steps(step, args.steps, clocks)
     clk = clocks.stop()
-    moe.check_device_errors(stream)
 
     # ---- end to end through the public API with host buffers ----
     x_pin = torch.from_numpy(xs_host.view(np.int16)).view(torch.bfloat16).pin_memory()
@@ -321,7 +438,7 @@ def run_ours(args):
     e2e_steps = max(1, args.steps // 2)
 
     def e2e_step(i):
-        x_dev.copy_(x_pin[i % POOL], non_blocking=True)
+        x_dev.copy_(x_pin[i % pool], non_blocking=True)
         moe.layer_forward(d, x_dev, w_r, w1, v1, w2, out=out, ws=ws, stream=stream)
         out_pin.copy_(out, non_blocking=True)
 
@@ -337,27 +454,33 @@ def run_ours(args):
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, dev)
 
+    # ---- secondary workloads of the same layer (rank 0's view; no timing
+    # contract): the 2048-token prefill and the decode batch sweep ----
+    extra = {}
+    if not args.no_extra and args.workload == "dbrx-decode-t1":
+        extra["prefill"] = measure_extra(layer, "dbrx-prefill-t2048", 20, 3)
+        extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5)
+                                 for t in (2, 4, 8, 16, 32, 64)]
+
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
         return
 
-    # ---- roofline of the dominant kernel ----
-    dominant = max(kstats, key=lambda k: kstats[k][1])
-    n_dom, ms_dom = kstats[dominant]
-    avg_s = ms_dom / n_dom / 1e3
-    alg = algorithmic_bytes(dominant, shape, T, U_mean)
-    peaks, peak_src = measured_peaks()
-    peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
-    achieved = alg / avg_s / 1e9
-    traffic = committed_traffic(dominant, args.workload)
     step_bytes = sum(algorithmic_bytes(k, shape, T, U_mean) for k in kstats)
-
-    us_per_token = ms_max * 1e3 / (T * world)
+    step_flops = 2.0 * T * K * 3 * D * F
+    if prefill:  # whole-job tensor throughput
+        metric, unit, hib = METRIC_PREFILL, "TFLOP/s", True
+        value = step_flops * world / (ms_max / 1e3) / 1e12
+        e2e_value = step_flops * world / (e2e_ms / 1e3) / 1e12
+    else:
+        metric, unit, hib = METRIC, UNIT, False
+        value = ms_max * 1e3 / (T * world)
+        e2e_value = e2e_ms * 1e3 / (T * world)
     line = {
-        "metric": METRIC, "value": round(us_per_token, 3), "unit": UNIT,
+        "metric": metric, "value": round(value, 3), "unit": unit,
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(ms_max, 5), "higher_is_better": False,
+        "ms_per_step": round(ms_max, 5), "higher_is_better": hib,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,0.02^2) bf16 weights, N(0,1) tokens, gap-conditioned router)",
         "config": {
@@ -365,27 +488,21 @@ def run_ours(args):
             "top_k": K, "tokens_per_step": T, "accumulate": "f32",
             "distinct_experts_per_step": U_mean,
             "l2": "inputs larger than L2: each step streams its selected experts' weights "
-                  f"({step_bytes / 1e9:.2f} GB) vs 129 MB L2",
+                  f"({U_mean * 3 * D * F * 2 / 1e9:.2f} GB) vs 129 MB L2",
             "parallelism": "replicas only" if world > 1 else "single GPU",
         },
-        "achieved_hbm_gbs_step": round(step_bytes / (ms_max / 1e3) / 1e9, 1),
-        "roofline": {
-            "kernel": dominant, "bound": "hbm", "achieved": round(achieved, 1),
-            "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
-            "peak_source": f"{peak_src} hbm_gbs" + (" (burst copy)" if peak_src == "measured" else ""),
-            "traffic": traffic, "algorithmic_bytes_per_launch": alg,
-            "avg_launch_us": round(avg_s * 1e6, 2),
-            "timing": "CUDA events around each launch on its stream, over a second "
-                      "pass of the same K steps",
-        },
-        "kernels": {k: {"launches": v[0], "avg_us": round(v[1] / v[0] * 1e3, 2),
-                        "share": round(v[1] / sum(s[1] for s in kstats.values()), 4)}
-                    for k, v in kstats.items()},
+        "roofline": (tensor_roofline(kstats, shape, T, args.workload) if prefill
+                     else hbm_roofline(kstats, shape, T, U_mean, args.workload)),
+        "kernels": kernel_table(kstats),
         "gpu_launches": int(launches),
         "clocks": clk,
-        "e2e": {"value": round(e2e_ms * 1e3 / (T * world), 3), "unit": UNIT,
+        "e2e": {"value": round(e2e_value, 3), "unit": unit,
                 "h2d_bytes_per_step": T * D * 2, "d2h_bytes_per_step": T * D * 2},
     }
+    if not prefill:
+        line["achieved_hbm_gbs_step"] = round(step_bytes / (ms_max / 1e3) / 1e9, 1)
+    if extra:
+        line["extra"] = extra
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(shape, T, xs_host, w_r_host, (w1, v1, w2),
                                             args.cpu_seconds)
@@ -405,12 +522,28 @@ def host_weights(shape, weights_dev):
 
 def cpu_baseline(shape, T, xs_host, w_r_host, weights_dev, budget_s):
     """The oracle, as it stands, on a bounded sample of the same workload:
-    whole token-steps from the same token pool, until the time budget is used."""
+    whole decode token-steps from the same token pool (prefill: tokens of the
+    first batch), until the time budget is used."""
     import oracle
 
     w1, v1, w2 = host_weights(shape, weights_dev)
+    prefill = T >= PREFILL_MIN_TOKENS
     n, t_total = 0, 0.0
-    while n < POOL and (t_total < budget_s or n == 0):
+    if prefill:
+        chunk = 16
+        while n < T and (t_total < budget_s or n == 0):
+            toks = np.arange(n, min(T, n + chunk), dtype=np.int32)
+            t0 = time.perf_counter()
+            oracle.layer_tokens(xs_host[0], w_r_host, w1, v1, w2, shape.dtype, shape.top_k,
+                                tokens=toks)
+            t_total += time.perf_counter() - t0
+            n += toks.size
+        flops = 2.0 * n * shape.top_k * 3 * shape.d_model * shape.ffn_hidden
+        return {"value": round(flops / t_total / 1e12, 6), "unit": "TFLOP/s",
+                "cores": oracle.num_threads(), "kind": "oracle",
+                "sample": f"{n} of the {T} tokens of one batch ({t_total:.1f} s of fp64 CPU work)"}
+    pool = xs_host.shape[0]
+    while n < pool and (t_total < budget_s or n == 0):
         t0 = time.perf_counter()
         oracle.layer_tokens(xs_host[n], w_r_host, w1, v1, w2, shape.dtype, shape.top_k)
         t_total += time.perf_counter() - t0
@@ -422,15 +555,19 @@ def cpu_baseline(shape, T, xs_host, w_r_host, weights_dev, budget_s):
 
 
 def run_reference(args):
-    """Reference arm: the fp64 oracle timed on this machine's host cores, one
-    token-step of the same workload per step; rank 0 only."""
+    """Reference arm: the fp64 oracle timed on this machine's host cores on the
+    same workload; rank 0 only.  Decode: one token-step per step.  Prefill: a
+    step is a bounded sample of 16 tokens of the batch, reported as
+    throughput."""
     rank, local, world = dist_env()
     if rank != 0:
         return
     import oracle
 
     shape, T = WORKLOADS[args.workload]
-    xs_host, w_r_host = token_pool(shape, T, SEED)
+    prefill = T >= PREFILL_MIN_TOKENS
+    pool = 1 if prefill else POOL
+    xs_host, w_r_host = token_pool(shape, T, SEED, pool)
     try:
         import torch
 
@@ -441,34 +578,53 @@ def run_reference(args):
         w = gen.device_expert_weights(shape, SEED, torch.device("cuda", local))
         w1, v1, w2 = host_weights(shape, w)
         del w
+        torch.cuda.empty_cache()
         src = "device-drawn seeded weights copied to host"
     except (RuntimeError, ImportError):
         w1, v1, w2 = gen.host_expert_weights(shape, SEED)
         src = "host-drawn seeded weights"
+    chunk = 16
+
+    def one(i):
+        if prefill:
+            t0 = (i * chunk) % T
+            toks = np.arange(t0, t0 + chunk, dtype=np.int32)
+            oracle.layer_tokens(xs_host[0], w_r_host, w1, v1, w2, shape.dtype, shape.top_k,
+                                tokens=toks)
+        else:
+            oracle.layer_tokens(xs_host[i % pool], w_r_host, w1, v1, w2, shape.dtype, shape.top_k)
+
     tw = time.perf_counter()
     for i in range(args.warmup):
-        oracle.layer_tokens(xs_host[i % POOL], w_r_host, w1, v1, w2, shape.dtype, shape.top_k)
+        one(i)
     per_step = (time.perf_counter() - tw) / max(1, args.warmup)
     # a bounded sample: at most ~150 s of oracle work however large K is
     steps = args.steps if per_step * args.steps <= 150 else max(3, int(150 / max(per_step, 1e-9)))
     t0 = time.perf_counter()
     for i in range(steps):
-        oracle.layer_tokens(xs_host[i % POOL], w_r_host, w1, v1, w2, shape.dtype, shape.top_k)
+        one(i)
     dt = time.perf_counter() - t0
     ms = dt / steps * 1e3
-    us_tok = ms * 1e3 / T
+    if prefill:
+        flops = 2.0 * chunk * shape.top_k * 3 * shape.d_model * shape.ffn_hidden
+        metric, unit, hib = METRIC_PREFILL, "TFLOP/s", True
+        value = round(flops / (ms / 1e3) / 1e12, 6)
+        sample = f"{steps} steps of {chunk} of the {T} tokens (of {args.steps} requested)"
+    else:
+        metric, unit, hib = METRIC, UNIT, False
+        value = round(ms * 1e3 / T, 1)
+        sample = f"{steps} token-steps of {T} token(s) (of {args.steps} requested)"
     line = {
-        "impl": "reference", "metric": METRIC, "value": round(us_tok, 1), "unit": UNIT,
+        "impl": "reference", "metric": metric, "value": value, "unit": unit,
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(ms, 3), "higher_is_better": False, "scaling": "weak",
+        "ms_per_step": round(ms, 3), "higher_is_better": hib, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": f"synthetic ({src})",
         "config": {"workload": args.workload, "d_model": shape.d_model,
                    "ffn_hidden": shape.ffn_hidden, "n_experts": shape.n_experts,
                    "top_k": shape.top_k, "tokens_per_step": T},
-        "cpu_baseline": {"value": round(us_tok, 1), "unit": UNIT, "kind": "oracle",
-                         "cores": oracle.num_threads(),
-                         "sample": f"{steps} token-steps of {T} token(s) (of {args.steps} requested)"},
-        "e2e": {"value": round(us_tok, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
+        "cpu_baseline": {"value": value, "unit": unit, "kind": "oracle",
+                         "cores": oracle.num_threads(), "sample": sample},
+        "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)

@@ -1,0 +1,460 @@
+// Grouped expert GEMMs on the tcgen05 tensor cores (prefill and larger
+// decode batches), bf16 inputs, fp32 accumulation in tensor memory.
+//
+// Table 1 notes (d),(e) of arxiv 2506.23635: every expert is three
+// D_embed x D_ffn matrices.  With the slots sorted by expert (moe_dispatch),
+// the expert FFN is two grouped GEMMs with a variable number of rows per
+// expert:
+//
+//   UP   (GLU):  h[j, f] = SiLU(x_j . W1[e,f,:]) * (x_j . V1[e,f,:])   -> bf16
+//   DOWN:        y[j, d] = h[j, :] . W2[e,d,:]                          -> fp32
+//
+// for the sorted slots j of expert e (x_j = the gathered token rows).
+// Tile = 128 slots (M, the A operand, K-major) x 256 weight rows (N, the B
+// operand, K-major) x 64 of the reduction dimension per pipeline stage.  In
+// UP the 256 weight rows are 128 rows of W1 followed by the same 128 rows of
+// V1, so one accumulator holds a (columns 0..127) and b (columns 128..255)
+// for the same f, and the GLU runs in the epilogue straight from tensor
+// memory.
+//
+// Per CTA (one per SM, persistent), 6 warps:
+//   warp 0     TMA producer (one lane): A and B tiles into a 4-stage ring,
+//              128-byte swizzle, completion on mbarriers;
+//   warp 1     tensor-memory allocator and MMA issuer (one lane):
+//              tcgen05.mma kind::f16, M=128, N=256, K=16, into one of two
+//              256-column fp32 accumulators; tcgen05.commit frees a stage
+//              and hands a finished accumulator to the epilogue;
+//   warps 2-5  epilogue: tcgen05.ld of their 32 tensor-memory lanes, GLU or
+//              plain copy, stores to global memory.
+// Tiles are numbered expert by expert (weight tile outer, slot tile inner, so
+// CTAs working at the same time share weight tiles in L2) from the device
+// resident dispatch offsets; CTA b takes tiles b, b+G, ...  No host sync.
+// Every mbarrier wait is bounded (see ptx.cuh).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "ptx.cuh"
+
+namespace moe {
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64;
+constexpr int kStages = 4;
+constexpr int kThreadsTc = 192;
+constexpr uint32_t kStageA = BM * BK * 2;           // 16 KB
+constexpr uint32_t kStageB = BN * BK * 2;           // 32 KB
+constexpr uint32_t kStageBytes = kStageA + kStageB;  // 48 KB
+constexpr uint32_t kTmemCols = 2 * BN;              // two accumulators
+constexpr size_t kTcHeaderBytes = 2048;
+constexpr size_t kSmemTc = 1024 /*align slack*/ + kStages * kStageBytes + kTcHeaderBytes;
+
+enum Mode { kUp = 0, kDown = 1 };
+
+struct TcHeader {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint64_t done;
+    uint32_t tmem_base;
+    int tprefix[257];  // tile prefix over experts
+};
+static_assert(sizeof(TcHeader) <= kTcHeaderBytes, "tcgen05 kernel header too large");
+
+// ---- tcgen05 wrappers --------------------------------------------------------
+
+__device__ __forceinline__ void tmem_alloc(uint32_t *holder, uint32_t cols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     ptx::smem_u32(holder)),
+                 "r"(cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, both K-major, one instruction of K=16.
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on an mbarrier once all earlier tcgen05 ops of this thread finish.
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            ptx::smem_u32(bar))
+        : "memory");
+}
+
+// 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand written by TMA with the
+// 128-byte swizzle; 8-row groups 1024 bytes apart; descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// kind::f16 instruction descriptor: bf16 A and B, fp32 D, both K-major.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                            ((uint32_t)(BM >> 4) << 24);
+
+// ---- tile schedule -------------------------------------------------------------
+
+// tprefix[e] = sum over earlier experts of ceil(n_e / BM) * n_tiles_n.
+__device__ void tile_prefix(const int32_t *offsets, int E, int S, int ntn, int *tprefix,
+                            unsigned *err) {
+    const int lane = threadIdx.x & 31;
+    int run = 0;
+    for (int base = 0; base < E; base += 32) {
+        const int e = base + lane;
+        int c = 0;
+        if (e < E) {
+            const int lo = offsets[e], hi = offsets[e + 1];
+            if (lo < 0 || hi < lo || hi > S) set_error(err, kErrIndex);
+            else c = ((hi - lo + BM - 1) / BM) * ntn;
+        }
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (e < E) tprefix[e] = run + incl - c;
+        run += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) tprefix[E] = run;
+}
+
+struct Tile {
+    int e, mt, nt, row0, rows;  // rows: valid slots in this M tile
+};
+
+__device__ __forceinline__ Tile tile_of(const int *tprefix, const int32_t *offsets, int E, int ntn,
+                                        int u) {
+    Tile t;
+    t.e = chunk_expert(tprefix, E, u);
+    const int r = u - tprefix[t.e];
+    const int n_e = offsets[t.e + 1] - offsets[t.e];
+    const int mtiles = (n_e + BM - 1) / BM;
+    t.nt = r / mtiles;
+    t.mt = r - t.nt * mtiles;
+    t.row0 = offsets[t.e] + t.mt * BM;
+    t.rows = min(BM, n_e - t.mt * BM);
+    return t;
+}
+
+// ---- the kernel ------------------------------------------------------------------
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreadsTc, 1)
+k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+          const __grid_constant__ CUtensorMap tmB1, const int32_t *__restrict__ offsets, int E,
+          int S, int Kdim, int Nw, bf16 *__restrict__ h_out, float *__restrict__ y_out,
+          unsigned *err) {
+    // Kdim: reduction length (D for UP, F for DOWN); Nw: weight rows per
+    // expert (F for UP, D for DOWN) = the output width.
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    TcHeader *hd = reinterpret_cast<TcHeader *>(smem + kStages * kStageBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int ntn = MODE == kUp ? (Nw + 127) / 128 : (Nw + BN - 1) / BN;
+    const int nk = (Kdim + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&hd->full[s], 1);
+            ptx::mbar_init(&hd->empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(&hd->tfull[b], 1);
+            ptx::mbar_init(&hd->tempty[b], 4);
+        }
+        ptx::mbar_init(&hd->done, 1);
+        ptx::fence_barrier_init();
+        ptx::prefetch_tmap(&tmA);
+        ptx::prefetch_tmap(&tmB0);
+        if (MODE == kUp) ptx::prefetch_tmap(&tmB1);
+    }
+    if (warp == 1) tmem_alloc(&hd->tmem_base, kTmemCols);
+    ptx::grid_dependency_wait();  // offsets and the A operand come from earlier kernels
+    if (warp == 2) tile_prefix(offsets, E, S, ntn, hd->tprefix, err);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = hd->tmem_base;
+    const int n_tiles = hd->tprefix[E];
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            const uint64_t pol_a = ptx::policy_evict_last();
+            const uint64_t pol_b = ptx::policy_evict_first();
+            uint32_t it = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; u < n_tiles && ok; u += gridDim.x) {
+                const Tile t = tile_of(hd->tprefix, offsets, E, ntn, u);
+                const int brow = MODE == kUp ? t.e * Nw + t.nt * 128 : t.e * Nw + t.nt * BN;
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const uint32_t s = it % kStages, ph = (it / kStages) & 1;
+                    if (!(ok = ptx::mbar_wait(&hd->empty[s], ph ^ 1, err))) break;
+                    unsigned char *sa = smem + s * kStageBytes;
+                    unsigned char *sb = sa + kStageA;
+                    ptx::mbar_arrive_expect_tx(&hd->full[s], kStageBytes);
+                    ptx::tma_load_2d(sa, &tmA, kb * BK, t.row0, &hd->full[s], pol_a);
+                    if (MODE == kUp) {
+                        ptx::tma_load_2d(sb, &tmB0, kb * BK, brow, &hd->full[s], pol_b);
+                        ptx::tma_load_2d(sb + kStageB / 2, &tmB1, kb * BK, brow, &hd->full[s],
+                                         pol_b);
+                    } else {
+                        ptx::tma_load_2d(sb, &tmB0, kb * BK, brow, &hd->full[s], pol_b);
+                    }
+                }
+            }
+            // let loads still in flight land before the block can exit
+            for (uint32_t k = (it > kStages ? it - kStages : 0); k < it; ++k)
+                ptx::mbar_wait(&hd->full[k % kStages], (k / kStages) & 1, err);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            uint32_t it = 0, tl = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; u < n_tiles && ok; u += gridDim.x, ++tl) {
+                const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
+                if (!(ok = ptx::mbar_wait(&hd->tempty[acc], aph ^ 1, err))) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + acc * BN;
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const uint32_t s = it % kStages, ph = (it / kStages) & 1;
+                    if (!(ok = ptx::mbar_wait(&hd->full[s], ph, err))) break;
+                    tc_fence_after();
+                    const uint32_t sa = ptx::smem_u32(smem + s * kStageBytes);
+                    const uint64_t adesc = smem_desc(sa), bdesc = smem_desc(sa + kStageA);
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, kIdesc,
+                                 (kb | kk) != 0 ? 1u : 0u);
+                    mma_commit(&hd->empty[s]);  // stage free once these MMAs finish
+                }
+                if (ok) mma_commit(&hd->tfull[acc]);
+            }
+            // every MMA issued by this thread has completed once `done` flips
+            mma_commit(&hd->done);
+            ptx::mbar_wait(&hd->done, 0, err);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int q = warp & 3;          // tensor-memory lane quarter of this warp
+        const int m = q * 32 + lane;     // row of the tile = slot offset
+        uint32_t tl = 0;
+        for (int u = blockIdx.x; u < n_tiles; u += gridDim.x, ++tl) {
+            const Tile t = tile_of(hd->tprefix, offsets, E, ntn, u);
+            const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
+            if (!ptx::mbar_wait(&hd->tfull[acc], aph, err)) break;
+            tc_fence_after();
+            const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + acc * BN;
+            const bool row_ok = m < t.rows;
+            const size_t j = (size_t)t.row0 + m;
+            if (MODE == kUp) {
+                const int f0 = t.nt * 128;
+#pragma unroll 1
+                for (int c = 0; c < 128; c += 32) {
+                    float a[32], b[32];
+                    tmem_ld32(base + c, a);
+                    tmem_ld32(base + 128 + c, b);
+                    tmem_ld_wait();
+                    if (row_ok) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float h0 = silu(a[2 * i]) * b[2 * i];
+                            const float h1 = silu(a[2 * i + 1]) * b[2 * i + 1];
+                            const __nv_bfloat162 p2 = __floats2bfloat162_rn(h0, h1);
+                            pk[i] = *reinterpret_cast<const uint32_t *>(&p2);
+                        }
+                        bf16 *dst = h_out + j * Nw + f0 + c;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)  // 8 columns per 16-byte store
+                            if (f0 + c + g * 8 < Nw)
+                                *reinterpret_cast<uint4 *>(dst + g * 8) =
+                                    make_uint4(pk[4 * g], pk[4 * g + 1], pk[4 * g + 2], pk[4 * g + 3]);
+                    }
+                }
+            } else {
+                const int d0 = t.nt * BN;
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    float v[32];
+                    tmem_ld32(base + c, v);
+                    tmem_ld_wait();
+                    if (row_ok) {
+                        float *dst = y_out + j * Nw + d0 + c;
+#pragma unroll
+                        for (int g = 0; g < 8; ++g)  // 4 columns per 16-byte store
+                            if (d0 + c + g * 4 < Nw)
+                                *reinterpret_cast<float4 *>(dst + g * 4) =
+                                    make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&hd->tempty[acc]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// ---- gather of the A operand: x_sorted[j, :] = x[perm[j] / K, :] ----------------
+
+__global__ void __launch_bounds__(256)
+k_gather_rows(int S, int D, int K, const bf16 *__restrict__ x, const int32_t *__restrict__ perm,
+              bf16 *__restrict__ xs, unsigned *err) {
+    ptx::grid_dependency_wait();
+    const int nv = D >> 3;  // 16-byte vectors per row
+    const long long total = (long long)S * nv;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int j = (int)(i / nv), v = (int)(i - (long long)j * nv);
+        int slot = perm[j];
+        if (slot < 0 || slot >= S) {
+            set_error(err, kErrIndex);
+            slot = 0;
+        }
+        const uint4 val = __ldg(reinterpret_cast<const uint4 *>(x + (size_t)(slot / K) * D) + v);
+        reinterpret_cast<uint4 *>(xs + (size_t)j * D)[v] = val;
+    }
+}
+
+// ---- host: tensor maps -----------------------------------------------------------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 row-major [rows, cols] tensor, box {64 columns, box_rows}, 128-byte
+// swizzle, zero fill outside the tensor.
+bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int MODE>
+cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUtensorMap &b1,
+                        const int32_t *offsets, int E, int S, int Kdim, int Nw, bf16 *h_out,
+                        float *y_out, cudaStream_t st) {
+    const void *kern = (const void *)k_gemm_tc<MODE>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemTc);
+    if (e != cudaSuccess) return e;
+    unsigned *err = device_info().err;
+    CUtensorMap ma = a, mb0 = b0, mb1 = b1;
+    void *args[] = {&ma, &mb0, &mb1, &offsets, &E, &S, &Kdim, &Nw, &h_out, &y_out, &err};
+    LaunchScope ls(MODE == kUp ? "gemm_up_glu_tc" : "gemm_down_tc", st);
+    return launch_pdl(kern, dim3(device_info().sm_count), dim3(kThreadsTc), kSmemTc, st, args);
+}
+
+}  // namespace
+
+bool tc_path_ok(const moe_dims &d) {
+    return d.w_dtype == MOE_BF16 && d.x_dtype == MOE_BF16 && encode_fn() != nullptr;
+}
+
+cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const int32_t *perm,
+                               void *x_sorted, cudaStream_t st) {
+    const int S = T * d.top_k;
+    const long long total = (long long)S * (d.d_model / 8);
+    const long long cap = (long long)device_info().sm_count * 8;
+    const int grid = (int)std::max(1LL, std::min((total + 255) / 256, cap));
+    int Sv = S, D = d.d_model, K = d.top_k;
+    const bf16 *xp = static_cast<const bf16 *>(x);
+    bf16 *xs = static_cast<bf16 *>(x_sorted);
+    unsigned *err = device_info().err;
+    void *args[] = {&Sv, &D, &K, &xp, &perm, &xs, &err};
+    LaunchScope ls("gather_rows", st);
+    return launch_pdl((const void *)k_gather_rows, dim3(grid), dim3(256), 0, st, args);
+}
+
+cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, const int32_t *offsets,
+                              const void *w1, const void *v1, void *h, cudaStream_t st) {
+    const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
+    CUtensorMap a, b0, b1;
+    if (!make_map(&a, x_sorted, (uint64_t)S, (uint64_t)D, BM) ||
+        !make_map(&b0, w1, (uint64_t)E * F, (uint64_t)D, 128) ||
+        !make_map(&b1, v1, (uint64_t)E * F, (uint64_t)D, 128))
+        return cudaErrorInvalidValue;
+    return launch_gemm<kUp>(a, b0, b1, offsets, E, S, D, F, static_cast<bf16 *>(h), nullptr, st);
+}
+
+cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
+                                const void *w2, float *y_sorted, cudaStream_t st) {
+    const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
+    CUtensorMap a, b0;
+    if (!make_map(&a, h, (uint64_t)S, (uint64_t)F, BM) ||
+        !make_map(&b0, w2, (uint64_t)E * D, (uint64_t)F, BN))
+        return cudaErrorInvalidValue;
+    return launch_gemm<kDown>(a, b0, b0, offsets, E, S, F, D, nullptr, y_sorted, st);
+}
+
+}  // namespace moe

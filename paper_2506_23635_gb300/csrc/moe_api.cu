@@ -523,8 +523,14 @@ WsLayout ws_layout(const moe_dims &d, int64_t T) {
     L.offsets = o; o += up(((size_t)d.n_experts + 1) * 4);
     L.perm = o; o += up(S * 4);
     L.inv_perm = o; o += up(S * 4);
-    L.h = o; o += up(S * d.ffn_hidden * 4);
-    L.y = o; o += (T > kFusedCombineMaxTokens) ? up(S * d.d_model * 4) : 0;
+    const bool bf = d.w_dtype == MOE_BF16;
+    // GLU hidden vectors: bf16 on the bf16 paths, fp32 on the fp32 path
+    L.h = o; o += up(S * d.ffn_hidden * (bf ? 2 : 4));
+    // gathered token rows (tensor-core path, bf16 only)
+    L.xs = o; o += bf ? up(S * d.d_model * 2) : 0;
+    // ungated expert outputs: the tensor-core path, and the fp32 path above
+    // the fused-combine limit
+    L.y = o; o += (bf || T > kFusedCombineMaxTokens) ? up(S * d.d_model * 4) : 0;
     L.total = o;
     return L;
 }
@@ -649,6 +655,10 @@ cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t 
     return launch_combine<float, float>(d, T, y, inv, gate, res, out, st);
 }
 
+bool use_stream_path(const moe_dims &d, int T) {
+    return T <= kStreamMaxTokens && stream_path_ok(d, T);
+}
+
 template <typename P> P *at(void *ws, size_t off) {
     return reinterpret_cast<P *>(static_cast<char *>(ws) + off);
 }
@@ -707,12 +717,20 @@ moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x, const 
     cudaStream_t st = (cudaStream_t)stream;
     float *h = at<float>(ws, L.h);
     cudaError_t e;
-    if (stream_path_ok(*dims, T)) {
+    if (use_stream_path(*dims, T)) {
         // bf16 weights, few slots: bulk-copy pipelined kernels, bf16 h
         e = launch_up_glu_stream(*dims, T, x, perm, offsets, w1, v1, h, st);
         if (e == cudaSuccess)
             e = launch_down_stream(*dims, T, h, offsets, nullptr, w2, nullptr, nullptr, nullptr,
                                    y_sorted, false, st);
+        return cuda_status(e);
+    }
+    if (tc_path_ok(*dims)) {
+        // bf16 weights: gather the token rows, then the two tcgen05 GEMMs
+        void *xs = at<void>(ws, L.xs);
+        e = launch_gather_rows(*dims, T, x, perm, xs, st);
+        if (e == cudaSuccess) e = launch_gemm_up_tc(*dims, T, xs, offsets, w1, v1, h, st);
+        if (e == cudaSuccess) e = launch_gemm_down_tc(*dims, T, h, offsets, w2, y_sorted, st);
         return cuda_status(e);
     }
     e = launch_up_glu_gemv(*dims, T, x, perm, offsets, w1, v1, h, st);
@@ -766,13 +784,24 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
         if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
     }
     if (e != cudaSuccess) return MOE_ERR_CUDA;
-    if (stream_path_ok(d, T)) {
+    if (use_stream_path(d, T)) {
         // decode, bf16: bulk-copy pipelined kernels, combine fused into the
-        // down projection (T*K <= 64 slots, so T <= 64)
+        // down projection
         e = launch_up_glu_stream(d, T, x, perm, offsets, w1, v1, h, st);
         if (e == cudaSuccess)
             e = launch_down_stream(d, T, h, offsets, inv, w2, gate, residual_opt, out, nullptr,
                                    true, st);
+        return cuda_status(e);
+    }
+    if (tc_path_ok(d)) {
+        // bf16: gathered token rows, tcgen05 GEMMs (GLU fused into the up
+        // projection's epilogue), then the gated combine
+        void *xs = at<void>(ws, L.xs);
+        float *y = at<float>(ws, L.y);
+        e = launch_gather_rows(d, T, x, perm, xs, st);
+        if (e == cudaSuccess) e = launch_gemm_up_tc(d, T, xs, offsets, w1, v1, h, st);
+        if (e == cudaSuccess) e = launch_gemm_down_tc(d, T, h, offsets, w2, y, st);
+        if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st);
         return cuda_status(e);
     }
     e = launch_up_glu_gemv(d, T, x, perm, offsets, w1, v1, h, st);

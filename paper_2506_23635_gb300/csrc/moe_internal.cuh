@@ -146,7 +146,7 @@ struct LaunchScope {
 
 // Workspace layout of moe_layer_forward / moe_expert_ffn for T tokens.
 struct WsLayout {
-    size_t idx, gate, counts, offsets, perm, inv_perm, h, y, total;
+    size_t idx, gate, counts, offsets, perm, inv_perm, h, xs, y, total;
 };
 WsLayout ws_layout(const moe_dims &d, int64_t T);
 
@@ -181,9 +181,21 @@ inline cudaError_t launch_pdl(const void *func, dim3 grid, dim3 block, size_t sm
 
 constexpr int kFusedCombineMaxTokens = 64;
 
+// tcgen05 grouped GEMMs (ffn_tc.cu), bf16 only; h is bf16, y_sorted fp32.
+bool tc_path_ok(const moe_dims &d);
+cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const int32_t *perm,
+                               void *x_sorted, cudaStream_t st);
+cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
+                              const int32_t *offsets, const void *w1, const void *v1, void *h,
+                              cudaStream_t st);
+cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
+                                const void *w2, float *y_sorted, cudaStream_t st);
+
 // Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
-// kStreamMaxSlots slots; the GLU hidden vectors h are bf16.
+// kStreamMaxSlots slots; the GLU hidden vectors h are bf16.  Batches of at
+// most kStreamMaxTokens tokens take them; larger ones take the tcgen05 GEMMs.
 constexpr int kStreamMaxSlots = 64;
+constexpr int kStreamMaxTokens = 1;
 bool stream_path_ok(const moe_dims &d, int T);
 cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
                                  const int32_t *offsets, const void *w1, const void *v1, void *h,
