@@ -195,9 +195,16 @@ def test_bad_arguments_with_real_tensors():
         m.route(bad, x, w)
 
 
-def test_launch_count_and_profile():
+@pytest.mark.parametrize("T,kernels", [
+    (1, {"route_dispatch_small", "up_glu_stream", "down_combine_stream"}),
+    (3, {"route_dispatch_small", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
+    (9, {"route", "dispatch", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
+])
+def test_launch_count_and_profile(T, kernels):
+    """One token: fused routing + the two streaming kernels; more tokens: the
+    tensor-core path.  Every launch is counted and event-timed."""
     m = moe()
-    L = _host((64, 64, 4, 2, 3, "bf16"))
+    L = _host((64, 64, 4, 2, T, "bf16"))
     d = _dims(m, L.shape)
     x, w_r, w1, v1, w2 = _devlayer(L)
     m.layer_forward(d, x, w_r, w1, v1, w2)
@@ -207,8 +214,7 @@ def test_launch_count_and_profile():
     m.profile_enable(True)
     m.layer_forward(d, x, w_r, w1, v1, w2)
     m.profile_enable(False)
-    stats = m.profile_read()
-    # tiny batch: fused route+dispatch, up projection, down projection + combine
-    assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == 3
-    assert set(stats) == {"route_dispatch_small", "up_glu_stream", "down_combine_stream"}
+    stats = {k: v for k, v in m.profile_read().items() if v[0] > 0}
+    assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == len(kernels)
+    assert set(stats) == kernels
     assert all(v[1] > 0 for v in stats.values())
