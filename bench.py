@@ -391,6 +391,88 @@ def measure_extra(layer, workload, steps, warmup):
     return r
 
 
+def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True):
+    """The 16-layer DBRX-shaped stack (about 101 GB of bf16 weights resident,
+    each layer independently seeded), x_{l+1} = x_l + MoE_l(RMSNorm0(x_l)) with
+    an fp32 residual stream; decode at batch 1 and 8 for 64 consecutive steps,
+    each step a fresh seeded batch of tokens.  Reports per-token latency over
+    the stack; with `graph`, also the same steps replayed from one CUDA graph
+    capture of a whole step."""
+    import torch
+
+    shape = gen.DBRX
+    D, F, E, K = shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k
+    layers = []
+    for l in range(n_layers):
+        w_r = gen.host_to_torch(gen.host_normal((D, E), gen.W_STD, "bf16", SEED, "stack-w_r", l),
+                                "bf16", dev)
+        layers.append((w_r,) + gen.device_expert_weights(shape, SEED + 1 + l, dev, layer=l))
+    sw = moe.StackWeights(layers)
+    d = moe.dims(D, F, E, K, torch.bfloat16, torch.bfloat16, torch.float32)
+    stream = torch.cuda.current_stream(dev)
+    res = {"layers": n_layers, "resident_weight_gb": round(n_layers * 3 * E * D * F * 2 / 1e9, 2),
+           "steps": steps}
+    for T in batches:
+        xs = torch.stack([gen.host_to_torch(gen.host_normal((T, D), 1.0, "bf16", SEED, "stack-x",
+                                                            T, s), "bf16", dev).float()
+                          for s in range(steps)])
+        resid = torch.empty((T, D), dtype=torch.float32, device=dev)
+        ws = torch.empty(moe.stack_workspace_size(d, T), dtype=torch.uint8, device=dev)
+
+        def step(s):
+            resid.copy_(xs[s % steps])
+            moe.stack_forward(d, sw, resid, ws=ws, stream=stream)
+
+        for s in range(3):
+            step(s)
+        moe.check_device_errors(stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(steps):
+            step(s)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        moe.check_device_errors(stream)
+        ms = e0.elapsed_time(e1) / steps
+        r = {"ms_per_step": round(ms, 4), "us_per_token_step": round(ms * 1e3 / T, 2),
+             "tokens_per_s": round(T / (ms / 1e3), 1)}
+        if graph:
+            try:
+                g = torch.cuda.CUDAGraph()
+                xin = torch.empty_like(resid)
+                gs = torch.cuda.Stream(dev)
+                gs.wait_stream(stream)
+                with torch.cuda.stream(gs):
+                    for _ in range(2):
+                        resid.copy_(xin)
+                        moe.stack_forward(d, sw, resid, ws=ws, stream=gs)
+                torch.cuda.synchronize()
+                with torch.cuda.graph(g, stream=gs):
+                    resid.copy_(xin)
+                    moe.stack_forward(d, sw, resid, ws=ws, stream=gs)
+                for s in range(3):
+                    xin.copy_(xs[s])
+                    g.replay()
+                torch.cuda.synchronize()
+                e0.record(stream)
+                for s in range(steps):
+                    xin.copy_(xs[s % steps])
+                    g.replay()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                moe.check_device_errors(stream)
+                gms = e0.elapsed_time(e1) / steps
+                r["graph"] = {"ms_per_step": round(gms, 4),
+                              "us_per_token_step": round(gms * 1e3 / T, 2)}
+            except Exception as exc:  # report, keep the plain numbers
+                r["graph"] = {"error": str(exc)[:200]}
+        res[f"batch{T}"] = r
+    del layers, sw
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_ours(args):
     import torch
 
@@ -461,6 +543,7 @@ def run_ours(args):
         extra["prefill"] = measure_extra(layer, "dbrx-prefill-t2048", 20, 3)
         extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5)
                                  for t in (2, 4, 8, 16, 32, 64)]
+        extra["stack"] = measure_stack(moe, dev)
 
     if rank != 0:
         if dist is not None:

@@ -76,8 +76,8 @@ typedef struct {
     int32_t n_experts;  /* E, Sec. 2.1 (16 for DBRX) */
     int32_t top_k;      /* K, Sec. 2.1 (4 for DBRX) */
     int32_t w_dtype;    /* moe_dtype of w_router, w1, v1, w2 */
-    int32_t x_dtype;    /* moe_dtype of x and of a residual */
-    int32_t out_dtype;  /* moe_dtype of out */
+    int32_t x_dtype;    /* moe_dtype of x */
+    int32_t out_dtype;  /* moe_dtype of out and of a residual */
 } moe_dims;
 
 /* Bytes of workspace moe_layer_forward and moe_expert_ffn need for up to
@@ -131,7 +131,7 @@ moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x,
 
 /* Step 4 -- weighted combine (Sec. 4.2 "weighted sum"; Sec. 4.3).
  *   y_sorted     [T*K, D] float32;  inv_perm [T*K];  topk_gate [T, K]
- *   residual_opt [T, D]   x_dtype, added if non-NULL
+ *   residual_opt [T, D]   out_dtype, added if non-NULL; may be `out` itself
  *   out          [T, D]   out_dtype
  *   out[t,:] = residual[t,:] + sum_{k=0..K-1} gate[t,k] * y_sorted[inv_perm[t*K+k],:]
  * summed in ascending k. */
@@ -143,7 +143,9 @@ moe_status moe_combine(const moe_dims *dims, int32_t T, const float *y_sorted,
 /* The whole layer: route, dispatch, expert FFN and combine, with the gate
  * and combine fused into the expert kernels where the token count allows.
  *   x [T,D], w_router [D,E], w1/v1 [E,F,D], w2 [E,D,F] as above;
- *   residual_opt [T,D] x_dtype or NULL;  out [T,D] out_dtype;
+ *   residual_opt [T,D] out_dtype or NULL (may be `out` itself: each
+ *   residual element is read before the same output element is written);
+ *   out [T,D] out_dtype;
  *   ws  workspace of at least moe_workspace_size(dims, T) bytes.
  * No host synchronisation; capturable in a CUDA graph. */
 moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x,
@@ -151,6 +153,31 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x,
                              const void *v1, const void *w2,
                              const void *residual_opt, void *out, void *ws,
                              size_t ws_bytes, moe_stream_t stream);
+
+/* ---- stack of layers (decode through consecutive MoE blocks) -------------
+ * The paper runs DBRX's 40 decoder layers (Table 1); a stack of MoE blocks
+ * needs the glue between them, which the paper does not print.  Reading
+ * used here: a parameter-free RMS pre-norm and a residual add,
+ *   x_{l+1} = x_l + MoE_l( RMSNorm0(x_l) ),
+ *   RMSNorm0(r) = r / sqrt(mean(r^2) + eps),
+ * with the residual stream in out_dtype (fp32 for the DBRX stack) and the
+ * normalised layer input rounded to x_dtype.
+ *
+ * moe_prenorm: x_norm[t,:] = RMSNorm0(resid[t,:]).
+ *   resid [T, D] out_dtype;  x_norm [T, D] x_dtype;  eps > 0.
+ * moe_stack_workspace_size: bytes moe_stack_forward needs for max_tokens.
+ * moe_stack_forward: applies n_layers layers in order to resid in place.
+ *   w_router, w1, v1, w2: HOST arrays of n_layers DEVICE pointers, each
+ *   laid out as for moe_layer_forward;  resid [T, D] out_dtype, in/out. */
+moe_status moe_prenorm(const moe_dims *dims, int32_t T, const void *resid,
+                       void *x_norm, float eps, moe_stream_t stream);
+moe_status moe_stack_workspace_size(const moe_dims *dims, int32_t max_tokens,
+                                    size_t *bytes);
+moe_status moe_stack_forward(const moe_dims *dims, int32_t n_layers, int32_t T,
+                             const void *const *w_router, const void *const *w1,
+                             const void *const *v1, const void *const *w2,
+                             void *resid, float eps, void *ws, size_t ws_bytes,
+                             moe_stream_t stream);
 
 /* ---- layer without a caller workspace ----------------------------------
  * The paper has no counterpart of this entry point; it serves callers that

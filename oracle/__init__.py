@@ -24,7 +24,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "moe_oracle.c")
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "libmoe_oracle.so")
-_DT = {"f32": 0, "bf16": 1}
+_DT = {"f32": 0, "bf16": 1, "f64": 2}
 _lock = threading.Lock()
 _lib = None
 
@@ -55,6 +55,8 @@ def _bind(path: str) -> ctypes.CDLL:
     lib.orc_layer_dense_masked.argtypes = [I, I, I, I, I, P, I, P, P, P, P, I, P]
     lib.orc_layer_dense_masked.restype = I
     lib.orc_num_threads.restype = I
+    lib.orc_rmsnorm0.argtypes = [I, I, P, ctypes.c_double, P]
+    lib.orc_round_bf16.argtypes = [ctypes.c_size_t, P, P]
     return lib
 
 
@@ -67,7 +69,7 @@ def _p(a: np.ndarray):
 
 
 def _storage(a: np.ndarray, dtype: str) -> np.ndarray:
-    return _c(a, np.uint16 if dtype == "bf16" else np.float32)
+    return _c(a, {"bf16": np.uint16, "f32": np.float32, "f64": np.float64}[dtype])
 
 
 class OracleLib:
@@ -81,13 +83,14 @@ class OracleLib:
         """Threads the oracle's parallel loops use."""
         return int(self.lib.orc_num_threads())
 
-    def router_logits(self, x, w_r, dtype: str) -> np.ndarray:
+    def router_logits(self, x, w_r, dtype: str, x_dtype: str = None) -> np.ndarray:
         """logits[t,e] = sum_d x[t,d] W_r[d,e] in fp64 (no bias)."""
-        x, w_r = _storage(x, dtype), _storage(w_r, dtype)
+        xdt = dtype if x_dtype is None else x_dtype
+        x, w_r = _storage(x, xdt), _storage(w_r, dtype)
         T, D = x.shape
         E = w_r.shape[1]
         out = np.empty((T, E), np.float64)
-        self.lib.orc_router_logits(T, D, E, _p(x), _DT[dtype], _p(w_r), _DT[dtype],
+        self.lib.orc_router_logits(T, D, E, _p(x), _DT[xdt], _p(w_r), _DT[dtype],
                                    _p(out))
         return out
 
@@ -129,13 +132,15 @@ class OracleLib:
         return h, y
 
     def layer_tokens(self, x, w_r, w1, v1, w2, dtype: str, top_k: int,
-                     tokens=None, residual=None):
+                     tokens=None, residual=None, x_dtype: str = None):
         """The sparse MoE layer for the listed tokens (default: all).
 
         Returns (out [n,D] f64, idx [n,K] i32, gate [n,K] f64).  ``residual``
-        ([T,D] float64) is added to each output row when given.
+        ([T,D] float64) is added to each output row when given.  ``x_dtype``
+        (default: ``dtype``) is the storage type of x, "f64" included.
         """
-        x = _storage(x, dtype)
+        xdt = dtype if x_dtype is None else x_dtype
+        x = _storage(x, xdt)
         w_r, w1, v1, w2 = (_storage(a, dtype) for a in (w_r, w1, v1, w2))
         T, D = x.shape
         E, F, _ = w1.shape
@@ -146,11 +151,62 @@ class OracleLib:
         gate = np.empty((n, top_k), np.float64)
         res = None if residual is None else _c(residual, np.float64)
         rc = self.lib.orc_layer_tokens(T, D, F, E, top_k, n, _p(tok), _p(x),
-                                       _DT[dtype], _p(w_r), _p(w1), _p(v1), _p(w2),
+                                       _DT[xdt], _p(w_r), _p(w1), _p(v1), _p(w2),
                                        _DT[dtype], _p(res), _p(out), _p(idx), _p(gate))
         if rc != 0:
             raise ValueError("token index out of range")
         return out, idx, gate
+
+    def rmsnorm0(self, x64: np.ndarray, eps: float) -> np.ndarray:
+        """Parameter-free RMS pre-norm of each row (fp64)."""
+        x = _c(x64, np.float64)
+        T, D = x.shape
+        out = np.empty_like(x)
+        self.lib.orc_rmsnorm0(T, D, _p(x), float(eps), _p(out))
+        return out
+
+    def round_bf16(self, x64: np.ndarray) -> np.ndarray:
+        """Nearest bfloat16 value of each element (ties to even), as fp64."""
+        x = _c(x64, np.float64)
+        out = np.empty_like(x)
+        self.lib.orc_round_bf16(x.size, _p(x), _p(out))
+        return out
+
+    def stack_tokens(self, x0, layers, dtype: str, top_k: int, eps: float,
+                     layer_callback=None):
+        """Tokens through stacked layers: x_{l+1} = x_l + MoE_l(RMSNorm0(x_l)).
+
+        x0: [n, D] token rows (storage ``dtype``, widened exactly); layers: a
+        sequence of (w_r, w1, v1, w2) storage arrays, or a callable l -> that
+        tuple (so a caller can bring one layer at a time to the host).
+        Returns the fp64 residual stream after the last layer and an array
+        [n_layers, n] of each token's gap between its K-th and (K+1)-th router
+        logit divided by the RMS of its logits at that layer (how well
+        conditioned the routing was; +inf when K = E)."""
+        x = _to_f64(x0, dtype) if dtype != "f64" else _c(x0, np.float64)
+        n_layers = len(layers) if not callable(layers) else None
+        gaps = []
+        l = 0
+        while n_layers is None or l < n_layers:
+            lw = layers(l) if callable(layers) else layers[l]
+            if lw is None:
+                break
+            w_r, w1, v1, w2 = lw
+            xn = self.rmsnorm0(x, eps)
+            if dtype == "bf16":  # the layer input is stored in bf16 (reading C9)
+                xn = self.round_bf16(xn)
+            out, idx, _ = self.layer_tokens(xn, w_r, w1, v1, w2, dtype, top_k, residual=x,
+                                            x_dtype="f64")
+            logits = self.router_logits(xn, w_r, dtype, x_dtype="f64")
+            if top_k >= logits.shape[1]:
+                gaps.append(np.full(logits.shape[0], np.inf))
+            else:
+                srt = -np.sort(-logits, axis=1)
+                rms = np.sqrt(np.mean(logits * logits, axis=1))
+                gaps.append((srt[:, top_k - 1] - srt[:, top_k]) / rms)
+            x = out
+            l += 1
+        return x, np.array(gaps)
 
     def layer_dense_masked(self, x, w_r, w1, v1, w2, dtype: str,
                            top_k: int) -> np.ndarray:
@@ -232,6 +288,18 @@ def layer_dense_masked(*a, **k):
 
 def layer_steps(*a, **k):
     return default().layer_steps(*a, **k)
+
+
+def stack_tokens(*a, **k):
+    return default().stack_tokens(*a, **k)
+
+
+def rmsnorm0(*a, **k):
+    return default().rmsnorm0(*a, **k)
+
+
+def round_bf16(*a, **k):
+    return default().round_bf16(*a, **k)
 
 
 def _to_f64(a, dtype):

@@ -53,7 +53,10 @@ static double orc_load(const void *base, int dtype, size_t i)
     return (double)((const float *)base)[i];
 }
 
-static size_t orc_elem_size(int dtype) { return dtype == ORC_BF16 ? 2u : 4u; }
+static size_t orc_elem_size(int dtype)
+{
+    return dtype == ORC_BF16 ? 2u : (dtype == ORC_F64 ? 8u : 4u);
+}
 
 /* Router logits, reading C1: a plain product with no bias. */
 void orc_router_logits(int T, int D, int E, const void *x, int xdt,
@@ -235,6 +238,37 @@ int orc_layer_dense_masked(int T, int D, int F, int E, int K, const void *x,
     }
     free(xt); free(lg); free(mask); free(h); free(y); free(idx); free(g);
     return 0;
+}
+
+/* Parameter-free RMS pre-norm between stacked layers (reading C9; the paper
+ * does not print the glue between MoE blocks):
+ * out[t,:] = x[t,:] / sqrt(mean_d x[t,d]^2 + eps). */
+void orc_rmsnorm0(int T, int D, const double *x, double eps, double *out)
+{
+    for (int t = 0; t < T; ++t) {
+        const double *r = x + (size_t)t * D;
+        double ss = 0.0;
+        for (int d = 0; d < D; ++d) ss += r[d] * r[d];
+        const double s = 1.0 / sqrt(ss / D + eps);
+        for (int d = 0; d < D; ++d) out[(size_t)t * D + d] = r[d] * s;
+    }
+}
+
+/* Storage rounding of an activation to bfloat16 (8 significant bits): the
+ * representable value nearest to v, ties to the one with an even last
+ * significant bit.  Used for the stacked layers' normalised input, which the
+ * layer stores in bf16 (the paper's inference keeps activations in bf16,
+ * Sec. 5.1).  Finite normal range only. */
+void orc_round_bf16(size_t n, const double *in, double *out)
+{
+    for (size_t i = 0; i < n; ++i) {
+        const double v = in[i];
+        if (v == 0.0 || !isfinite(v)) { out[i] = v; continue; }
+        int e;
+        frexp(v, &e);                      /* |v| = m 2^e, m in [0.5, 1) */
+        const double ulp = ldexp(1.0, e - 8);
+        out[i] = nearbyint(v / ulp) * ulp; /* default mode: ties to even */
+    }
 }
 
 /* Number of OpenMP threads the parallel loops above use (1 without OpenMP). */

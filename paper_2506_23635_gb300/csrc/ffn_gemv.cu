@@ -288,10 +288,10 @@ cudaError_t launch_down_gemv(const moe_dims &d, int T, const float *h, const int
         return down_impl<float, float, float>(d, T, h, perm, offsets, w2, gate, y_sorted,
                                               nullptr, nullptr, false, st);
     }
-    // residual has x_dtype == w_dtype
+    // the residual has the output's dtype
     if (wb && ob) return down_impl<bf16, bf16, bf16>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
-    if (wb) return down_impl<bf16, float, bf16>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
-    if (ob) return down_impl<float, bf16, float>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
+    if (wb) return down_impl<bf16, float, float>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
+    if (ob) return down_impl<float, bf16, bf16>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
     return down_impl<float, float, float>(d, T, h, perm, offsets, w2, gate, nullptr, residual, out, true, st);
 }
 

@@ -441,7 +441,7 @@ cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const in
     if (d.out_dtype == MOE_BF16)
         return down_stream_impl<bf16, bf16, true>(d, T, h, offsets, inv_perm, w2, gate, residual,
                                                   out, nullptr, st);
-    return down_stream_impl<float, bf16, true>(d, T, h, offsets, inv_perm, w2, gate, residual, out,
+    return down_stream_impl<float, float, true>(d, T, h, offsets, inv_perm, w2, gate, residual, out,
                                                nullptr, st);
 }
 

@@ -426,6 +426,35 @@ k_combine(int T, int D, int K, const float *__restrict__ y, const int32_t *__res
 }
 
 // ===========================================================================
+// Stack glue (reading C9): x_norm[t,:] = bf16( r[t,:] / sqrt(mean(r[t,:]^2) + eps) )
+// One block per token; fp32 sum of squares reduced in a fixed order.
+// ===========================================================================
+template <typename TR, typename TX>
+__global__ void __launch_bounds__(256)
+k_prenorm(int T, int D, const TR *__restrict__ r, TX *__restrict__ xn, float eps) {
+    __shared__ float red[8];
+    ptx::grid_dependency_wait();
+    for (int t = blockIdx.x; t < T; t += gridDim.x) {
+        const TR *row = r + (size_t)t * D;
+        float ss = 0.f;
+        for (int d = threadIdx.x; d < D; d += 256) {
+            const float v = to_f(row[d]);
+            ss = fmaf(v, v, ss);
+        }
+        ss = warp_sum(ss);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+        __syncthreads();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        const float scale = rsqrtf(tot / (float)D + eps);
+        for (int d = threadIdx.x; d < D; d += 256)
+            xn[(size_t)t * D + d] = from_f<TX>(to_f(row[d]) * scale);
+        __syncthreads();
+    }
+}
+
+// ===========================================================================
 // host side
 // ===========================================================================
 
@@ -648,15 +677,29 @@ cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const int32
 
 cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t *inv,
                         const float *gate, const void *res, void *out, cudaStream_t st) {
-    const bool xb = d.x_dtype == MOE_BF16, ob = d.out_dtype == MOE_BF16;
-    if (xb && ob) return launch_combine<bf16, bf16>(d, T, y, inv, gate, res, out, st);
-    if (xb) return launch_combine<float, bf16>(d, T, y, inv, gate, res, out, st);
-    if (ob) return launch_combine<bf16, float>(d, T, y, inv, gate, res, out, st);
+    // the residual has the output's dtype
+    if (d.out_dtype == MOE_BF16) return launch_combine<bf16, bf16>(d, T, y, inv, gate, res, out, st);
     return launch_combine<float, float>(d, T, y, inv, gate, res, out, st);
 }
 
 bool use_stream_path(const moe_dims &d, int T) {
     return T <= kStreamMaxTokens && stream_path_ok(d, T);
+}
+
+cudaError_t prenorm_any(const moe_dims &d, int T, const void *r, void *xn, float eps,
+                        cudaStream_t st) {
+    const int grid = std::max(1, std::min(T, device_info().sm_count * 8));
+    int Tv = T, D = d.d_model;
+    void *args[] = {&Tv, &D, const_cast<void **>(&r), &xn, &eps};
+    const void *kern;
+    if (d.out_dtype == MOE_F32)
+        kern = d.x_dtype == MOE_BF16 ? (const void *)k_prenorm<float, bf16>
+                                     : (const void *)k_prenorm<float, float>;
+    else
+        kern = d.x_dtype == MOE_BF16 ? (const void *)k_prenorm<bf16, bf16>
+                                     : (const void *)k_prenorm<bf16, float>;
+    LaunchScope ls("prenorm", st);
+    return launch_pdl(kern, dim3(grid), dim3(256), 0, st, args);
 }
 
 template <typename P> P *at(void *ws, size_t off) {
@@ -814,6 +857,58 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
         if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st);
     }
     return cuda_status(e);
+}
+
+moe_status moe_prenorm(const moe_dims *dims, int32_t T, const void *resid, void *x_norm,
+                       float eps, moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(resid) || !ok_ptr(x_norm) || !(eps > 0.f)) return MOE_ERR_INVALID_ARG;
+    return cuda_status(prenorm_any(*dims, T, resid, x_norm, eps, (cudaStream_t)stream));
+}
+
+moe_status moe_stack_workspace_size(const moe_dims *dims, int32_t max_tokens, size_t *bytes) {
+    size_t layer = 0;
+    moe_status s = moe_workspace_size(dims, max_tokens, &layer);
+    if (s != MOE_OK) return s;
+    const size_t xn = ((size_t)max_tokens * dims->d_model * (dims->x_dtype == MOE_BF16 ? 2 : 4) +
+                       255) & ~size_t(255);
+    *bytes = xn + layer;
+    return MOE_OK;
+}
+
+moe_status moe_stack_forward(const moe_dims *dims, int32_t n_layers, int32_t T,
+                             const void *const *w_router, const void *const *w1,
+                             const void *const *v1, const void *const *w2, void *resid, float eps,
+                             void *ws, size_t ws_bytes, moe_stream_t stream) {
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (n_layers < 0) return MOE_ERR_INVALID_ARG;
+    if (T == 0 || n_layers == 0) return MOE_OK;
+    if (!w_router || !w1 || !v1 || !w2 || !ok_ptr(resid) || !(eps > 0.f))
+        return MOE_ERR_INVALID_ARG;
+    for (int l = 0; l < n_layers; ++l)
+        if (!ok_ptr(w_router[l]) || !ok_ptr(w1[l]) || !ok_ptr(v1[l]) || !ok_ptr(w2[l]))
+            return MOE_ERR_INVALID_ARG;
+    size_t need = 0;
+    if ((s = moe_stack_workspace_size(dims, T, &need)) != MOE_OK) return s;
+    if (!ws || !aligned16(ws) || ws_bytes < need) return MOE_ERR_WORKSPACE;
+    const size_t xn_bytes = need - ws_layout(*dims, T).total;
+    void *xn = ws;
+    void *lws = static_cast<char *>(ws) + xn_bytes;
+    for (int l = 0; l < n_layers; ++l) {
+        if (prenorm_any(*dims, T, resid, xn, eps, (cudaStream_t)stream) != cudaSuccess)
+            return MOE_ERR_CUDA;
+        // resid <- resid + MoE_l(x_norm): the combine reads each residual
+        // element before it writes the same element
+        s = moe_layer_forward(dims, T, xn, w_router[l], w1[l], v1[l], w2[l], resid, resid, lws,
+                              ws_bytes - xn_bytes, stream);
+        if (s != MOE_OK) return s;
+    }
+    return MOE_OK;
 }
 
 const char *moe_status_string(moe_status status) {

@@ -28,6 +28,7 @@ _STATUS = {
 EXPORTS = (
     "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
     "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc", "moe_status_string",
+    "moe_prenorm", "moe_stack_workspace_size", "moe_stack_forward",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
     "moe_profile_reset", "moe_profile_read",
 )
@@ -81,6 +82,10 @@ def lib() -> ctypes.CDLL:
         "moe_combine": [DP, I32, P, P, P, P, P, P],
         "moe_layer_forward": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
         "moe_layer_forward_noalloc": [DP, I32, P, P, P, P, P, P, P, P],
+        "moe_prenorm": [DP, I32, P, P, ctypes.c_float, P],
+        "moe_stack_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
+        "moe_stack_forward": [DP, I32, I32, ctypes.POINTER(P), ctypes.POINTER(P),
+                              ctypes.POINTER(P), ctypes.POINTER(P), P, ctypes.c_float, P, SZ, P],
         "moe_get_last_error": [P],
         "moe_status_string": [ctypes.c_int],
         "moe_profile_enable": [ctypes.c_int],
@@ -201,6 +206,51 @@ def layer_forward(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, ws=None,
                                    _ptr(w2), _ptr(residual), _ptr(out), _ptr(ws), ws.numel(),
                                    _stream(stream)), "moe_layer_forward")
     return out
+
+
+STACK_EPS = 1e-6  # RMS pre-norm epsilon of the stacked layers
+
+
+def prenorm(d: Dims, resid, x_norm=None, eps: float = STACK_EPS, stream=None):
+    """x_norm = RMSNorm0(resid) rounded to x_dtype (the glue between layers)."""
+    T = resid.shape[0]
+    if x_norm is None:
+        x_norm = torch.empty((T, d.d_model), dtype=_tdt(d.x_dtype), device=resid.device)
+    _check(lib().moe_prenorm(ctypes.byref(d), T, _ptr(resid), _ptr(x_norm), eps,
+                             _stream(stream)), "moe_prenorm")
+    return x_norm
+
+
+def stack_workspace_size(d: Dims, max_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().moe_stack_workspace_size(ctypes.byref(d), max_tokens, ctypes.byref(n)),
+           "moe_stack_workspace_size")
+    return int(n.value)
+
+
+class StackWeights:
+    """Device pointers of every layer's W_r, W1, V1, W2 as C arrays (the
+    tensors must outlive this object's use)."""
+
+    def __init__(self, layers):
+        n = len(layers)
+        self.n = n
+        self.tensors = layers
+        arr = lambda i: (ctypes.c_void_p * n)(*[ctypes.c_void_p(l[i].data_ptr()) for l in layers])
+        self.w_r, self.w1, self.v1, self.w2 = arr(0), arr(1), arr(2), arr(3)
+
+
+def stack_forward(d: Dims, weights: StackWeights, resid, ws=None, eps: float = STACK_EPS,
+                  stream=None):
+    """resid <- resid + MoE_l(RMSNorm0(resid)) for every layer, in place."""
+    T = resid.shape[0]
+    if ws is None:
+        ws = torch.empty(max(stack_workspace_size(d, T), 256), dtype=torch.uint8,
+                         device=resid.device)
+    _check(lib().moe_stack_forward(ctypes.byref(d), weights.n, T, weights.w_r, weights.w1,
+                                   weights.v1, weights.w2, _ptr(resid), eps, _ptr(ws),
+                                   ws.numel(), _stream(stream)), "moe_stack_forward")
+    return resid
 
 
 NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024  # MOE_NOALLOC_SCRATCH_BYTES

@@ -296,4 +296,83 @@ def pin_layer_steps_agree(orc):
     assert st["counts"].sum() == idx.size
 
 
+# --------------------------------------------------------------------------
+# stack glue (reading C9): RMSNorm0 and the residual stream
+# --------------------------------------------------------------------------
+
+
+def pin_rmsnorm0_closed_form(orc):
+    """[3, 4]: mean square 12.5, so the row becomes [3, 4] / sqrt(12.5 + eps);
+    in general mean(out^2) = ms / (ms + eps) and the direction is kept."""
+    eps = 1e-6
+    out = orc.rmsnorm0(np.array([[3.0, 4.0]]), eps)
+    _close(out[0], np.array([3.0, 4.0]) / math.sqrt(12.5 + eps), 1e-15, msg="rmsnorm [3,4]")
+    x = np.random.default_rng(31).normal(size=(5, 24)) * 7.0
+    y = orc.rmsnorm0(x, eps)
+    ms = (x * x).mean(axis=1)
+    _close((y * y).mean(axis=1), ms / (ms + eps), 1e-13, msg="mean square")
+    ratio = y / x
+    _close(ratio, np.broadcast_to(ratio[:, :1], ratio.shape), 1e-13, msg="direction kept")
+
+
+def pin_round_bf16_cases(orc):
+    """bf16 keeps 8 significant bits: spacing 2^-7 on [1, 2).  Exact cases:
+    1 + 2^-8 is a tie and goes to the even 1; 1 + 3*2^-8 is a tie and goes to
+    the even 1 + 2^-6; 1 + 0.75*2^-7 rounds up; values already on the grid
+    stay; and every float32 goes where the integer round-half-even of its bit
+    pattern sends it."""
+    cases = {1.0 + 2.0 ** -8: 1.0, 1.0 + 3 * 2.0 ** -8: 1.0 + 2.0 ** -6,
+             1.0 + 0.75 * 2.0 ** -7: 1.0 + 2.0 ** -7, -(1.0 + 2.0 ** -8): -1.0,
+             3.0: 3.0, 0.0: 0.0, 2.0 ** -20 * (1 + 2.0 ** -8): 2.0 ** -20}
+    got = orc.round_bf16(np.array(list(cases)))
+    assert np.array_equal(got, np.array(list(cases.values()))), "bf16 rounding cases"
+    x32 = np.random.default_rng(38).normal(size=512).astype(np.float32) * 100
+    want = gen.bf16_bits_to_f64(gen.f32_to_bf16_bits(x32))
+    assert np.array_equal(orc.round_bf16(x32.astype(np.float64)), want), "vs bit rounding"
+
+
+def _stack_layers(seed, n_layers, D=32, F=48, E=5, K=2, dt="f32"):
+    rng = np.random.default_rng(seed)
+    layers = []
+    for _ in range(n_layers):
+        layers.append((gen.store(rng.normal(size=(D, E)) * 0.5, dt),
+                       gen.store(rng.normal(size=(E, F, D)) * 0.2, dt),
+                       gen.store(rng.normal(size=(E, F, D)) * 0.2, dt),
+                       gen.store(rng.normal(size=(E, D, F)) * 0.2, dt)))
+    return layers
+
+
+def pin_stack_zero_w2_is_identity(orc):
+    """Zero down projections make every MoE block zero: the stack returns its
+    input exactly."""
+    layers = [(w_r, w1, v1, np.zeros_like(w2)) for (w_r, w1, v1, w2) in _stack_layers(32, 3)]
+    x0 = gen.store(np.random.default_rng(33).normal(size=(4, 32)), "f32")
+    out, _ = orc.stack_tokens(x0, layers, "f32", 2, 1e-6)
+    assert np.array_equal(out, gen.to_f64(x0, "f32")), "zero MoE blocks"
+
+
+def pin_stack_prenorm_scale_invariance(orc):
+    """The pre-norm makes a block's input independent of the residual's scale,
+    so one block adds the same vector to x and to c*x: f(c x) - c x = f(x) - x."""
+    layers = _stack_layers(34, 1)
+    x0 = np.random.default_rng(35).normal(size=(4, 32))
+    a, _ = orc.stack_tokens(x0, layers, "f64", 2, 1e-12)
+    b, _ = orc.stack_tokens(3.0 * x0, layers, "f64", 2, 1e-12)
+    _close(b - 3.0 * x0, a - x0, 1e-9, 1e-12, msg="pre-norm scale invariance")
+
+
+def pin_stack_residual_composition(orc):
+    """Two stacked blocks = block 1 applied to the output of block 0, and each
+    block adds its MoE output to the residual (checked against the single
+    layer with the residual passed in)."""
+    layers = _stack_layers(36, 2)
+    x0 = np.random.default_rng(37).normal(size=(3, 32))
+    two, _ = orc.stack_tokens(x0, layers, "f64", 2, 1e-6)
+    one, _ = orc.stack_tokens(x0, layers[:1], "f64", 2, 1e-6)
+    w_r, w1, v1, w2 = layers[1]
+    xn = orc.rmsnorm0(one, 1e-6)
+    moe, _, _ = orc.layer_tokens(xn, w_r, w1, v1, w2, "f32", 2, x_dtype="f64")
+    _close(two, one + moe, 1e-13, 1e-13, msg="residual composition")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -101,7 +101,8 @@ def test_layer_residual_and_bf16_out(T):
     assert out.dtype == torch.bfloat16
     assert_parity(to_numpy(out), want, "bf16", "layer + residual")
     d32 = _dims(m, sh, out_dtype=torch.float32)
-    out32 = m.layer_forward(d32, x, w_r, w1, v1, w2, residual=dev(res, "bf16"))
+    # the residual has the output's dtype
+    out32 = m.layer_forward(d32, x, w_r, w1, v1, w2, residual=dev(res, "bf16").float())
     assert out32.dtype == torch.float32
     assert_parity(to_numpy(out32), want, "bf16", "layer + residual, f32 out")
 

@@ -1,0 +1,135 @@
+"""Stacked MoE blocks with the parameter-free RMS pre-norm and the residual
+add between them (the 16-layer DBRX-shaped stack of the decode benchmark)
+against the fp64 oracle.
+
+With bf16 layer inputs every block perturbs the residual stream by a few
+1e-3 relative, so a later router whose K-th and (K+1)-th logits are closer
+than that may pick either expert: both are correct within the precision.
+Those tokens are ill-conditioned; the bf16 tests compare the tokens whose
+routing gap stays above 2% of the logit RMS at every layer (about 7 times the
+expected perturbation), and require enough of them.  Both sides store the
+normalised layer input in bf16; the remaining difference is the bf16 GLU
+hidden vector of every layer, so the one-layer bound is compounded over the
+stacked layers (see _filtered_parity)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2506_23635_gb300 import inputs as gen
+from tests.gpu_util import dev, need_gpu, to_numpy
+
+pytestmark = pytest.mark.gpu
+
+EPS = 1e-6
+WELL_CONDITIONED = 0.02
+
+
+def moe():
+    need_gpu()
+    from paper_2506_23635_gb300 import moe as m
+    return m
+
+
+def _layers(shape, n_layers, seed, router_std=gen.W_STD):
+    out = []
+    for l in range(n_layers):
+        w_r = gen.host_normal((shape.d_model, shape.n_experts), router_std, shape.dtype,
+                              seed, "stack-w_r", l)
+        w1, v1, w2 = gen.host_expert_weights(shape, seed + 1000 * (l + 1))
+        out.append((w_r, w1, v1, w2))
+    return out
+
+
+def _run_gpu(m, shape, layers, x0, out_dtype=torch.float32):
+    tdt = gen.torch_dtype(shape.dtype)
+    d = m.dims(shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k, tdt, tdt, out_dtype)
+    dl = [tuple(dev(a, shape.dtype) for a in lw) for lw in layers]
+    sw = m.StackWeights(dl)
+    resid = dev(x0, shape.dtype).to(out_dtype).contiguous()
+    m.stack_forward(d, sw, resid, eps=EPS)
+    assert m.get_last_error() == 0
+    return to_numpy(resid)
+
+
+def test_prenorm():
+    m = moe()
+    T, D = 5, 6144
+    r = np.random.default_rng(1).normal(size=(T, D)) * 3.0
+    want = oracle.rmsnorm0(r.astype(np.float32).astype(np.float64), EPS)
+    d = m.dims(D, 64, 4, 2, torch.bfloat16, torch.bfloat16, torch.float32)
+    xn = m.prenorm(d, torch.from_numpy(r.astype(np.float32)).cuda(), eps=EPS)
+    assert xn.dtype == torch.bfloat16
+    got = to_numpy(xn)
+    # one bf16 rounding of each element
+    assert np.all(np.abs(got - want) <= 2.0 ** -8 * np.abs(want) + 1e-30)
+
+
+def test_stack_fp32_sixteen_layers():
+    """The tiny layer's shape in fp32, 16 layers, 3 consecutive steps of fresh
+    tokens (fp32 keeps the residual stream within ~1e-6 of the oracle, far
+    inside every routing gap)."""
+    m = moe()
+    shape = gen.TINY
+    layers = _layers(shape, 16, 51, router_std=0.1)
+    for step in range(3):
+        x0 = gen.host_normal((8, shape.d_model), 1.0, "f32", 52, "stack-x", step)
+        want, gaps = oracle.stack_tokens(x0, layers, "f32", shape.top_k, EPS)
+        assert np.min(gaps) > 1e-4
+        got = _run_gpu(m, shape, layers, x0)
+        rel = np.linalg.norm(got - want) / np.linalg.norm(want)
+        assert rel <= 1e-4, f"step {step}: rel L2 {rel:.2e}"
+
+
+def _filtered_parity(got, want, gaps, min_tokens):
+    """bf16 bound of one layer output (rel L2 5e-3, max abs 2e-2 RMS),
+    compounded over the L stacked layers: the layers' rounding errors are
+    independent, so they add in quadrature -> both limits times sqrt(L)."""
+    ok = np.all(gaps >= WELL_CONDITIONED, axis=0)
+    assert ok.sum() >= min_tokens, f"only {ok.sum()} well-conditioned tokens"
+    L = gaps.shape[0]
+    g, w = got[ok], want[ok]
+    err = g - w
+    rel = np.linalg.norm(err) / np.linalg.norm(w)
+    rms = np.sqrt(np.mean(w * w))
+    assert rel <= 5e-3 * np.sqrt(L), f"{L} layers: rel L2 {rel:.3e}"
+    assert np.max(np.abs(err)) <= 2e-2 * np.sqrt(L) * rms, f"{L} layers: max abs"
+    return int(ok.sum())
+
+
+def test_stack_bf16_sixteen_layers():
+    """bf16 weights and layer inputs, fp32 residual stream, 16 layers."""
+    m = moe()
+    shape = gen.LayerShape(512, 1024, 16, 4, "bf16")
+    layers = _layers(shape, 16, 61, router_std=0.1)
+    x0 = gen.host_normal((48, shape.d_model), 1.0, "bf16", 62, "stack-x")
+    want, gaps = oracle.stack_tokens(x0, layers, "bf16", shape.top_k, EPS)
+    got = _run_gpu(m, shape, layers, x0)
+    _filtered_parity(got, want, gaps, 8)
+
+
+def test_stack_dbrx_three_layers():
+    """Full DBRX-shaped layers (D=6144, F=10752, E=16, K=4): three stacked
+    blocks, 8 tokens; weights drawn on the device and brought to the host one
+    layer at a time for the oracle."""
+    m = moe()
+    sh = gen.DBRX
+    n_layers, T = 3, 8
+    devw = [gen.device_expert_weights(sh, 71, "cuda", layer=l) for l in range(n_layers)]
+    routers = [gen.host_normal((sh.d_model, sh.n_experts), gen.W_STD, "bf16", 71, "stack-w_r", l)
+               for l in range(n_layers)]
+    x0 = gen.host_normal((T, sh.d_model), 1.0, "bf16", 72, "stack-x")
+    d = m.dims(sh.d_model, sh.ffn_hidden, sh.n_experts, sh.top_k, torch.bfloat16,
+               torch.bfloat16, torch.float32)
+    sw = m.StackWeights([(dev(routers[l], "bf16"),) + devw[l] for l in range(n_layers)])
+    resid = dev(x0, "bf16").float().contiguous()
+    m.stack_forward(d, sw, resid, eps=EPS)
+    assert m.get_last_error() == 0
+    got = to_numpy(resid)
+
+    def layer(l):
+        return (routers[l],) + tuple(gen.torch_to_host(t, "bf16") for t in devw[l])
+
+    want, gaps = oracle.stack_tokens(x0, lambda l: layer(l) if l < n_layers else None, "bf16",
+                                     sh.top_k, EPS)
+    _filtered_parity(got, want, gaps, 3)

@@ -34,6 +34,14 @@ MUTATIONS = [
     ("combine_ungated", "for (int d = 0; d < D; ++d) o[d] += g[k] * y[d];",
      "for (int d = 0; d < D; ++d) o[d] += y[d];"),
     ("dense_mask_ungated", "mask[idx[k]] = g[k];", "mask[idx[k]] = 1.0;"),
+    ("bf16_round_to_9_bits", "const double ulp = ldexp(1.0, e - 8);",
+     "const double ulp = ldexp(1.0, e - 9);"),
+    ("bf16_round_truncates", "out[i] = nearbyint(v / ulp) * ulp;",
+     "out[i] = trunc(v / ulp) * ulp;"),
+    ("rmsnorm_no_sqrt", "const double s = 1.0 / sqrt(ss / D + eps);",
+     "const double s = 1.0 / (ss / D + eps);"),
+    ("rmsnorm_sum_not_mean", "const double s = 1.0 / sqrt(ss / D + eps);",
+     "const double s = 1.0 / sqrt(ss + eps);"),
 ]
 
 
