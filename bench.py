@@ -360,6 +360,20 @@ def tensor_roofline(kstats, shape, T, workload):
                       "of the same K steps"}
 
 
+def eq1_refit(shape, T, U, ms):
+    """The paper's Eq. 1 refit to one layer on this GPU (measured peaks):
+    max(load of the selected experts, compute of the slots), vs measured."""
+    from paper_2506_23635_gb300 import perf_model
+
+    peaks, _ = measured_peaks()
+    m = perf_model.gb300_moe_layer_time(
+        T, U, float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS)) * 1e9,
+        float(peaks.get("bf16_tflops", 1910.6)) * 1e12, shape.d_model, shape.ffn_hidden,
+        shape.top_k)
+    return {"model_ms": round(m["time"] * 1e3, 4), "bound": m["bound"],
+            "measured_over_model": round(ms / (m["time"] * 1e3), 3)}
+
+
 def measure_extra(layer, workload, steps, warmup):
     """A secondary workload of the same layer: a few timed steps."""
     shape, T = WORKLOADS[workload]
@@ -377,12 +391,13 @@ def measure_extra(layer, workload, steps, warmup):
     r = {"workload": workload, "tokens_per_step": T, "steps": steps,
          "ms_per_step": round(ms, 4), "us_per_token_step": round(ms * 1e3 / T, 3),
          "kernels": kernel_table(kstats)}
+    U = layer.distinct_experts(xs, w_r)
+    r["eq1_refit"] = eq1_refit(shape, T, U, ms)
     if T >= PREFILL_MIN_TOKENS:
         flops = 2.0 * T * shape.top_k * 3 * shape.d_model * shape.ffn_hidden
         r["tflops"] = round(flops / (ms / 1e3) / 1e12, 1)
         r["roofline"] = tensor_roofline(kstats, shape, T, workload)
     else:
-        U = layer.distinct_experts(xs, w_r)
         step_bytes = U * 3 * shape.d_model * shape.ffn_hidden * 2
         r["distinct_experts_per_step"] = U
         r["achieved_hbm_gbs_step"] = round(step_bytes / (ms / 1e3) / 1e9, 1)
@@ -584,6 +599,7 @@ def run_ours(args):
     }
     if not prefill:
         line["achieved_hbm_gbs_step"] = round(step_bytes / (ms_max / 1e3) / 1e9, 1)
+    line["eq1_refit"] = eq1_refit(shape, T, U_mean, ms_max)
     if extra:
         line["extra"] = extra
     if world == 1 and not args.no_cpu_baseline:
