@@ -52,6 +52,9 @@ WORKLOADS = {
     # a 512-token prefill of the same 4-expert layer: the small case for
     # captures of the tensor-core GEMMs
     "dbrx4-prefill-t512": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 512),
+    # the tiny fp32 layer (D=256, F=512, E=4, K=2), 8 tokens: the reference
+    # arm's smallest case (runs anywhere, no GPU needed)
+    "tiny-decode-t8": (gen.TINY, 8),
 }
 PREFILL_MIN_TOKENS = 512
 
