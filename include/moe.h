@@ -216,6 +216,21 @@ const char *moe_status_string(moe_status status);
  * asynchronous CUDA fault. */
 moe_status moe_get_last_error(moe_stream_t stream);
 
+/* ---- failure detection ---------------------------------------------------
+ * Every device-side wait in the pipelined kernels gives up after a wall-time
+ * limit (2 s), records MOE_ERR_TIMEOUT and lets its kernel return, so a
+ * broken pipeline ends instead of hanging the GPU.
+ * moe_selftest_wait_timeout exercises exactly that path: one thread waits on
+ * an mbarrier that nothing completes, with the given limit (<= 10 s); it
+ * writes 1 to *gave_up (a DEVICE int) when the wait gave up, and the next
+ * moe_get_last_error returns MOE_ERR_TIMEOUT.  The context stays usable.
+ * Host-side fault injection: with MOE_INJECT_FAILURE="<entry>:<status>" in
+ * the environment, the named entry point (moe_route, moe_dispatch,
+ * moe_expert_ffn, moe_combine, moe_layer_forward, moe_prenorm,
+ * moe_stack_forward) returns that status at once without launching. */
+moe_status moe_selftest_wait_timeout(uint64_t limit_ns, int32_t *gave_up,
+                                     moe_stream_t stream);
+
 /* ---- launch accounting and per-kernel timing (benchmarks) ---------------
  * moe_launch_count: number of kernels this library has launched since load.
  * moe_profile_enable(1): every later kernel launch is bracketed by a pair of

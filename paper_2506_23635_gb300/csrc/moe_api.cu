@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <atomic>
 #include <mutex>
+#include <stdlib.h>
 #include <string.h>
 #include <string>
 #include <vector>
@@ -455,6 +456,18 @@ k_prenorm(int T, int D, const TR *__restrict__ r, TX *__restrict__ xn, float eps
 }
 
 // ===========================================================================
+// Self-test of the bounded waits: one thread waits on an mbarrier that
+// nothing will complete.  The wait gives up after limit_ns, records
+// kErrTimeout and the kernel returns normally.
+// ===========================================================================
+__global__ void k_wait_timeout_selftest(uint64_t limit_ns, unsigned *err, int *gave_up) {
+    __shared__ uint64_t bar;
+    ptx::mbar_init(&bar, 1);
+    ptx::fence_barrier_init();
+    *gave_up = ptx::mbar_wait_limit(&bar, 0, err, limit_ns) ? 0 : 1;
+}
+
+// ===========================================================================
 // host side
 // ===========================================================================
 
@@ -571,6 +584,25 @@ using namespace moe;
 namespace {
 
 bool dt_ok(int32_t v) { return v == MOE_F32 || v == MOE_BF16; }
+
+// Host-side fault injection for callers' error paths: MOE_INJECT_FAILURE
+// "<entry point>:<status>" makes that entry return the status at once,
+// before anything is validated or launched.  Read on every call (tests set
+// it per process); nothing is injected when it is unset.
+moe_status injected(const char *entry) {
+    const char *v = getenv("MOE_INJECT_FAILURE");
+    if (!v) return MOE_OK;
+    const size_t n = strlen(entry);
+    if (strncmp(v, entry, n) != 0 || v[n] != ':') return MOE_OK;
+    const int code = atoi(v + n + 1);
+    return (code > 0 && code <= MOE_ERR_DEVICE_INDEX) ? (moe_status)code : MOE_OK;
+}
+
+#define MOE_INJECT(name)                                \
+    do {                                                \
+        moe_status inj_ = injected(name);               \
+        if (inj_ != MOE_OK) return inj_;                \
+    } while (0)
 
 moe_status check_dims(const moe_dims *d) {
     if (!d) return MOE_ERR_INVALID_ARG;
@@ -722,6 +754,7 @@ moe_status moe_workspace_size(const moe_dims *dims, int32_t max_tokens, size_t *
 
 moe_status moe_route(const moe_dims *dims, int32_t T, const void *x, const void *w_router,
                      float *logits_opt, int32_t *topk_idx, float *topk_gate, moe_stream_t stream) {
+    MOE_INJECT("moe_route");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -735,6 +768,7 @@ moe_status moe_route(const moe_dims *dims, int32_t T, const void *x, const void 
 moe_status moe_dispatch(const moe_dims *dims, int32_t T, const int32_t *topk_idx,
                         int32_t *counts, int32_t *offsets, int32_t *perm, int32_t *inv_perm,
                         moe_stream_t stream) {
+    MOE_INJECT("moe_dispatch");
     moe_status s = check_dims(dims);
     if (s == MOE_ERR_UNSUPPORTED) s = MOE_OK;  // dispatch does not read floating point data
     if (s != MOE_OK) return s;
@@ -748,6 +782,7 @@ moe_status moe_dispatch(const moe_dims *dims, int32_t T, const int32_t *topk_idx
 moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x, const int32_t *perm,
                           const int32_t *offsets, const void *w1, const void *v1, const void *w2,
                           float *y_sorted, void *ws, size_t ws_bytes, moe_stream_t stream) {
+    MOE_INJECT("moe_expert_ffn");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -786,6 +821,7 @@ moe_status moe_expert_ffn(const moe_dims *dims, int32_t T, const void *x, const 
 moe_status moe_combine(const moe_dims *dims, int32_t T, const float *y_sorted,
                        const int32_t *inv_perm, const float *topk_gate, const void *residual_opt,
                        void *out, moe_stream_t stream) {
+    MOE_INJECT("moe_combine");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -800,6 +836,7 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
                              const void *w1, const void *v1, const void *w2,
                              const void *residual_opt, void *out, void *ws, size_t ws_bytes,
                              moe_stream_t stream) {
+    MOE_INJECT("moe_layer_forward");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -861,6 +898,7 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
 
 moe_status moe_prenorm(const moe_dims *dims, int32_t T, const void *resid, void *x_norm,
                        float eps, moe_stream_t stream) {
+    MOE_INJECT("moe_prenorm");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -883,6 +921,7 @@ moe_status moe_stack_forward(const moe_dims *dims, int32_t n_layers, int32_t T,
                              const void *const *w_router, const void *const *w1,
                              const void *const *v1, const void *const *w2, void *resid, float eps,
                              void *ws, size_t ws_bytes, moe_stream_t stream) {
+    MOE_INJECT("moe_stack_forward");
     moe_status s = check_dims(dims);
     if (s != MOE_OK) return s;
     if ((s = check_T(dims, T)) != MOE_OK) return s;
@@ -937,6 +976,14 @@ moe_status moe_get_last_error(moe_stream_t stream) {
     if (v == kErrIndex) return MOE_ERR_DEVICE_INDEX;
     if (v == kErrTimeout) return MOE_ERR_TIMEOUT;
     return MOE_OK;
+}
+
+moe_status moe_selftest_wait_timeout(uint64_t limit_ns, int32_t *gave_up, moe_stream_t stream) {
+    if (!gave_up || limit_ns == 0 || limit_ns > 10000000000ull) return MOE_ERR_INVALID_ARG;
+    LaunchScope ls("selftest_wait_timeout", (cudaStream_t)stream);
+    k_wait_timeout_selftest<<<1, 1, 0, (cudaStream_t)stream>>>(limit_ns, device_info().err,
+                                                              gave_up);
+    return cuda_status(cudaGetLastError());
 }
 
 int64_t moe_launch_count(void) { return g_launches.load(); }

@@ -62,17 +62,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Wait for the phase with the given parity to complete; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, unsigned *err) {
+// Wait for the phase with the given parity to complete; false (and
+// kErrTimeout recorded) once limit_ns of wall time have passed.
+__device__ __forceinline__ bool mbar_wait_limit(uint64_t *bar, uint32_t parity, unsigned *err,
+                                                uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
+        if ((it & 63u) == 0 && globaltimer() - t0 > limit_ns) {
             set_error(err, kErrTimeout);
             return false;
         }
     }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, unsigned *err) {
+    return mbar_wait_limit(bar, parity, err, kWaitLimitNs);
 }
 
 // ---- L2 policies -----------------------------------------------------------

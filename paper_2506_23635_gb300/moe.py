@@ -29,6 +29,7 @@ EXPORTS = (
     "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
     "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc", "moe_status_string",
     "moe_prenorm", "moe_stack_workspace_size", "moe_stack_forward",
+    "moe_selftest_wait_timeout",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
     "moe_profile_reset", "moe_profile_read",
 )
@@ -83,6 +84,7 @@ def lib() -> ctypes.CDLL:
         "moe_layer_forward": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
         "moe_layer_forward_noalloc": [DP, I32, P, P, P, P, P, P, P, P],
         "moe_prenorm": [DP, I32, P, P, ctypes.c_float, P],
+        "moe_selftest_wait_timeout": [ctypes.c_uint64, P, P],
         "moe_stack_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
         "moe_stack_forward": [DP, I32, I32, ctypes.POINTER(P), ctypes.POINTER(P),
                               ctypes.POINTER(P), ctypes.POINTER(P), P, ctypes.c_float, P, SZ, P],
@@ -267,6 +269,14 @@ def layer_forward_noalloc(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, 
                                            _ptr(v1), _ptr(w2), _ptr(residual), _ptr(out),
                                            _stream(stream)), "moe_layer_forward_noalloc")
     return out
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None) -> bool:
+    """Run the bounded-wait self test; True if the wait gave up."""
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    _check(lib().moe_selftest_wait_timeout(limit_ns, _ptr(flag), _stream(stream)),
+           "moe_selftest_wait_timeout")
+    return bool(flag.item())
 
 
 def get_last_error(stream=None) -> int:

@@ -139,3 +139,28 @@ def test_noalloc_validation(lib):
 
 def test_launch_count_starts_at_zero_without_launches(lib):
     assert lib.launch_count() >= 0
+
+
+def test_fault_injection_env(lib):
+    """MOE_INJECT_FAILURE makes the named entry return the given status before
+    anything is validated or launched (null pointers: nothing could launch)."""
+    code = (
+        "import ctypes, sys; sys.path.insert(0, %r)\n"
+        "from paper_2506_23635_gb300 import moe\n"
+        "L = moe.lib(); d = moe.dims(64, 64, 4, 2)\n"
+        "print(L.moe_route(ctypes.byref(d), 4, None, None, None, None, None, None),\n"
+        "      L.moe_layer_forward(ctypes.byref(d), 4, None, None, None, None, None, None, None,\n"
+        "                          None, 0, None))\n" % ROOT)
+    import subprocess
+    import sys
+    env = dict(os.environ, MOE_INJECT_FAILURE="moe_layer_forward:4")
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                         timeout=120)
+    assert out.returncode == 0, out.stderr
+    route_status, layer_status = map(int, out.stdout.split())
+    assert route_status == 1  # not injected: ordinary validation of the nulls
+    assert layer_status == 4  # injected MOE_ERR_CUDA
+    env["MOE_INJECT_FAILURE"] = "moe_route:5"
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                         timeout=120)
+    assert list(map(int, out.stdout.split())) == [5, 1]
