@@ -10,10 +10,11 @@
 //   DOWN:        y[j, d] = h[j, :] . W2[e,d,:]                          -> fp32
 //
 // for the sorted slots j of expert e (x_j = the gathered token rows).
-// Tile = 128 slots (M, the A operand, K-major) x 256 weight rows (N, the B
-// operand, K-major) x 64 of the reduction dimension per pipeline stage.  In
-// UP the 256 weight rows are 128 rows of W1 followed by the same 128 rows of
-// V1, so one accumulator holds a (columns 0..127) and b (columns 128..255)
+// Tile = 128 slots (M, the A operand, K-major) x BN = 256 weight rows (N, the
+// B operand, K-major) x 64 of the reduction dimension per pipeline stage
+// (Cfg keeps BN and the stage count template parameters).  In UP the BN
+// weight rows are BN/2 rows of W1 followed by the same BN/2 rows of V1, so
+// one accumulator holds a (first half of the columns) and b (second half)
 // for the same f, and the GLU runs in the epilogue straight from tensor
 // memory.
 //
@@ -21,8 +22,8 @@
 //   warp 0     TMA producer (one lane): A and B tiles into a 4-stage ring,
 //              128-byte swizzle, completion on mbarriers;
 //   warp 1     tensor-memory allocator and MMA issuer (one lane):
-//              tcgen05.mma kind::f16, M=128, N=256, K=16, into one of two
-//              256-column fp32 accumulators; tcgen05.commit frees a stage
+//              tcgen05.mma kind::f16, M=128, N=BN, K=16, into one of two
+//              BN-column fp32 accumulators; tcgen05.commit frees a stage
 //              and hands a finished accumulator to the epilogue;
 //   warps 2-5  epilogue: tcgen05.ld of their 32 tensor-memory lanes, GLU or
 //              plain copy, stores to global memory.
@@ -40,21 +41,39 @@
 namespace moe {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64;
-constexpr int kStages = 4;
+constexpr int BM = 128, BK = 64;
+constexpr int kMaxStages = 8;
 constexpr int kThreadsTc = 192;
-constexpr uint32_t kStageA = BM * BK * 2;           // 16 KB
-constexpr uint32_t kStageB = BN * BK * 2;           // 32 KB
-constexpr uint32_t kStageBytes = kStageA + kStageB;  // 48 KB
-constexpr uint32_t kTmemCols = 2 * BN;              // two accumulators
+constexpr uint32_t kStageA = BM * BK * 2;  // 16 KB
 constexpr size_t kTcHeaderBytes = 2048;
-constexpr size_t kSmemTc = 1024 /*align slack*/ + kStages * kStageBytes + kTcHeaderBytes;
 
 enum Mode { kUp = 0, kDown = 1 };
 
+// Tile shape of one instantiation: BN weight rows per tile (UP: BN/2 rows of
+// W1 and the same BN/2 rows of V1), STAGES pipeline stages.
+template <int MODE, int BN_, int STAGES_>
+struct Cfg {
+    static constexpr int BN = BN_;
+    static constexpr int kStages = STAGES_;
+    static constexpr int kCols = MODE == kUp ? BN / 2 : BN;  // output columns per tile
+    static constexpr uint32_t kStageB = BN * BK * 2;
+    static constexpr uint32_t kStageBytes = kStageA + kStageB;
+    static constexpr uint32_t kTmemCols = 2 * BN;  // two accumulators
+    static constexpr size_t kSmem = 1024 /*align slack*/ + kStages * kStageBytes + kTcHeaderBytes;
+    // kind::f16 instruction descriptor: bf16 A and B, fp32 D, both K-major,
+    // N = BN, M = 128
+    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                                       ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    static_assert(kStages <= kMaxStages, "too many stages");
+    static_assert(kCols % 32 == 0, "epilogue works in 32-column steps");
+    static_assert((kTmemCols & (kTmemCols - 1)) == 0 && kTmemCols >= 32 && kTmemCols <= 512,
+                  "tensor memory is allocated in powers of two");
+    static_assert(kSmem <= 227 * 1024, "shared memory");
+};
+
 struct TcHeader {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint64_t done;
@@ -133,10 +152,6 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
            ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-// kind::f16 instruction descriptor: bf16 A and B, fp32 D, both K-major.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
-
 // ---- tile schedule -------------------------------------------------------------
 
 // tprefix[e] = sum over earlier experts of ceil(n_e / BM) * n_tiles_n.
@@ -184,20 +199,25 @@ __device__ __forceinline__ Tile tile_of(const int *tprefix, const int32_t *offse
 
 // ---- the kernel ------------------------------------------------------------------
 
-template <int MODE>
+template <int MODE, class C>
 __global__ void __launch_bounds__(kThreadsTc, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
           const __grid_constant__ CUtensorMap tmB1, const int32_t *__restrict__ offsets, int E,
-          int S, int Kdim, int Nw, bf16 *__restrict__ h_out, float *__restrict__ y_out,
-          unsigned *err) {
+          int S, int Kdim, int Nw, uint32_t a_bytes, bf16 *__restrict__ h_out,
+          float *__restrict__ y_out, unsigned *err) {
     // Kdim: reduction length (D for UP, F for DOWN); Nw: weight rows per
-    // expert (F for UP, D for DOWN) = the output width.
+    // expert (F for UP, D for DOWN) = the output width.  a_bytes: bytes of
+    // the A box (rows x 128 B).  In a decode batch an expert holds at most T
+    // slots, so only ceil(T/16)*16 rows are loaded; the MMA still reads 128
+    // rows and the rows past the box give accumulator rows nobody stores.
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    constexpr int kStages = C::kStages, BN = C::BN, kCols = C::kCols;
+    constexpr uint32_t kStageBytes = C::kStageBytes, kStageB = C::kStageB;
     TcHeader *hd = reinterpret_cast<TcHeader *>(smem + kStages * kStageBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int ntn = MODE == kUp ? (Nw + 127) / 128 : (Nw + BN - 1) / BN;
+    const int ntn = (Nw + kCols - 1) / kCols;
     const int nk = (Kdim + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
@@ -215,7 +235,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         ptx::prefetch_tmap(&tmB0);
         if (MODE == kUp) ptx::prefetch_tmap(&tmB1);
     }
-    if (warp == 1) tmem_alloc(&hd->tmem_base, kTmemCols);
+    if (warp == 1) tmem_alloc(&hd->tmem_base, C::kTmemCols);
     ptx::grid_dependency_wait();  // offsets and the A operand come from earlier kernels
     if (warp == 2) tile_prefix(offsets, E, S, ntn, hd->tprefix, err);
     tc_fence_before();
@@ -233,13 +253,13 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             bool ok = true;
             for (int u = blockIdx.x; u < n_tiles && ok; u += gridDim.x) {
                 const Tile t = tile_of(hd->tprefix, offsets, E, ntn, u);
-                const int brow = MODE == kUp ? t.e * Nw + t.nt * 128 : t.e * Nw + t.nt * BN;
+                const int brow = t.e * Nw + t.nt * kCols;
                 for (int kb = 0; kb < nk; ++kb, ++it) {
                     const uint32_t s = it % kStages, ph = (it / kStages) & 1;
                     if (!(ok = ptx::mbar_wait(&hd->empty[s], ph ^ 1, err))) break;
                     unsigned char *sa = smem + s * kStageBytes;
                     unsigned char *sb = sa + kStageA;
-                    ptx::mbar_arrive_expect_tx(&hd->full[s], kStageBytes);
+                    ptx::mbar_arrive_expect_tx(&hd->full[s], a_bytes + kStageB);
                     ptx::tma_load_2d(sa, &tmA, kb * BK, t.row0, &hd->full[s], pol_a);
                     if (MODE == kUp) {
                         ptx::tma_load_2d(sb, &tmB0, kb * BK, brow, &hd->full[s], pol_b);
@@ -272,7 +292,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     const uint64_t adesc = smem_desc(sa), bdesc = smem_desc(sa + kStageA);
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk)
-                        mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, kIdesc,
+                        mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, C::kIdesc,
                                  (kb | kk) != 0 ? 1u : 0u);
                     mma_commit(&hd->empty[s]);  // stage free once these MMAs finish
                 }
@@ -297,12 +317,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             const bool row_ok = m < t.rows;
             const size_t j = (size_t)t.row0 + m;
             if (MODE == kUp) {
-                const int f0 = t.nt * 128;
+                const int f0 = t.nt * kCols;
 #pragma unroll 1
-                for (int c = 0; c < 128; c += 32) {
+                for (int c = 0; c < kCols; c += 32) {
                     float a[32], b[32];
                     tmem_ld32(base + c, a);
-                    tmem_ld32(base + 128 + c, b);
+                    tmem_ld32(base + kCols + c, b);
                     tmem_ld_wait();
                     if (row_ok) {
                         uint32_t pk[16];
@@ -346,7 +366,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+    if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
 }
 
 // ---- gather of the A operand: x_sorted[j, :] = x[perm[j] / K, :] ----------------
@@ -400,19 +420,35 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, ui
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int MODE>
+template <int MODE, class C>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUtensorMap &b1,
-                        const int32_t *offsets, int E, int S, int Kdim, int Nw, bf16 *h_out,
-                        float *y_out, cudaStream_t st) {
-    const void *kern = (const void *)k_gemm_tc<MODE>;
+                        const int32_t *offsets, int E, int S, int Kdim, int Nw, uint32_t a_bytes,
+                        bf16 *h_out, float *y_out, cudaStream_t st) {
+    const void *kern = (const void *)k_gemm_tc<MODE, C>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemTc);
+                                         (int)C::kSmem);
     if (e != cudaSuccess) return e;
     unsigned *err = device_info().err;
     CUtensorMap ma = a, mb0 = b0, mb1 = b1;
-    void *args[] = {&ma, &mb0, &mb1, &offsets, &E, &S, &Kdim, &Nw, &h_out, &y_out, &err};
+    void *args[] = {&ma, &mb0, &mb1, &offsets, &E, &S, &Kdim, &Nw, &a_bytes, &h_out, &y_out,
+                    &err};
     LaunchScope ls(MODE == kUp ? "gemm_up_glu_tc" : "gemm_down_tc", st);
-    return launch_pdl(kern, dim3(device_info().sm_count), dim3(kThreadsTc), kSmemTc, st, args);
+    return launch_pdl(kern, dim3(device_info().sm_count), dim3(kThreadsTc), C::kSmem, st, args);
+}
+
+// Both projections use 256-row weight tiles with 4 stages: narrower tiles
+// balance the SMs better when few experts are selected, but hold too few
+// weight bytes in flight per SM to stream at the HBM rate (measured: 64-row
+// down-projection tiles ran 1.6x slower at 64 tokens).
+using UpWide = Cfg<kUp, 256, 4>;
+using DownWide = Cfg<kDown, 256, 4>;
+
+// Rows of the A box: a whole 128-row slot tile, or for batches under 128
+// tokens (an expert then holds at most T slots, all in one slot tile) just
+// T rounded up to 16.
+uint32_t a_box_rows(int T) {
+    if (T >= BM) return BM;
+    return (uint32_t)((T + 15) / 16 * 16);
 }
 
 }  // namespace
@@ -439,22 +475,26 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
 cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, const int32_t *offsets,
                               const void *w1, const void *v1, void *h, cudaStream_t st) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
+    const uint32_t arows = a_box_rows(T);
     CUtensorMap a, b0, b1;
-    if (!make_map(&a, x_sorted, (uint64_t)S, (uint64_t)D, BM) ||
-        !make_map(&b0, w1, (uint64_t)E * F, (uint64_t)D, 128) ||
-        !make_map(&b1, v1, (uint64_t)E * F, (uint64_t)D, 128))
+    if (!make_map(&a, x_sorted, (uint64_t)S, (uint64_t)D, arows) ||
+        !make_map(&b0, w1, (uint64_t)E * F, (uint64_t)D, UpWide::kCols) ||
+        !make_map(&b1, v1, (uint64_t)E * F, (uint64_t)D, UpWide::kCols))
         return cudaErrorInvalidValue;
-    return launch_gemm<kUp>(a, b0, b1, offsets, E, S, D, F, static_cast<bf16 *>(h), nullptr, st);
+    return launch_gemm<kUp, UpWide>(a, b0, b1, offsets, E, S, D, F, arows * BK * 2,
+                                    static_cast<bf16 *>(h), nullptr, st);
 }
 
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
+    const uint32_t arows = a_box_rows(T);
     CUtensorMap a, b0;
-    if (!make_map(&a, h, (uint64_t)S, (uint64_t)F, BM) ||
-        !make_map(&b0, w2, (uint64_t)E * D, (uint64_t)F, BN))
+    if (!make_map(&a, h, (uint64_t)S, (uint64_t)F, arows) ||
+        !make_map(&b0, w2, (uint64_t)E * D, (uint64_t)F, DownWide::BN))
         return cudaErrorInvalidValue;
-    return launch_gemm<kDown>(a, b0, b0, offsets, E, S, F, D, nullptr, y_sorted, st);
+    return launch_gemm<kDown, DownWide>(a, b0, b0, offsets, E, S, F, D, arows * BK * 2, nullptr,
+                                        y_sorted, st);
 }
 
 }  // namespace moe
