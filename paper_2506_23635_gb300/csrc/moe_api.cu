@@ -161,123 +161,150 @@ k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restri
     select_topk(E, K, t0 + warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate, nullptr);
 }
 
+// ---------------------------------------------------------------------------
+// Staged router for the tiny-batch kernel: the whole W_r [D, E] is
+// bulk-copied into shared memory (one wait for memory), then every token's
+// logits are computed by 8/n warps that each take a slice of d and add their
+// partial sums in a fixed order; the token rows are read from global memory
+// (coalesced across the warp).  (For larger batches k_route, which shares
+// each router row load among 4 tokens, measured faster.)
+// ---------------------------------------------------------------------------
+constexpr int kStagedWarps = 8;
+constexpr int kStagedThreads = kStagedWarps * 32;
+constexpr size_t kStagedRouterMax = 196 * 1024 + 1024;  // W_r bytes that are staged
+
+// 16 experts' partial logits of one token over rows [d_lo, d_hi) of a router
+// held in shared memory; lane l takes rows d_lo + l, d_lo + l + 32, ... so a
+// warp reads 32 consecutive router rows per step (no bank conflicts beyond
+// 2-way).  Summed across the warp (every lane ends with all 16).
+template <typename TX, typename TW>
+__device__ __forceinline__ void warp_logits16(const TX *xrow, const TW *wr_s, int E, int e0, int ne,
+                                              int d_lo, int d_hi, float (&acc)[16]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+    const bool vec = (E % 8) == 0 && sizeof(TW) == 2;
+#pragma unroll 4
+    for (int d = d_lo + lane; d < d_hi; d += 32) {
+        const float xv = to_f(xrow[d]);
+        const TW *row = wr_s + (size_t)d * E + e0;
+        float w[16];
+        if (vec) {
+            const uint4 u0 = *reinterpret_cast<const uint4 *>(row);
+            unpack_bf16x2(u0.x, w[0], w[1]); unpack_bf16x2(u0.y, w[2], w[3]);
+            unpack_bf16x2(u0.z, w[4], w[5]); unpack_bf16x2(u0.w, w[6], w[7]);
+            if (ne > 8) {
+                const uint4 u1 = *reinterpret_cast<const uint4 *>(row + 8);
+                unpack_bf16x2(u1.x, w[8], w[9]); unpack_bf16x2(u1.y, w[10], w[11]);
+                unpack_bf16x2(u1.z, w[12], w[13]); unpack_bf16x2(u1.w, w[14], w[15]);
+            } else {
+#pragma unroll
+                for (int j = 8; j < 16; ++j) w[j] = 0.f;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) w[j] = j < ne ? to_f(row[j]) : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < 16; ++j) acc[j] = fmaf(xv, w[j], acc[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) acc[j] = warp_sum(acc[j]);
+}
+
+// Stage W_r into dynamic shared memory (bulk copies on one mbarrier).
+template <typename TW>
+__device__ __forceinline__ bool stage_router(unsigned char *dst, const TW *wr, uint32_t bytes,
+                                             uint64_t *bar, unsigned *err) {
+    if (threadIdx.x == 0) {
+        const uint64_t pol = ptx::policy_evict_last();
+        ptx::mbar_arrive_expect_tx(bar, bytes);
+        constexpr uint32_t kChunk = 32768;
+        for (uint32_t o = 0; o < bytes; o += kChunk)
+            ptx::bulk_g2s(dst + o, reinterpret_cast<const unsigned char *>(wr) + o,
+                          min(kChunk, bytes - o), bar, pol);
+    }
+    return ptx::mbar_wait(bar, 0, err);
+}
+
+// Logits + top-k of tokens [t0, t0+n) (n <= 8) by the 8 warps of the block.
+template <typename TX, typename TW>
+__device__ void staged_batch(int t0, int n, int D, int E, int K, const TX *__restrict__ x,
+                             const TW *wr_s, float (*part)[256], float (*lg)[256],
+                             float (*pk)[256], float *__restrict__ logits_opt,
+                             int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
+                             int *sidx) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpt = kStagedWarps / n;  // warps per token
+    const int tk = warp / wpt, pt = warp - tk * wpt;
+    if (tk < n) {
+        const int d_lo = (int)((long long)D * pt / wpt), d_hi = (int)((long long)D * (pt + 1) / wpt);
+        const TX *xrow = x + (size_t)(t0 + tk) * D;
+        for (int e0 = 0; e0 < E; e0 += 16) {
+            const int ne = min(16, E - e0);
+            float acc[16];
+            warp_logits16<TX, TW>(xrow, wr_s, E, e0, ne, d_lo, d_hi, acc);
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                if (lane == j && j < ne) part[warp][e0 + j] = acc[j];
+        }
+    }
+    __syncthreads();
+    if (warp < n) {
+        for (int e = lane; e < E; e += 32) {
+            float v = 0.f;
+            for (int p = 0; p < wpt; ++p) v += part[warp * wpt + p][e];
+            lg[warp][e] = v;
+        }
+        __syncwarp();
+        select_topk(E, K, t0 + warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
+                    sidx ? sidx + warp * K : nullptr);
+    }
+    __syncthreads();
+}
+
 // Route and dispatch of a tiny batch (T <= 4, T*K <= 32) in one block: the
 // top-k indices stay in shared memory and warp 0 ranks the slots (ranks of
 // equal experts from __match_any_sync, so the order is the stable one).
-// When the router matrix and the tokens fit in shared memory (STAGED), they
-// are brought in first by bulk copies on one mbarrier, so the block waits for
-// memory once instead of once per loop trip.
+// When the router matrix fits in shared memory (`staged`) it is bulk-copied
+// there first.
 template <typename TX, typename TW>
-__device__ void smem_logits(int D, int E, const TX *xs, const TW *wrs, int nt, float (*lg)[256],
-                            float (*red)[kRouteTokens * 16]) {
-    constexpr int TT = kRouteTokens, NT = kSmallThreads, NW = NT / 32;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const bool vec = (E % 8) == 0;
-    for (int e0 = 0; e0 < E; e0 += 16) {
-        const int ne = min(16, E - e0);
-        float acc[TT][16];
-#pragma unroll
-        for (int a = 0; a < TT; ++a)
-#pragma unroll
-            for (int j = 0; j < 16; ++j) acc[a][j] = 0.f;
-        for (int d = threadIdx.x; d < D; d += NT) {
-            float xv[TT];
-#pragma unroll
-            for (int a = 0; a < TT; ++a) xv[a] = a < nt ? to_f(xs[(size_t)a * D + d]) : 0.f;
-            const TW *wrow = wrs + (size_t)d * E + e0;
-            float w[16];
-            if (vec && sizeof(TW) == 2) {
-                const uint4 u0 = *reinterpret_cast<const uint4 *>(wrow);
-                unpack_bf16x2(u0.x, w[0], w[1]); unpack_bf16x2(u0.y, w[2], w[3]);
-                unpack_bf16x2(u0.z, w[4], w[5]); unpack_bf16x2(u0.w, w[6], w[7]);
-                if (ne > 8) {
-                    const uint4 u1 = *reinterpret_cast<const uint4 *>(wrow + 8);
-                    unpack_bf16x2(u1.x, w[8], w[9]); unpack_bf16x2(u1.y, w[10], w[11]);
-                    unpack_bf16x2(u1.z, w[12], w[13]); unpack_bf16x2(u1.w, w[14], w[15]);
-                } else {
-#pragma unroll
-                    for (int j = 8; j < 16; ++j) w[j] = 0.f;
-                }
-            } else {
-#pragma unroll
-                for (int j = 0; j < 16; ++j) w[j] = j < ne ? to_f(wrow[j]) : 0.f;
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-#pragma unroll
-                for (int a = 0; a < TT; ++a) acc[a][j] = fmaf(xv[a], w[j], acc[a][j]);
-        }
-#pragma unroll
-        for (int a = 0; a < TT; ++a) {
-            if (a >= nt) break;
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const float v = warp_sum(acc[a][j]);
-                if (lane == 0) red[warp][a * 16 + j] = v;
-            }
-        }
-        __syncthreads();
-        for (int i = threadIdx.x; i < TT * 16; i += NT) {
-            const int a = i >> 4, j = i & 15;
-            if (a < nt && j < ne) {
-                float s = 0.f;
-#pragma unroll
-                for (int w = 0; w < NW; ++w) s += red[w][i];
-                lg[a][e0 + j] = s;
-            }
-        }
-        __syncthreads();
-    }
-}
-
-template <typename TX, typename TW>
-__global__ void __launch_bounds__(kSmallThreads)
+__global__ void __launch_bounds__(kStagedThreads)
 k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
                        const TW *__restrict__ wr, float *__restrict__ logits_opt,
                        int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
                        int32_t *__restrict__ counts, int32_t *__restrict__ offsets,
                        int32_t *__restrict__ perm, int32_t *__restrict__ inv_perm, int staged,
                        unsigned *err) {
-    extern __shared__ __align__(128) unsigned char dsm[];  // staged: W_r, then x
-    __shared__ float red[kSmallThreads / 32][kRouteTokens * 16];
-    __shared__ float lg[kRouteTokens][256];
-    __shared__ float pk[kRouteTokens][256];
+    extern __shared__ __align__(128) unsigned char wsm[];  // W_r when staged
+    __shared__ float part[kStagedWarps][256];
+    __shared__ float lg[kStagedWarps][256];
+    __shared__ float pk[kStagedWarps][256];
     __shared__ int sidx[kSmallMaxSlots];
     __shared__ int cnt[256];
     __shared__ int offs[257];
     __shared__ uint64_t bar;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int e = threadIdx.x; e < E; e += kSmallThreads) cnt[e] = 0;
+    for (int e = threadIdx.x; e < E; e += kStagedThreads) cnt[e] = 0;
     if (staged) {
-        const uint32_t wr_bytes = (uint32_t)D * E * sizeof(TW);
-        const uint32_t x_off = (wr_bytes + 127u) & ~127u;
-        const uint32_t x_bytes = (uint32_t)T * D * sizeof(TX);
         if (threadIdx.x == 0) {
             ptx::mbar_init(&bar, 1);
             ptx::fence_barrier_init();
         }
         __syncthreads();
         ptx::grid_dependency_wait();  // x may come from the previous kernel
-        if (threadIdx.x == 0) {
-            const uint64_t pol = ptx::policy_evict_last();
-            ptx::mbar_arrive_expect_tx(&bar, wr_bytes + x_bytes);
-            constexpr uint32_t kChunk = 32768;
-            for (uint32_t o = 0; o < wr_bytes; o += kChunk)
-                ptx::bulk_g2s(dsm + o, reinterpret_cast<const unsigned char *>(wr) + o,
-                              min(kChunk, wr_bytes - o), &bar, pol);
-            ptx::bulk_g2s(dsm + x_off, x, x_bytes, &bar, pol);
-        }
-        if (!ptx::mbar_wait(&bar, 0, err)) return;  // every thread waits; none has synced since
-        smem_logits<TX, TW>(D, E, reinterpret_cast<const TX *>(dsm + x_off),
-                            reinterpret_cast<const TW *>(dsm), T, lg, red);
+        if (!stage_router<TW>(wsm, wr, (uint32_t)((size_t)D * E * sizeof(TW)), &bar, err)) return;
+        staged_batch<TX, TW>(0, T, D, E, K, x, reinterpret_cast<const TW *>(wsm), part, lg, pk,
+                             logits_opt, topk_idx, topk_gate, sidx);
     } else {
         ptx::grid_dependency_wait();
-        block_logits<TX, TW, kSmallThreads>(D, E, x, wr, 0, T, lg, red);
+        block_logits<TX, TW, kStagedThreads>(D, E, x, wr, 0, T, lg,
+                                            reinterpret_cast<float (*)[kRouteTokens * 16]>(part));
+        if (warp < T)
+            select_topk(E, K, warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
+                        sidx + warp * K);
+        __syncthreads();
     }
-    if (warp < T)
-        select_topk(E, K, warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
-                    sidx + warp * K);
-    __syncthreads();
     if (warp != 0) return;
     const int S = T * K;
     const int e = lane < S ? sidx[lane] : -1;
@@ -627,6 +654,10 @@ bool ok_opt(const void *p) { return p == nullptr || aligned16(p); }
 
 moe_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA; }
 
+size_t router_bytes(const moe_dims &d) {
+    return (size_t)d.d_model * d.n_experts * (d.w_dtype == MOE_BF16 ? 2 : 4);
+}
+
 template <typename TX, typename TW>
 cudaError_t launch_route(const moe_dims &d, int T, const void *x, const void *wr, float *logits,
                          int32_t *idx, float *gate, cudaStream_t st) {
@@ -648,21 +679,18 @@ cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x,
     const TW *wp = static_cast<const TW *>(wr);
     float *logits = nullptr;
     unsigned *err = device_info().err;
-    // stage W_r and x in shared memory when they fit next to the static arrays
-    const size_t wr_bytes = (size_t)D * E * sizeof(TW);
-    const size_t dyn = ((wr_bytes + 127) & ~size_t(127)) + (size_t)T * D * sizeof(TX);
-    int staged = dyn <= kSmallStageBytes ? 1 : 0;
+    const size_t wrb = router_bytes(d);
+    int staged = wrb <= kStagedRouterMax ? 1 : 0;
     const void *kern = (const void *)k_route_dispatch_small<TX, TW>;
-    const size_t smem = staged ? dyn : 0;
     if (staged) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kSmallStageBytes);
+                                             (int)kStagedRouterMax);
         if (e != cudaSuccess) return e;
     }
     void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &logits, &idx, &gate, &counts, &offsets, &perm, &inv,
                     &staged, &err};
     LaunchScope ls("route_dispatch_small", st);
-    return launch_pdl(kern, dim3(1), dim3(kSmallThreads), smem, st, args);
+    return launch_pdl(kern, dim3(1), dim3(kStagedThreads), staged ? wrb : 0, st, args);
 }
 
 bool small_route_ok(const moe_dims &d, int T) {
