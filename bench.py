@@ -491,6 +491,31 @@ def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True):
     return res
 
 
+def measure_dense(layer, T, steps=100, warmup=3):
+    """Busy full loading (Sec. 4.2) on the same layer: every expert computes
+    every token, unselected gates zero -- the paper's static baseline."""
+    shape = layer.shape
+    _, _, xs, w_r, _, out = layer.inputs(T, 16)
+    w1, v1, w2 = layer.w
+    d, moe = layer.d, layer.moe
+    import torch
+
+    ws = torch.empty(moe.dense_workspace_size(d, T), dtype=torch.uint8, device=layer.dev)
+
+    def step(i):
+        moe.layer_forward_dense(d, xs[i % 16], w_r, w1, v1, w2, out=out, ws=ws, stream=layer.stream)
+
+    for i in range(warmup):
+        step(i)
+    ms, _, kstats = layer.time_steps(step, steps)
+    all_bytes = shape.n_experts * 3 * shape.d_model * shape.ffn_hidden * 2
+    peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
+    return {"tokens_per_step": T, "ms_per_step": round(ms, 4),
+            "achieved_hbm_gbs_step": round(all_bytes / (ms / 1e3) / 1e9, 1),
+            "frac_of_hbm_step": round(all_bytes / (ms / 1e3) / 1e9 / peak, 4),
+            "kernels": kernel_table(kstats)}
+
+
 def run_ours(args):
     import torch
 
@@ -561,6 +586,7 @@ def run_ours(args):
         extra["prefill"] = measure_extra(layer, "dbrx-prefill-t2048", 20, 3)
         extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5)
                                  for t in (2, 4, 8, 16, 32, 64)]
+        extra["busy_full_loading"] = [measure_dense(layer, t) for t in (1, 8)]
         extra["stack"] = measure_stack(moe, dev)
 
     if rank != 0:

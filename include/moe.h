@@ -154,6 +154,23 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x,
                              const void *residual_opt, void *out, void *ws,
                              size_t ws_bytes, moe_stream_t stream);
 
+/* ---- busy full loading (comparison baseline) -----------------------------
+ * Sec. 4.2 "Busy Full Loading": every expert computes every token and the
+ * outputs of the experts the router did not select are zeroed in the
+ * weighted sum.  The result equals moe_layer_forward's (within rounding);
+ * the cost is all E experts' weights and E/K times the FLOPs.  Kept as the
+ * baseline the paper's sparse strategies are measured against.
+ * Same arguments as moe_layer_forward; bf16 weights only (else
+ * MOE_ERR_UNSUPPORTED); workspace of moe_dense_workspace_size bytes. */
+moe_status moe_dense_workspace_size(const moe_dims *dims, int32_t max_tokens,
+                                    size_t *bytes);
+moe_status moe_layer_forward_dense(const moe_dims *dims, int32_t T,
+                                   const void *x, const void *w_router,
+                                   const void *w1, const void *v1,
+                                   const void *w2, const void *residual_opt,
+                                   void *out, void *ws, size_t ws_bytes,
+                                   moe_stream_t stream);
+
 /* ---- stack of layers (decode through consecutive MoE blocks) -------------
  * The paper runs DBRX's 40 decoder layers (Table 1); a stack of MoE blocks
  * needs the glue between them, which the paper does not print.  Reading
@@ -226,8 +243,9 @@ moe_status moe_get_last_error(moe_stream_t stream);
  * moe_get_last_error returns MOE_ERR_TIMEOUT.  The context stays usable.
  * Host-side fault injection: with MOE_INJECT_FAILURE="<entry>:<status>" in
  * the environment, the named entry point (moe_route, moe_dispatch,
- * moe_expert_ffn, moe_combine, moe_layer_forward, moe_prenorm,
- * moe_stack_forward) returns that status at once without launching. */
+ * moe_expert_ffn, moe_combine, moe_layer_forward, moe_layer_forward_dense,
+ * moe_prenorm, moe_stack_forward) returns that status at once without
+ * launching. */
 moe_status moe_selftest_wait_timeout(uint64_t limit_ns, int32_t *gave_up,
                                      moe_stream_t stream);
 

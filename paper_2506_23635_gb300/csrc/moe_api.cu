@@ -483,6 +483,28 @@ k_prenorm(int T, int D, const TR *__restrict__ r, TX *__restrict__ xn, float eps
 }
 
 // ===========================================================================
+// Busy full loading (Sec. 4.2): every expert takes every token, and the
+// experts the router did not select get gate 0 in the weighted sum.
+// k_densify turns the top-k routing into that dense form: slot (t, e) of
+// the dense layout has expert e and gate g[t,k] if e = idx[t,k], else 0.
+// ===========================================================================
+__global__ void __launch_bounds__(256)
+k_densify(int T, int E, int K, const int32_t *__restrict__ idx, const float *__restrict__ gate,
+          int32_t *__restrict__ didx, float *__restrict__ dgate) {
+    ptx::grid_dependency_wait();
+    const long long total = (long long)T * E;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int t = (int)(i / E), e = (int)(i - (long long)t * E);
+        float g = 0.f;
+        for (int k = 0; k < K; ++k)
+            if (idx[(size_t)t * K + k] == e) g = gate[(size_t)t * K + k];
+        didx[i] = e;
+        dgate[i] = g;
+    }
+}
+
+// ===========================================================================
 // Self-test of the bounded waits: one thread waits on an mbarrier that
 // nothing will complete.  The wait gives up after limit_ns, records
 // kErrTimeout and the kernel returns normally.
@@ -976,6 +998,71 @@ moe_status moe_stack_forward(const moe_dims *dims, int32_t n_layers, int32_t T,
         if (s != MOE_OK) return s;
     }
     return MOE_OK;
+}
+
+// Dense (busy-full-loading) layout: the layer's own workspace for top_k = E,
+// followed by the sparse routing [T, K] (indices and gates).
+moe_status moe_dense_workspace_size(const moe_dims *dims, int32_t max_tokens, size_t *bytes) {
+    moe_status s = check_dims(dims);
+    if (s == MOE_ERR_UNSUPPORTED) s = MOE_OK;
+    if (s != MOE_OK) return s;
+    if (!bytes || max_tokens < 0) return MOE_ERR_INVALID_ARG;
+    moe_dims dd = *dims;
+    dd.top_k = dims->n_experts;
+    if ((s = check_T(&dd, max_tokens)) != MOE_OK) return s;
+    const size_t sparse = (((size_t)max_tokens * dims->top_k * 8) + 255) & ~size_t(255);
+    *bytes = ws_layout(dd, max_tokens).total + sparse;
+    return MOE_OK;
+}
+
+moe_status moe_layer_forward_dense(const moe_dims *dims, int32_t T, const void *x,
+                                   const void *w_router, const void *w1, const void *v1,
+                                   const void *w2, const void *residual_opt, void *out, void *ws,
+                                   size_t ws_bytes, moe_stream_t stream) {
+    MOE_INJECT("moe_layer_forward_dense");
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    moe_dims dd = *dims;
+    dd.top_k = dims->n_experts;  // every expert takes every token
+    if ((s = check_T(&dd, T)) != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(x) || !ok_ptr(w_router) || !ok_ptr(w1) || !ok_ptr(v1) || !ok_ptr(w2) ||
+        !ok_opt(residual_opt) || !ok_ptr(out))
+        return MOE_ERR_INVALID_ARG;
+    if (!tc_path_ok(*dims)) return MOE_ERR_UNSUPPORTED;
+    size_t need = 0;
+    if ((s = moe_dense_workspace_size(dims, T, &need)) != MOE_OK) return s;
+    if (!ws || !aligned16(ws) || ws_bytes < need) return MOE_ERR_WORKSPACE;
+    const WsLayout L = ws_layout(dd, T);
+    cudaStream_t st = (cudaStream_t)stream;
+    int32_t *sidx = at<int32_t>(ws, L.total);
+    float *sgate = at<float>(ws, L.total + (size_t)T * dims->top_k * 4);
+    int32_t *didx = at<int32_t>(ws, L.idx);
+    float *dgate = at<float>(ws, L.gate);
+    int32_t *counts = at<int32_t>(ws, L.counts);
+    int32_t *offsets = at<int32_t>(ws, L.offsets);
+    int32_t *perm = at<int32_t>(ws, L.perm);
+    int32_t *inv = at<int32_t>(ws, L.inv_perm);
+    void *h = at<void>(ws, L.h);
+    void *xs = at<void>(ws, L.xs);
+    float *y = at<float>(ws, L.y);
+
+    cudaError_t e = route_any(*dims, T, x, w_router, nullptr, sidx, sgate, st);
+    if (e == cudaSuccess) {
+        const long long total = (long long)T * dd.n_experts;
+        const int grid = (int)std::max(1LL, std::min((total + 255) / 256,
+                                                     (long long)device_info().sm_count * 8));
+        int Tv = T, E = dd.n_experts, K = dims->top_k;
+        void *args[] = {&Tv, &E, &K, &sidx, &sgate, &didx, &dgate};
+        LaunchScope ls("densify", st);
+        e = launch_pdl((const void *)k_densify, dim3(grid), dim3(256), 0, st, args);
+    }
+    if (e == cudaSuccess) e = dispatch_any(dd, T, didx, counts, offsets, perm, inv, st);
+    if (e == cudaSuccess) e = launch_gather_rows(dd, T, x, perm, xs, st);
+    if (e == cudaSuccess) e = launch_gemm_up_tc(dd, T, xs, offsets, w1, v1, h, st);
+    if (e == cudaSuccess) e = launch_gemm_down_tc(dd, T, h, offsets, w2, y, st);
+    if (e == cudaSuccess) e = combine_any(dd, T, y, inv, dgate, residual_opt, out, st);
+    return cuda_status(e);
 }
 
 const char *moe_status_string(moe_status status) {

@@ -29,7 +29,7 @@ EXPORTS = (
     "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
     "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc", "moe_status_string",
     "moe_prenorm", "moe_stack_workspace_size", "moe_stack_forward",
-    "moe_selftest_wait_timeout",
+    "moe_selftest_wait_timeout", "moe_dense_workspace_size", "moe_layer_forward_dense",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
     "moe_profile_reset", "moe_profile_read",
 )
@@ -85,6 +85,8 @@ def lib() -> ctypes.CDLL:
         "moe_layer_forward_noalloc": [DP, I32, P, P, P, P, P, P, P, P],
         "moe_prenorm": [DP, I32, P, P, ctypes.c_float, P],
         "moe_selftest_wait_timeout": [ctypes.c_uint64, P, P],
+        "moe_dense_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
+        "moe_layer_forward_dense": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
         "moe_stack_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
         "moe_stack_forward": [DP, I32, I32, ctypes.POINTER(P), ctypes.POINTER(P),
                               ctypes.POINTER(P), ctypes.POINTER(P), P, ctypes.c_float, P, SZ, P],
@@ -277,6 +279,28 @@ def selftest_wait_timeout(limit_ns: int, stream=None) -> bool:
     _check(lib().moe_selftest_wait_timeout(limit_ns, _ptr(flag), _stream(stream)),
            "moe_selftest_wait_timeout")
     return bool(flag.item())
+
+
+def dense_workspace_size(d: Dims, max_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().moe_dense_workspace_size(ctypes.byref(d), max_tokens, ctypes.byref(n)),
+           "moe_dense_workspace_size")
+    return int(n.value)
+
+
+def layer_forward_dense(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, ws=None,
+                        stream=None):
+    """Busy full loading (Sec. 4.2): all experts on all tokens, unselected
+    gates zero.  Returns out [T, D] (out_dtype)."""
+    T = x.shape[0]
+    if out is None:
+        out = torch.empty((T, d.d_model), dtype=_tdt(d.out_dtype), device=x.device)
+    if ws is None:
+        ws = torch.empty(max(dense_workspace_size(d, T), 256), dtype=torch.uint8, device=x.device)
+    _check(lib().moe_layer_forward_dense(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(w1),
+                                         _ptr(v1), _ptr(w2), _ptr(residual), _ptr(out), _ptr(ws),
+                                         ws.numel(), _stream(stream)), "moe_layer_forward_dense")
+    return out
 
 
 def get_last_error(stream=None) -> int:

@@ -219,3 +219,44 @@ def test_launch_count_and_profile(T, kernels):
     assert m.launch_count() - n0 == sum(v[0] for v in stats.values()) == len(kernels)
     assert set(stats) == kernels
     assert all(v[1] > 0 for v in stats.values())
+
+
+@pytest.mark.parametrize("case", [(64, 96, 8, 2, 1), (128, 136, 16, 4, 9), (72, 40, 5, 3, 33)],
+                         ids=lambda c: "D{}F{}E{}K{}T{}".format(*c))
+def test_busy_full_loading_equals_sparse(case):
+    """Sec. 4.2 busy full loading (all experts, unselected gates zero) gives
+    the same layer as the sparse path: against the oracle's busy-full-loading
+    route and against the sparse CUDA path."""
+    m = moe()
+    D, F, E, K, T = case
+    L = _host((D, F, E, K, T, "bf16"), seed=19)
+    d = _dims(m, L.shape)
+    want = oracle.layer_dense_masked(L.x, L.w_r, L.w1, L.v1, L.w2, "bf16", K)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    dense = m.layer_forward_dense(d, x, w_r, w1, v1, w2)
+    assert m.get_last_error() == 0
+    assert_parity(to_numpy(dense), want, "bf16", "busy full loading vs oracle")
+    sparse = m.layer_forward(d, x, w_r, w1, v1, w2)
+    assert_parity(to_numpy(dense), to_numpy(sparse), "bf16", "busy full loading vs sparse")
+
+
+@pytest.mark.parametrize("case", [
+    (16384, 256, 4, 2, 1, "bf16"),     # wide token rows: too wide for the streaming kernels
+    (256, 16384, 4, 2, 3, "bf16"),     # wide hidden layer
+    (128, 192, 8, 2, 2048, "bf16"),    # many slot tiles per expert
+    (256, 512, 4, 2, 1, "f32"),        # one token on the fp32 path
+], ids=lambda c: "D{}F{}E{}K{}T{}{}".format(*c))
+def test_size_extremes(case):
+    m = moe()
+    D, F, E, K, T, dt = case
+    L = _host(case, seed=23)
+    sh = L.shape
+    d = _dims(m, sh)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    out = m.layer_forward(d, x, w_r, w1, v1, w2)
+    assert m.get_last_error() == 0
+    toks = np.unique(np.linspace(0, T - 1, min(T, 24)).astype(np.int32))
+    want, idx, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, dt, K, tokens=toks)
+    gi, _, _ = m.route(d, x, w_r)
+    assert np.array_equal(gi.cpu().numpy()[toks], idx)
+    assert_parity(to_numpy(out)[toks], want, dt, f"extremes {case}")
