@@ -9,6 +9,8 @@
 #include <string>
 #include <vector>
 
+#include <cooperative_groups.h>
+
 #include "moe_internal.cuh"
 #include "ptx.cuh"
 
@@ -334,6 +336,170 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
         const int pos = offs[e] + __popc(same & ((1u << lane) - 1u));
         perm[pos] = lane;
         inv_perm[lane] = pos;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Route and dispatch of a decode batch (T <= 64, T*K <= 256) in one launch of
+// a cluster of kClusterCtas CTAs.  CTA r bulk-copies rows [d0_r, d1_r) of W_r
+// into its shared memory and computes the partial logits of every token over
+// that slice of d; after a cluster barrier CTA 0 adds the kClusterCtas
+// partials in rank order (reading them through distributed shared memory),
+// selects the top-k of every token and ranks all T*K slots with a stable
+// counting sort, as k_dispatch does.  A second cluster barrier keeps the
+// other CTAs (and their shared memory) alive until CTA 0 has read it.
+// ---------------------------------------------------------------------------
+constexpr int kClusterCtas = 8;
+constexpr int kClusterThreads = 256;
+constexpr int kClusterMaxTokens = 64;
+constexpr int kClusterMaxSlots = 256;
+
+template <typename TX, typename TW>
+__global__ void __launch_bounds__(kClusterThreads)
+k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
+                         const TW *__restrict__ wr, int32_t *__restrict__ topk_idx,
+                         float *__restrict__ topk_gate, int32_t *__restrict__ counts,
+                         int32_t *__restrict__ offsets, int32_t *__restrict__ perm,
+                         int32_t *__restrict__ inv_perm, unsigned *err) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ __align__(128) unsigned char dsm[];
+    // dynamic: partial logits [T][E] fp32, then the staged router slice
+    float *part = reinterpret_cast<float *>(dsm);
+    const size_t part_bytes = (((size_t)T * E * 4) + 127) & ~size_t(127);
+    TW *wr_s = reinterpret_cast<TW *>(dsm + part_bytes);
+    __shared__ float pk[kStagedWarps][256];
+    __shared__ int sidx[kClusterMaxSlots];
+    __shared__ int cnt[256], run[256];
+    __shared__ int wh[kClusterThreads / 32][256];
+    __shared__ uint64_t bar;
+    const int rank = (int)cluster.block_rank();
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // this CTA's rows of d, a multiple of 8 rows (16-byte aligned slices)
+    const int n8 = D >> 3;
+    const int d0 = (int)((long long)n8 * rank / kClusterCtas) * 8;
+    const int d1 = (int)((long long)n8 * (rank + 1) / kClusterCtas) * 8;
+    const int dn = d1 - d0;
+
+    if (tid == 0) {
+        ptx::mbar_init(&bar, 1);
+        ptx::fence_barrier_init();
+    }
+    __syncthreads();
+    ptx::grid_dependency_wait();  // x may come from the previous kernel
+    bool ok = true;
+    if (dn > 0)
+        ok = stage_router<TW>(reinterpret_cast<unsigned char *>(wr_s), wr + (size_t)d0 * E,
+                              (uint32_t)((size_t)dn * E * sizeof(TW)), &bar, err);
+    // partial logits: token t is taken by a group of P threads (P = 256/T,
+    // at most 32), thread p of the group accumulating 16 experts over rows
+    // p, p+P, ... of the slice; the group then adds its P sums with shuffles
+    const int O = T * E;
+    int P = 32;
+    while (P > 1 && P * T > kClusterThreads) P >>= 1;
+    const int groups = kClusterThreads / P;
+    const int gp = tid % P;
+    const bool vec = (E % 8) == 0 && sizeof(TW) == 2;
+    for (int t0 = 0; t0 < T; t0 += groups) {
+        const int t = t0 + tid / P;
+        const TX *xr = x + (size_t)(t < T ? t : 0) * D + d0;
+        for (int e0 = 0; e0 < E; e0 += 16) {
+            const int ne = min(16, E - e0);
+            float acc[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+            if (ok && t < T) {
+#pragma unroll 4
+                for (int d = gp; d < dn; d += P) {
+                    const float xv = to_f(xr[d]);
+                    const TW *row = wr_s + (size_t)d * E + e0;
+                    float w[16];
+                    if (vec) {
+                        const uint4 u0 = *reinterpret_cast<const uint4 *>(row);
+                        unpack_bf16x2(u0.x, w[0], w[1]); unpack_bf16x2(u0.y, w[2], w[3]);
+                        unpack_bf16x2(u0.z, w[4], w[5]); unpack_bf16x2(u0.w, w[6], w[7]);
+                        if (ne > 8) {
+                            const uint4 u1 = *reinterpret_cast<const uint4 *>(row + 8);
+                            unpack_bf16x2(u1.x, w[8], w[9]); unpack_bf16x2(u1.y, w[10], w[11]);
+                            unpack_bf16x2(u1.z, w[12], w[13]); unpack_bf16x2(u1.w, w[14], w[15]);
+                        } else {
+#pragma unroll
+                            for (int j = 8; j < 16; ++j) w[j] = 0.f;
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) w[j] = j < ne ? to_f(row[j]) : 0.f;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) acc[j] = fmaf(xv, w[j], acc[j]);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                for (int off = P >> 1; off > 0; off >>= 1)
+                    acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], off);
+            if (t < T && gp == 0)
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    if (j < ne) part[(size_t)t * E + e0 + j] = acc[j];
+        }
+    }
+    cluster.sync();  // every CTA's partials are written
+    if (rank == 0) {
+        for (int o = tid; o < O; o += kClusterThreads) {
+            float v = 0.f;
+            for (int r = 0; r < kClusterCtas; ++r) v += cluster.map_shared_rank(part, r)[o];
+            part[o] = v;  // own partial was read first (r = 0)
+        }
+    }
+    cluster.sync();  // CTA 0 has read every partial; the others may leave
+    if (rank != 0) return;
+    __syncthreads();
+    // top-k of every token, one warp per token
+    for (int t = warp; t < T; t += kClusterThreads / 32)
+        select_topk(E, K, t, part + (size_t)t * E, pk[warp], nullptr, topk_idx, topk_gate,
+                    sidx + t * K);
+    // stable dispatch of the S <= 256 slots (one chunk of k_dispatch)
+    const int S = T * K;
+    for (int e = tid; e < E; e += kClusterThreads) cnt[e] = 0;
+    __syncthreads();
+    for (int sl = tid; sl < S; sl += kClusterThreads) atomicAdd(&cnt[sidx[sl]], 1);
+    __syncthreads();
+    if (warp == 0) {
+        int carry = 0;
+        for (int b0 = 0; b0 < E; b0 += 32) {
+            const int e = b0 + lane;
+            const int c = e < E ? cnt[e] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (e < E) {
+                run[e] = carry + incl - c;
+                counts[e] = c;
+                offsets[e] = carry + incl - c;
+            }
+            carry += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) offsets[E] = carry;
+    }
+    constexpr int NW = kClusterThreads / 32;
+    for (int i = tid; i < NW * E; i += kClusterThreads) wh[i / E][i % E] = 0;
+    __syncthreads();
+    const int sl = tid;
+    const int e = sl < S ? sidx[sl] : -1;
+    const unsigned same = __match_any_sync(0xffffffffu, e);
+    const int rk = __popc(same & ((1u << lane) - 1u));
+    if (e >= 0 && rk == 0) wh[warp][e] = __popc(same);
+    __syncthreads();
+    if (e >= 0) {
+        int pre = 0;
+        for (int w = 0; w < warp; ++w) pre += wh[w][e];
+        const int pos = run[e] + pre + rk;
+        perm[pos] = sl;
+        inv_perm[sl] = pos;
     }
 }
 
@@ -715,6 +881,62 @@ cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x,
     return launch_pdl(kern, dim3(1), dim3(kStagedThreads), staged ? wrb : 0, st, args);
 }
 
+template <typename TX, typename TW>
+cudaError_t launch_route_dispatch_cluster(const moe_dims &d, int T, const void *x,
+                                          const void *wr, int32_t *idx, float *gate,
+                                          int32_t *counts, int32_t *offsets, int32_t *perm,
+                                          int32_t *inv, cudaStream_t st) {
+    int Tv = T, D = d.d_model, E = d.n_experts, K = d.top_k;
+    const TX *xp = static_cast<const TX *>(x);
+    const TW *wp = static_cast<const TW *>(wr);
+    unsigned *err = device_info().err;
+    const int rows = (D / 8 + kClusterCtas - 1) / kClusterCtas * 8;
+    const size_t part_bytes = (((size_t)T * E * 4) + 127) & ~size_t(127);
+    const size_t smem = part_bytes + (size_t)rows * E * sizeof(TW);
+    const void *kern = (const void *)k_route_dispatch_cluster<TX, TW>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &idx, &gate, &counts, &offsets, &perm, &inv, &err};
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kClusterCtas);
+    cfg.blockDim = dim3(kClusterThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kClusterCtas;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    LaunchScope ls("route_dispatch_cluster", st);
+    return cudaLaunchKernelExC(&cfg, kern, args);
+}
+
+// Shared memory of the cluster kernel: the partial logits and one CTA's
+// eighth of the router.
+bool cluster_route_ok(const moe_dims &d, int T) {
+    if (T < 1 || T > kClusterMaxTokens || T * d.top_k > kClusterMaxSlots) return false;
+    const int rows = (d.d_model / 8 + kClusterCtas - 1) / kClusterCtas * 8;
+    const size_t smem = (((size_t)T * d.n_experts * 4) + 127) +
+                        (size_t)rows * d.n_experts * (d.w_dtype == MOE_BF16 ? 2 : 4);
+    return smem <= 160 * 1024;
+}
+
+cudaError_t route_dispatch_cluster_any(const moe_dims &d, int T, const void *x, const void *wr,
+                                       int32_t *idx, float *gate, int32_t *counts,
+                                       int32_t *offsets, int32_t *perm, int32_t *inv,
+                                       cudaStream_t st) {
+    if (d.w_dtype == MOE_BF16)
+        return launch_route_dispatch_cluster<bf16, bf16>(d, T, x, wr, idx, gate, counts, offsets,
+                                                         perm, inv, st);
+    return launch_route_dispatch_cluster<float, float>(d, T, x, wr, idx, gate, counts, offsets,
+                                                       perm, inv, st);
+}
+
 bool small_route_ok(const moe_dims &d, int T) {
     return T <= kRouteTokens && T * d.top_k <= kSmallMaxSlots;
 }
@@ -907,7 +1129,12 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
     float *h = at<float>(ws, L.h);
 
     cudaError_t e;
-    if (small_route_ok(d, T)) {
+    if (T == 1 && small_route_ok(d, T)) {
+        e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
+    } else if (cluster_route_ok(d, T)) {
+        e = route_dispatch_cluster_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv,
+                                       st);
+    } else if (small_route_ok(d, T)) {
         e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
     } else {
         e = route_any(d, T, x, w_router, nullptr, idx, gate, st);

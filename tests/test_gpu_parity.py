@@ -198,12 +198,14 @@ def test_bad_arguments_with_real_tensors():
 
 @pytest.mark.parametrize("T,kernels", [
     (1, {"route_dispatch_small", "up_glu_stream", "down_combine_stream"}),
-    (3, {"route_dispatch_small", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
-    (9, {"route", "dispatch", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
+    (3, {"route_dispatch_cluster", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
+    (64, {"route_dispatch_cluster", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
+    (70, {"route", "dispatch", "gather_rows", "gemm_up_glu_tc", "gemm_down_tc", "combine"}),
 ])
 def test_launch_count_and_profile(T, kernels):
-    """One token: fused routing + the two streaming kernels; more tokens: the
-    tensor-core path.  Every launch is counted and event-timed."""
+    """One token: fused routing + the two streaming kernels; 2..64 tokens: the
+    cluster routing kernel and the tensor-core path; more: separate routing
+    and dispatch.  Every launch is counted and event-timed."""
     m = moe()
     L = _host((64, 64, 4, 2, T, "bf16"))
     d = _dims(m, L.shape)
