@@ -52,6 +52,10 @@ WORKLOADS = {
     # a 512-token prefill of the same 4-expert layer: the small case for
     # captures of the tensor-core GEMMs
     "dbrx4-prefill-t512": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 512),
+    # DBRX's router (D=6144, E=16, K=4) on 8 tokens with narrow experts
+    # (F=1024, 0.6 GB resident): the small case for captures of the cluster
+    # route+dispatch kernel, whose work does not depend on F
+    "dbrx-router-t8": (gen.LayerShape(6144, 1024, 16, 4, "bf16"), 8),
     # the tiny fp32 layer (D=256, F=512, E=4, K=2), 8 tokens: the reference
     # arm's smallest case (runs anywhere, no GPU needed)
     "tiny-decode-t8": (gen.TINY, 8),

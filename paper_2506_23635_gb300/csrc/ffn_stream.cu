@@ -21,7 +21,7 @@
 //     finish together.
 //
 // k_up_glu_stream:  h[j,f] = bf16( SiLU(W1[e,f,:] . x_j) * (V1[e,f,:] . x_j) )
-//   tasks = (chunk of <= 4 slots of one expert, row f), split evenly over CTAs.
+//   tasks = (chunk of <= NS slots of one expert, row f), split evenly over CTAs.
 // k_down_stream:    y[j,d] = W2[e,d,:] . h[j,:] for the CTA's rows d and every
 //   slot j, kept in shared memory; then either the gated combine
 //   out[t,d] = residual + sum_k gate[t,k] y[inv_perm[t*K+k], d]  (k ascending)
@@ -344,13 +344,14 @@ struct UpPlan { int ns, n_stages; size_t smem; };
 struct DownPlan { int ns, n_stages, rows_max; size_t smem; };
 
 // Slots per chunk: an expert holds at most T slots (a token picks distinct
-// experts), so small T needs a narrower token-vector buffer and leaves room
-// for more stages.
-int up_ns(int T) { return T >= 4 ? 4 : (T >= 2 ? 2 : 1); }
-int down_ns(int T) { return T >= 2 ? 2 : 1; }
+// experts), so a batch of at most kStreamMaxTokens tokens needs a token-vector
+// buffer of kStreamMaxTokens rows and leaves the rest of shared memory for
+// weight stages.
+constexpr int kNs = kStreamMaxTokens;
 
 bool plan_up(const moe_dims &d, int T, UpPlan &p) {
-    p.ns = up_ns(T);
+    (void)T;
+    p.ns = kNs;
     const size_t fixed = kHeaderBytes + (size_t)2 * p.ns * d.d_model * 2;
     const size_t stage = (size_t)2 * d.d_model * 2;
     if (fixed + 2 * stage > kSmemBudget) return false;
@@ -361,7 +362,7 @@ bool plan_up(const moe_dims &d, int T, UpPlan &p) {
 
 bool plan_down(const moe_dims &d, int T, int grid, DownPlan &p) {
     const int S = T * d.top_k;
-    p.ns = down_ns(T);
+    p.ns = kNs;
     p.rows_max = (d.d_model + grid - 1) / grid;
     const size_t fixed = kHeaderBytes + (size_t)2 * p.ns * d.ffn_hidden * 2 +
                          (((size_t)S * p.rows_max * 4 + 15) & ~size_t(15));
@@ -376,7 +377,7 @@ bool plan_down(const moe_dims &d, int T, int grid, DownPlan &p) {
 
 bool stream_path_ok(const moe_dims &d, int T) {
     if (d.w_dtype != MOE_BF16 || d.x_dtype != MOE_BF16) return false;
-    if (T < 1 || T * d.top_k > kStreamMaxSlots) return false;
+    if (T < 1 || T > kStreamMaxTokens || T * d.top_k > kStreamMaxSlots) return false;
     const int grid = device_info().sm_count;
     UpPlan up;
     DownPlan dn;
@@ -388,9 +389,7 @@ cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const 
                                  cudaStream_t st) {
     UpPlan p;
     if (!plan_up(d, T, p)) return cudaErrorInvalidValue;
-    const void *kern = p.ns == 4 ? (const void *)k_up_glu_stream<4>
-                     : p.ns == 2 ? (const void *)k_up_glu_stream<2>
-                                 : (const void *)k_up_glu_stream<1>;
+    const void *kern = (const void *)k_up_glu_stream<kNs>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return e;
@@ -413,8 +412,7 @@ cudaError_t down_stream_impl(const moe_dims &d, int T, const void *h, const int3
     const int grid = std::min(device_info().sm_count, d.d_model);
     DownPlan p;
     if (!plan_down(d, T, grid, p)) return cudaErrorInvalidValue;
-    const void *kern = p.ns == 2 ? (const void *)k_down_stream<2, TO, TR, FUSED>
-                                 : (const void *)k_down_stream<1, TO, TR, FUSED>;
+    const void *kern = (const void *)k_down_stream<kNs, TO, TR, FUSED>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)p.smem);
     if (e != cudaSuccess) return e;
