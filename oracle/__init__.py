@@ -57,6 +57,12 @@ def _bind(path: str) -> ctypes.CDLL:
     lib.orc_num_threads.restype = I
     lib.orc_rmsnorm0.argtypes = [I, I, P, ctypes.c_double, P]
     lib.orc_round_bf16.argtypes = [ctypes.c_size_t, P, P]
+    D_ = ctypes.c_double
+    lib.orc_rope.argtypes = [I, I, I, D_, P, P]
+    lib.orc_attention.argtypes = [I, I, I, I, I, I, P, P, P, P, P, P]
+    lib.orc_attention.restype = I
+    lib.orc_sa_forward.argtypes = [I, I, I, I, I, D_, D_, I, I, P, P, P, P, P, I, I, P, P]
+    lib.orc_sa_forward.restype = I
     return lib
 
 
@@ -208,6 +214,76 @@ class OracleLib:
             l += 1
         return x, np.array(gaps)
 
+    # ---- self-attention block of a decoder layer (readings in moe_oracle.c)
+
+    def rope(self, u64: np.ndarray, pos, base: float) -> np.ndarray:
+        """Rotary embedding of u [T, H, dh] (fp64) at positions pos [T]."""
+        u = _c(u64, np.float64).copy()
+        T, H, dh = u.shape
+        pos = _c(pos, np.int32)
+        self.lib.orc_rope(T, H, dh, base, _p(pos), _p(u))
+        return u
+
+    def attention(self, q64, k_cache64, v_cache64, seq, pos) -> np.ndarray:
+        """Causal grouped-query attention of q [T, Hq, dh] over the caches
+        [n_seq, Hkv, L, dh] (fp64 values); returns ctx [T, Hq, dh]."""
+        q = _c(q64, np.float64)
+        kc, vc = _c(k_cache64, np.float64), _c(v_cache64, np.float64)
+        T, Hq, dh = q.shape
+        n_seq, Hkv, L, _ = kc.shape
+        seq, pos = _c(seq, np.int32), _c(pos, np.int32)
+        ctx = np.empty_like(q)
+        if self.lib.orc_attention(T, Hq, Hkv, dh, n_seq, L, _p(seq), _p(pos), _p(q), _p(kc),
+                                  _p(vc), _p(ctx)) != 0:
+            raise ValueError("sequence or position out of range")
+        return ctx
+
+    def sa_forward(self, x64, w_qkv, w_o, dtype: str, n_heads: int, n_kv_heads: int,
+                   base: float, eps: float, seq, pos, k_cache64, v_cache64):
+        """The self-attention block on the residual stream x [T, D] (fp64):
+        returns (x + Wo ctx, k_cache, v_cache) with the new tokens' keys and
+        values written into copies of the caches [n_seq, Hkv, L, dh]."""
+        x = _c(x64, np.float64).copy()
+        kc, vc = _c(k_cache64, np.float64).copy(), _c(v_cache64, np.float64).copy()
+        T, D = x.shape
+        n_seq, Hkv, L, dh = kc.shape
+        assert Hkv == n_kv_heads
+        wq, wo = _storage(w_qkv, dtype), _storage(w_o, dtype)
+        seq, pos = _c(seq, np.int32), _c(pos, np.int32)
+        rc = self.lib.orc_sa_forward(T, D, n_heads, n_kv_heads, dh, base, eps, n_seq, L,
+                                     _p(seq), _p(pos), _p(x), _p(wq), _p(wo), _DT[dtype],
+                                     1 if dtype == "bf16" else 0, _p(kc), _p(vc))
+        if rc != 0:
+            raise ValueError("sequence or position out of range")
+        return x, kc, vc
+
+    def decoder_layers(self, x0_64, layers, dtype: str, n_heads: int, n_kv_heads: int,
+                       base: float, eps: float, top_k: int, seq, pos, caches):
+        """Decoder layers x <- x + SA(x); x <- x + MoE(RMSNorm0(x)), in order.
+        layers: sequence of (w_qkv, w_o, w_r, w1, v1, w2); caches: list of
+        (k_cache, v_cache) fp64 per layer.  Returns the residual stream after
+        the last layer and the updated caches."""
+        x = _c(x0_64, np.float64)
+        out_caches = []
+        for (w_qkv, w_o, w_r, w1, v1, w2), (kc, vc) in zip(layers, caches):
+            x, kc, vc = self.sa_forward(x, w_qkv, w_o, dtype, n_heads, n_kv_heads, base, eps,
+                                        seq, pos, kc, vc)
+            x = self.moe_block(x, (w_r, w1, v1, w2), dtype, top_k, eps)
+            out_caches.append((kc, vc))
+        return x, out_caches
+
+    def moe_block(self, x64, layer, dtype: str, top_k: int, eps: float) -> np.ndarray:
+        """x + MoE(RMSNorm0(x)) on the fp64 residual stream x [T, D], the
+        normalised input stored in bf16 when the weights are (reading C9)."""
+        x = _c(x64, np.float64)
+        xn = self.rmsnorm0(x, eps)
+        if dtype == "bf16":
+            xn = self.round_bf16(xn)
+        w_r, w1, v1, w2 = layer
+        out, _, _ = self.layer_tokens(xn, w_r, w1, v1, w2, dtype, top_k, residual=x,
+                                      x_dtype="f64")
+        return out
+
     def layer_dense_masked(self, x, w_r, w1, v1, w2, dtype: str,
                            top_k: int) -> np.ndarray:
         """Busy full loading (Sec. 4.2): all experts on all tokens, unselected
@@ -300,6 +376,26 @@ def rmsnorm0(*a, **k):
 
 def round_bf16(*a, **k):
     return default().round_bf16(*a, **k)
+
+
+def rope(*a, **k):
+    return default().rope(*a, **k)
+
+
+def attention(*a, **k):
+    return default().attention(*a, **k)
+
+
+def sa_forward(*a, **k):
+    return default().sa_forward(*a, **k)
+
+
+def decoder_layers(*a, **k):
+    return default().decoder_layers(*a, **k)
+
+
+def moe_block(*a, **k):
+    return default().moe_block(*a, **k)
 
 
 def _to_f64(a, dtype):

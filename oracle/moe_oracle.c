@@ -271,6 +271,142 @@ void orc_round_bf16(size_t n, const double *in, double *out)
     }
 }
 
+/* ---- self-attention block of a decoder layer ----------------------------
+ * Table 1 (note (b)) sizes the self-attention of a DBRX layer only by its
+ * parameters, D_qkv_hidden x D_embed + D_embed^2 (D_qkv_hidden = 8,192,
+ * D_embed = 6,144), and its FLOPs as twice that; Table 2 books it under
+ * "Misc." with the router and the weighted sum.  Everything else is a
+ * reading (the paper is silent):
+ *
+ *   Wqkv [(Hq + 2 Hkv) dh, D]: rows [0, Hq dh) project the queries, the next
+ *     Hkv dh rows the keys, the last Hkv dh rows the values; Wo [D, Hq dh];
+ *     no biases.  Grouped queries: head h reads key/value head h / (Hq/Hkv).
+ *     (48 query heads and 8 key/value heads of 128 give D_qkv_hidden = 8,192.)
+ *   Rotary position embedding of queries and keys: in every head, dims i and
+ *     i + dh/2 (i < dh/2) turn by the angle pos * base^(-2i/dh).
+ *   Causal softmax attention scaled by 1/sqrt(dh): a token at position p of
+ *     sequence s attends to cache positions 0..p of s; the keys and values of
+ *     all tokens of a call are written to the cache before any token attends.
+ *   Block: resid += Wo . ctx, with ctx the attention of RMSNorm0(resid).
+ *     With bf16 storage the normalised input, the cached keys and values and
+ *     ctx are rounded to bf16: each is stored and read back by the next step.
+ *
+ * Cache layout: [n_seq, Hkv, L, dh] (keys and values alike), as doubles
+ * holding exactly the stored values. */
+
+/* u [T, H, dh]: row (t, h) turned by position pos[t]. */
+void orc_rope(int T, int H, int dh, double base, const int32_t *pos, double *u)
+{
+    const int half = dh / 2;
+    for (int t = 0; t < T; ++t)
+        for (int h = 0; h < H; ++h) {
+            double *r = u + ((size_t)t * H + h) * dh;
+            for (int i = 0; i < half; ++i) {
+                const double ang = (double)pos[t] * pow(base, -2.0 * i / dh);
+                const double c = cos(ang), s = sin(ang);
+                const double a = r[i], b = r[i + half];
+                r[i] = a * c - b * s;
+                r[i + half] = b * c + a * s;
+            }
+        }
+}
+
+/* ctx[t, h, :] = sum_j softmax_j(q[t,h,:] . K[s,g,j,:] / sqrt(dh)) V[s,g,j,:]
+ * over j = 0..pos[t], s = seq[t], g = h / (Hq/Hkv).  Returns -1 (nothing
+ * written) if a sequence or position is out of range. */
+int orc_attention(int T, int Hq, int Hkv, int dh, int n_seq, int L, const int32_t *seq,
+                  const int32_t *pos, const double *q, const double *kc, const double *vc,
+                  double *ctx)
+{
+    for (int t = 0; t < T; ++t)
+        if (seq[t] < 0 || seq[t] >= n_seq || pos[t] < 0 || pos[t] >= L) return -1;
+    const int group = Hq / Hkv;
+    const double scale = 1.0 / sqrt((double)dh);
+    #pragma omp parallel for schedule(dynamic)
+    for (int th = 0; th < T * Hq; ++th) {
+        const int t = th / Hq, h = th % Hq, g = h / group, n = pos[t] + 1;
+        const double *qr = q + (size_t)th * dh;
+        const double *kb = kc + ((size_t)seq[t] * Hkv + g) * L * dh;
+        const double *vb = vc + ((size_t)seq[t] * Hkv + g) * L * dh;
+        double *sc = malloc(sizeof(double) * (size_t)n);
+        double m = -INFINITY;
+        for (int j = 0; j < n; ++j) {
+            double dot = 0.0;
+            for (int i = 0; i < dh; ++i) dot += qr[i] * kb[(size_t)j * dh + i];
+            sc[j] = dot * scale;
+            if (sc[j] > m) m = sc[j];
+        }
+        double z = 0.0;
+        for (int j = 0; j < n; ++j) {
+            sc[j] = exp(sc[j] - m);
+            z += sc[j];
+        }
+        double *o = ctx + (size_t)th * dh;
+        for (int i = 0; i < dh; ++i) o[i] = 0.0;
+        for (int j = 0; j < n; ++j)
+            for (int i = 0; i < dh; ++i) o[i] += sc[j] / z * vb[(size_t)j * dh + i];
+        free(sc);
+    }
+    return 0;
+}
+
+/* The whole block for T tokens: x [T, D] is the residual stream (in/out),
+ * caches as above (updated), round = 1 for bf16 storage.  Returns -1 on a
+ * bad sequence or position (nothing written). */
+int orc_sa_forward(int T, int D, int Hq, int Hkv, int dh, double base, double eps, int n_seq,
+                   int L, const int32_t *seq, const int32_t *pos, double *x, const void *wqkv,
+                   const void *wo, int wdt, int round, double *kc, double *vc)
+{
+    for (int t = 0; t < T; ++t)
+        if (seq[t] < 0 || seq[t] >= n_seq || pos[t] < 0 || pos[t] >= L) return -1;
+    const int nq = Hq * dh, nkv = Hkv * dh, nr = nq + 2 * nkv;
+    double *xn = malloc(sizeof(double) * (size_t)T * D);
+    double *qkv = malloc(sizeof(double) * (size_t)T * nr);
+    double *q = malloc(sizeof(double) * (size_t)T * nq);
+    double *k = malloc(sizeof(double) * (size_t)T * nkv);
+    double *v = malloc(sizeof(double) * (size_t)T * nkv);
+    double *ctx = malloc(sizeof(double) * (size_t)T * nq);
+    orc_rmsnorm0(T, D, x, eps, xn);
+    if (round) orc_round_bf16((size_t)T * D, xn, xn);
+    #pragma omp parallel for schedule(static)
+    for (int r = 0; r < nr; ++r)
+        for (int t = 0; t < T; ++t) {
+            double acc = 0.0;
+            for (int d = 0; d < D; ++d)
+                acc += xn[(size_t)t * D + d] * orc_load(wqkv, wdt, (size_t)r * D + d);
+            qkv[(size_t)t * nr + r] = acc;
+        }
+    for (int t = 0; t < T; ++t) {
+        memcpy(q + (size_t)t * nq, qkv + (size_t)t * nr, sizeof(double) * nq);
+        memcpy(k + (size_t)t * nkv, qkv + (size_t)t * nr + nq, sizeof(double) * nkv);
+        memcpy(v + (size_t)t * nkv, qkv + (size_t)t * nr + nq + nkv, sizeof(double) * nkv);
+    }
+    orc_rope(T, Hq, dh, base, pos, q);
+    orc_rope(T, Hkv, dh, base, pos, k);
+    if (round) {
+        orc_round_bf16((size_t)T * nkv, k, k);
+        orc_round_bf16((size_t)T * nkv, v, v);
+    }
+    for (int t = 0; t < T; ++t)
+        for (int g = 0; g < Hkv; ++g) {
+            const size_t at = (((size_t)seq[t] * Hkv + g) * L + pos[t]) * dh;
+            memcpy(kc + at, k + ((size_t)t * Hkv + g) * dh, sizeof(double) * dh);
+            memcpy(vc + at, v + ((size_t)t * Hkv + g) * dh, sizeof(double) * dh);
+        }
+    orc_attention(T, Hq, Hkv, dh, n_seq, L, seq, pos, q, kc, vc, ctx);
+    if (round) orc_round_bf16((size_t)T * nq, ctx, ctx);
+    #pragma omp parallel for schedule(static)
+    for (int d = 0; d < D; ++d)
+        for (int t = 0; t < T; ++t) {
+            double acc = 0.0;
+            for (int c = 0; c < nq; ++c)
+                acc += ctx[(size_t)t * nq + c] * orc_load(wo, wdt, (size_t)d * nq + c);
+            x[(size_t)t * D + d] += acc;
+        }
+    free(xn); free(qkv); free(q); free(k); free(v); free(ctx);
+    return 0;
+}
+
 /* Number of OpenMP threads the parallel loops above use (1 without OpenMP). */
 int orc_num_threads(void)
 {

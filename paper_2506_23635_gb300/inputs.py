@@ -299,3 +299,79 @@ def device_expert_weights(shape: LayerShape, seed: int, device, layer: int = 0):
         device_normal_(v1[e], W_STD, seed, "dev-v1", layer, e)
         device_normal_(w2[e], W_STD, seed, "dev-w2", layer, e)
     return w1, v1, w2
+
+
+# --------------------------------------------------------------------------
+# self-attention block of a decoder layer
+# --------------------------------------------------------------------------
+
+
+@dataclasses.dataclass(frozen=True)
+class AttnShape:
+    """Grouped-query self-attention: n_heads query heads share n_kv_heads
+    key/value heads of head_dim; (n_heads + 2 n_kv_heads) * head_dim is the
+    width of the fused query/key/value projection (Table 1's D_qkv_hidden)."""
+    d_model: int
+    n_heads: int
+    n_kv_heads: int
+    head_dim: int
+    rope_base: float = 500000.0
+    dtype: str = "bf16"
+
+    @property
+    def qkv_rows(self) -> int:
+        return (self.n_heads + 2 * self.n_kv_heads) * self.head_dim
+
+    @property
+    def ctx_width(self) -> int:
+        return self.n_heads * self.head_dim
+
+
+# 48 query heads and 8 key/value heads of 128: D_qkv_hidden = 8,192 (Table 1)
+DBRX_ATTN = AttnShape(6144, 48, 8, 128)
+
+
+def cache_std(shape: AttnShape) -> float:
+    """Standard deviation of a projected key or value for unit-RMS input and
+    N(0, W_STD^2) weights: the scale of the synthetic earlier cache entries."""
+    return W_STD * float(np.sqrt(shape.d_model))
+
+
+def host_attn_weights(shape: AttnShape, seed: int, layer: int = 0):
+    """w_qkv [(Hq + 2 Hkv) dh, D] and w_o [D, Hq dh], N(0, W_STD^2)."""
+    w_qkv = host_normal((shape.qkv_rows, shape.d_model), W_STD, shape.dtype, seed, "wqkv", layer)
+    w_o = host_normal((shape.d_model, shape.ctx_width), W_STD, shape.dtype, seed, "wo", layer)
+    return w_qkv, w_o
+
+
+def host_kv_cache(shape: AttnShape, n_seq: int, max_len: int, seed: int, layer: int = 0):
+    """Key and value caches [n_seq, Hkv, max_len, dh] filled with synthetic
+    earlier entries (normal, at the scale a projection produces)."""
+    dims = (n_seq, shape.n_kv_heads, max_len, shape.head_dim)
+    k = host_normal(dims, cache_std(shape), shape.dtype, seed, "kcache", layer)
+    v = host_normal(dims, cache_std(shape), shape.dtype, seed, "vcache", layer)
+    return k, v
+
+
+def device_attn_weights(shape: AttnShape, seed: int, device, layer: int = 0):
+    import torch
+
+    tdt = torch_dtype(shape.dtype)
+    w_qkv = torch.empty((shape.qkv_rows, shape.d_model), dtype=tdt, device=device)
+    w_o = torch.empty((shape.d_model, shape.ctx_width), dtype=tdt, device=device)
+    device_normal_(w_qkv, W_STD, seed, "dev-wqkv", layer)
+    device_normal_(w_o, W_STD, seed, "dev-wo", layer)
+    return w_qkv, w_o
+
+
+def device_kv_cache(shape: AttnShape, n_seq: int, max_len: int, seed: int, device,
+                    layer: int = 0):
+    import torch
+
+    tdt = torch_dtype(shape.dtype)
+    dims = (n_seq, shape.n_kv_heads, max_len, shape.head_dim)
+    k = torch.empty(dims, dtype=tdt, device=device)
+    v = torch.empty(dims, dtype=tdt, device=device)
+    device_normal_(k, cache_std(shape), seed, "dev-kcache", layer)
+    device_normal_(v, cache_std(shape), seed, "dev-vcache", layer)
+    return k, v

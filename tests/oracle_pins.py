@@ -375,4 +375,181 @@ def pin_stack_residual_composition(orc):
     _close(two, one + moe, 1e-13, 1e-13, msg="residual composition")
 
 
+# --------------------------------------------------------------------------
+# self-attention block of a decoder layer (readings in moe_oracle.c)
+# --------------------------------------------------------------------------
+
+
+def _rope_generator(dh, base):
+    """Skew-symmetric generator of the rotary embedding: the plane of dims
+    (i, i + dh/2) turns at angular rate base^(-2i/dh)."""
+    G = np.zeros((dh, dh))
+    h = dh // 2
+    for i in range(h):
+        w = base ** (-2.0 * i / dh)
+        G[i + h, i] = w
+        G[i, i + h] = -w
+    return G
+
+
+def pin_rope_matrix_exponential(orc):
+    """rope(u, p) = expm(p G) u for the generator G (scipy's matrix
+    exponential, not the oracle's cos/sin); position 0 is the identity and
+    every head keeps its norm."""
+    from scipy.linalg import expm
+    rng = np.random.default_rng(41)
+    for dh, base in ((8, 10000.0), (16, 500000.0), (2, 7.0)):
+        u = rng.normal(size=(4, 3, dh))
+        pos = np.array([0, 1, 17, 250], np.int32)
+        got = orc.rope(u, pos, base)
+        G = _rope_generator(dh, base)
+        for t in range(4):
+            R = expm(pos[t] * G)
+            _close(got[t], u[t] @ R.T, 1e-10, 1e-12, f"rope dh={dh} pos={pos[t]}")
+        assert np.array_equal(got[0], u[0]), "rope at position 0"
+        _close(np.linalg.norm(got, axis=-1), np.linalg.norm(u, axis=-1), 1e-12, 0, "rope norm")
+
+
+def _sdpa(q, k, v, causal):
+    """torch's scaled_dot_product_attention in fp64 on the CPU; q [Hq, n, dh],
+    k, v [Hkv, m, dh]; grouped queries by repeating each key/value head."""
+    import torch
+    g = q.shape[0] // k.shape[0]
+    tq = torch.from_numpy(q)[None]
+    tk = torch.from_numpy(k).repeat_interleave(g, dim=0)[None]
+    tv = torch.from_numpy(v).repeat_interleave(g, dim=0)[None]
+    out = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, is_causal=causal)
+    return out[0].numpy()
+
+
+def pin_attention_against_sdpa(orc):
+    """Prefill of one sequence (positions 0..n-1, causal) and decode tokens of
+    several sequences at scattered positions, against torch's attention."""
+    rng = np.random.default_rng(43)
+    Hq, Hkv, dh, L = 6, 2, 16, 40
+    # prefill: tokens 0..n-1 of sequence 1
+    n = 23
+    kc = rng.normal(size=(3, Hkv, L, dh))
+    vc = rng.normal(size=(3, Hkv, L, dh))
+    q = rng.normal(size=(n, Hq, dh)) * 2.0
+    seq = np.full(n, 1, np.int32)
+    pos = np.arange(n, dtype=np.int32)
+    got = orc.attention(q, kc, vc, seq, pos)
+    want = _sdpa(q.transpose(1, 0, 2), kc[1, :, :n], vc[1, :, :n], True).transpose(1, 0, 2)
+    _close(got, want, 1e-10, 1e-12, "attention prefill vs sdpa")
+    # decode: one token per sequence, each at its own position
+    seq = np.array([2, 0, 1], np.int32)
+    pos = np.array([39, 0, 11], np.int32)
+    q = rng.normal(size=(3, Hq, dh)) * 2.0
+    got = orc.attention(q, kc, vc, seq, pos)
+    for t in range(3):
+        s, p = seq[t], pos[t]
+        want = _sdpa(q[t][:, None, :], kc[s, :, :p + 1], vc[s, :, :p + 1], False)[:, 0, :]
+        _close(got[t], want, 1e-10, 1e-12, f"attention decode token {t}")
+    assert np.array_equal(got[1], np.repeat(vc[0, :, 0], Hq // Hkv, axis=0)), \
+        "one cached position: ctx is that value row, for every head of the group"
+
+
+def _sa_case(rng, D=24, Hq=4, Hkv=2, dh=8, n_seq=2, L=12, dt="f32"):
+    nr = (Hq + 2 * Hkv) * dh
+    w_qkv = gen.store(rng.normal(size=(nr, D)) * 0.2, dt)
+    w_o = gen.store(rng.normal(size=(D, Hq * dh)) * 0.2, dt)
+    kc = gen.to_f64(gen.store(rng.normal(size=(n_seq, Hkv, L, dh)), dt), dt)
+    vc = gen.to_f64(gen.store(rng.normal(size=(n_seq, Hkv, L, dh)), dt), dt)
+    return w_qkv, w_o, kc, vc
+
+
+def pin_sa_block_composition(orc):
+    """The block is rmsnorm0 -> projection (numpy matmul) -> rotary (matrix
+    exponential) -> cache write -> torch attention -> output projection ->
+    residual add; D differs from Hq*dh so an operand read the wrong way
+    round cannot fit."""
+    from scipy.linalg import expm
+    rng = np.random.default_rng(47)
+    D, Hq, Hkv, dh, base, eps = 24, 4, 2, 8, 1000.0, 1e-6
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh)
+    x = rng.normal(size=(5, D)) * 3.0
+    seq = np.array([0, 0, 0, 1, 1], np.int32)
+    pos = np.array([4, 5, 6, 0, 1], np.int32)
+    got, gk, gv = orc.sa_forward(x, w_qkv, w_o, "f32", Hq, Hkv, base, eps, seq, pos, kc, vc)
+    xn = x / np.sqrt(np.mean(x * x, axis=1, keepdims=True) + eps)
+    qkv = xn @ gen.to_f64(w_qkv, "f32").T
+    q = qkv[:, :Hq * dh].reshape(5, Hq, dh)
+    k = qkv[:, Hq * dh:(Hq + Hkv) * dh].reshape(5, Hkv, dh)
+    v = qkv[:, (Hq + Hkv) * dh:].reshape(5, Hkv, dh)
+    G = _rope_generator(dh, base)
+    R = [expm(p * G) for p in pos]
+    q = np.stack([q[t] @ R[t].T for t in range(5)])
+    k = np.stack([k[t] @ R[t].T for t in range(5)])
+    wk, wv = kc.copy(), vc.copy()
+    for t in range(5):
+        wk[seq[t], :, pos[t]] = k[t]
+        wv[seq[t], :, pos[t]] = v[t]
+    _close(gk, wk, 1e-10, 1e-12, "cached keys")
+    _close(gv, wv, 1e-10, 1e-12, "cached values")
+    ctx = np.stack([_sdpa(q[t][:, None, :], wk[seq[t], :, :pos[t] + 1],
+                          wv[seq[t], :, :pos[t] + 1], False)[:, 0, :] for t in range(5)])
+    want = x + ctx.reshape(5, Hq * dh) @ gen.to_f64(w_o, "f32").T
+    _close(got, want, 1e-9, 1e-11, "self-attention block")
+
+
+def pin_sa_incremental_equals_prefill(orc):
+    """Prefilling a sequence in one call equals feeding its tokens one per
+    call (the cache carries the earlier keys and values); a second sequence
+    in the same call does not disturb the first."""
+    rng = np.random.default_rng(53)
+    D, Hq, Hkv, dh, base, eps = 24, 4, 2, 8, 1000.0, 1e-6
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh)
+    n = 6
+    x = rng.normal(size=(n, D))
+    seq = np.zeros(n, np.int32)
+    pos = np.arange(n, dtype=np.int32)
+    full, fk, fv = orc.sa_forward(x, w_qkv, w_o, "f32", Hq, Hkv, base, eps, seq, pos, kc, vc)
+    k1, v1 = kc, vc
+    for t in range(n):
+        o, k1, v1 = orc.sa_forward(x[t:t + 1], w_qkv, w_o, "f32", Hq, Hkv, base, eps,
+                                   seq[t:t + 1], pos[t:t + 1], k1, v1)
+        _close(o[0], full[t], 1e-10, 1e-12, f"incremental token {t}")
+    _close(k1, fk, 0, 1e-14, "incremental caches")
+    x2 = rng.normal(size=(1, D))
+    both, _, _ = orc.sa_forward(np.vstack([x, x2]), w_qkv, w_o, "f32", Hq, Hkv, base, eps,
+                                np.append(seq, 1).astype(np.int32),
+                                np.append(pos, 3).astype(np.int32), kc, vc)
+    _close(both[:n], full, 1e-10, 1e-12, "another sequence in the same call")
+
+
+def pin_sa_causality(orc):
+    """Changing a later token of a prefill leaves every earlier token's
+    output unchanged and changes the later one."""
+    rng = np.random.default_rng(59)
+    D, Hq, Hkv, dh = 24, 4, 2, 8
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh)
+    n = 5
+    x = rng.normal(size=(n, D))
+    seq = np.zeros(n, np.int32)
+    pos = np.arange(n, dtype=np.int32)
+    a, _, _ = orc.sa_forward(x, w_qkv, w_o, "f32", Hq, Hkv, 1000.0, 1e-6, seq, pos, kc, vc)
+    x[3] += 1.0
+    b, _, _ = orc.sa_forward(x, w_qkv, w_o, "f32", Hq, Hkv, 1000.0, 1e-6, seq, pos, kc, vc)
+    assert np.array_equal(a[:3], b[:3]), "earlier tokens saw a later one"
+    assert not np.allclose(a[3:], b[3:]), "later tokens did not change"
+
+
+def pin_sa_bf16_storage(orc):
+    """With bf16 storage the cached keys and values are bf16 values (the
+    rounding of the f32-storage result); a zero output projection leaves
+    the residual unchanged."""
+    rng = np.random.default_rng(61)
+    D, Hq, Hkv, dh = 24, 4, 2, 8
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh, dt="bf16")
+    x = rng.normal(size=(3, D))
+    seq = np.array([0, 1, 1], np.int32)
+    pos = np.array([2, 7, 8], np.int32)
+    zero_o = gen.store(np.zeros((D, Hq * dh)), "bf16")
+    out, k, v = orc.sa_forward(x, w_qkv, zero_o, "bf16", Hq, Hkv, 1000.0, 1e-6, seq, pos, kc, vc)
+    assert np.array_equal(out, x), "zero output projection"
+    for c in (k, v):
+        assert np.array_equal(gen.to_f64(gen.store(c, "bf16"), "bf16"), c), "cache not bf16"
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

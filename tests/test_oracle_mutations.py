@@ -42,6 +42,19 @@ MUTATIONS = [
      "const double s = 1.0 / (ss / D + eps);"),
     ("rmsnorm_sum_not_mean", "const double s = 1.0 / sqrt(ss / D + eps);",
      "const double s = 1.0 / sqrt(ss + eps);"),
+    ("rope_turns_backwards", "r[i] = a * c - b * s;\n                r[i + half] = b * c + a * s;",
+     "r[i] = a * c + b * s;\n                r[i + half] = b * c - a * s;"),
+    ("rope_frequency", "pow(base, -2.0 * i / dh)", "pow(base, -1.0 * i / dh)"),
+    ("rope_adjacent_pairs", "const double a = r[i], b = r[i + half];",
+     "const double a = r[2 * (i % (half / 2 + 1))], b = r[i + half];"),
+    ("attention_unscaled", "sc[j] = dot * scale;", "sc[j] = dot;"),
+    ("attention_misses_own_position", "n = pos[t] + 1;", "n = pos[t] + (pos[t] == 0);"),
+    ("gqa_interleaved", "g = h / group,", "g = h % Hkv,"),
+    ("wo_transposed", "orc_load(wo, wdt, (size_t)d * nq + c)", "orc_load(wo, wdt, (size_t)c * D + d)"),
+    ("keys_not_rotated", "    orc_rope(T, Hkv, dh, base, pos, k);\n", "\n"),
+    ("values_from_keys", "qkv + (size_t)t * nr + nq + nkv, sizeof(double) * nkv);",
+     "qkv + (size_t)t * nr + nq, sizeof(double) * nkv);"),
+    ("cache_not_rounded", "        orc_round_bf16((size_t)T * nkv, v, v);\n", "\n"),
 ]
 
 
