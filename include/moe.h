@@ -65,7 +65,9 @@ typedef enum {
     MOE_ERR_WORKSPACE = 3,    /* workspace missing or too small */
     MOE_ERR_CUDA = 4,         /* a CUDA call or kernel launch failed */
     MOE_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up */
-    MOE_ERR_DEVICE_INDEX = 6  /* a kernel met an expert index outside [0,E) */
+    MOE_ERR_DEVICE_INDEX = 6  /* a kernel met an index outside its range: an expert
+                                 outside [0,E), or a cache sequence / position
+                                 outside the cache (moe_sa_*) */
 } moe_status;
 
 typedef enum { MOE_F32 = 0, MOE_BF16 = 1 } moe_dtype;
@@ -244,8 +246,8 @@ moe_status moe_get_last_error(moe_stream_t stream);
  * Host-side fault injection: with MOE_INJECT_FAILURE="<entry>:<status>" in
  * the environment, the named entry point (moe_route, moe_dispatch,
  * moe_expert_ffn, moe_combine, moe_layer_forward, moe_layer_forward_dense,
- * moe_prenorm, moe_stack_forward) returns that status at once without
- * launching. */
+ * moe_prenorm, moe_stack_forward, moe_sa_qkv, moe_sa_attend, moe_sa_forward,
+ * moe_decoder_forward) returns that status at once without launching. */
 moe_status moe_selftest_wait_timeout(uint64_t limit_ns, int32_t *gave_up,
                                      moe_stream_t stream);
 
@@ -265,6 +267,94 @@ int64_t moe_launch_count(void);
 void moe_profile_enable(int on);
 void moe_profile_reset(void);
 int32_t moe_profile_read(moe_kernel_stat *stats, int32_t max_stats);
+
+/* ---- self-attention block and whole decoder layers ---------------------
+ * Table 1 (note (b)) sizes a DBRX layer's self-attention only by its
+ * parameters, D_qkv_hidden x D_embed + D_embed^2 with D_qkv_hidden = 8,192,
+ * and Table 2 books its time under "Misc." beside the router and the
+ * weighted sum.  The paper prints nothing else about it; this library reads
+ * it as the standard DBRX block:
+ *   - grouped-query attention: n_heads query heads share n_kv_heads
+ *     key/value heads of head_dim (48 + 2 x 8 heads of 128 give 8,192);
+ *     query head h reads key/value head h / (n_heads / n_kv_heads);
+ *   - rotary position embedding of queries and keys: in every head, dims i
+ *     and i + head_dim/2 turn by the angle pos * rope_base^(-2i/head_dim);
+ *   - causal softmax attention scaled by 1/sqrt(head_dim); no biases;
+ *   - the pre-norm residual block  resid += w_o . Attn(RMSNorm0(resid)),
+ *     RMSNorm0 as in moe_prenorm (no learned scale).
+ * Storage: the normalised input, the cached keys and values and the
+ * attention output ctx are bf16; projections accumulate in fp32; the
+ * residual stream is fp32.
+ *
+ * Layouts (row-major): w_qkv [(Hq + 2 Hkv) dh, D] bf16 -- the query rows,
+ * then the key rows, then the value rows; w_o [D, Hq dh] bf16; k_cache and
+ * v_cache [n_seq, Hkv, max_len, dh] bf16, owned by the caller; q [T, Hq, dh]
+ * fp32; ctx [T, Hq dh] bf16; resid [T, D] fp32.
+ *
+ * Tokens: token t is position pos[t] of sequence seq[t] (device int32
+ * arrays of T entries).  A call first writes every new token's key and value
+ * at (seq[t], pos[t]) and then lets each token attend to positions
+ * 0..pos[t] of its sequence: a prefill passes consecutive positions of one
+ * sequence, a decode step one token per sequence.  The caller keeps the
+ * (seq, pos) pairs of a call distinct and the positions below pos[t]
+ * filled by earlier calls.  A token whose seq or pos lies outside the cache
+ * is recorded as MOE_ERR_DEVICE_INDEX, writes nothing to the cache and gets a
+ * zero ctx.
+ *
+ * Limits: head_dim == 128; n_kv_heads divides n_heads and n_heads /
+ * n_kv_heads <= 8; d_model a multiple of 8 in [8, 49152];
+ * (n_heads + 2 n_kv_heads) * 128 <= 49152; n_seq >= 1, max_len >= 1;
+ * rope_base > 1; T <= 65536.  bf16 only. */
+typedef struct {
+    int32_t d_model;     /* D */
+    int32_t n_heads;     /* Hq: query heads */
+    int32_t n_kv_heads;  /* Hkv: key/value heads */
+    int32_t head_dim;    /* dh */
+    float rope_base;     /* rotary base (DBRX: 500000) */
+} moe_sa_dims;
+
+/* moe_sa_workspace_size: bytes of scratch the moe_sa_* calls need for up to
+ * max_tokens tokens. */
+moe_status moe_sa_workspace_size(const moe_sa_dims *dims, int32_t max_tokens, size_t *bytes);
+
+/* moe_sa_qkv: from the normalised input x_norm [T, D] (bf16): q = the
+ * rotated queries (fp32 out), and the rotated keys and the values of the T
+ * tokens written into k_cache / v_cache at (seq[t], pos[t]). */
+moe_status moe_sa_qkv(const moe_sa_dims *dims, int32_t T, const void *x_norm,
+                      const void *w_qkv, const int32_t *seq, const int32_t *pos,
+                      int32_t n_seq, int32_t max_len, float *q, void *k_cache,
+                      void *v_cache, void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/* moe_sa_attend: ctx[t, h dh .. (h+1) dh) = softmax over positions
+ * 0..pos[t] of q[t,h] . K / sqrt(dh), applied to V (bf16 out). */
+moe_status moe_sa_attend(const moe_sa_dims *dims, int32_t T, const float *q,
+                         const int32_t *seq, const int32_t *pos, int32_t n_seq,
+                         int32_t max_len, const void *k_cache, const void *v_cache,
+                         void *ctx, void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/* moe_sa_forward: the whole block in place on resid:
+ * resid += w_o . Attn(RMSNorm0(resid)), caches updated as in moe_sa_qkv. */
+moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq,
+                          const int32_t *pos, int32_t n_seq, int32_t max_len, float *resid,
+                          const void *w_qkv, const void *w_o, void *k_cache, void *v_cache,
+                          float eps, void *ws, size_t ws_bytes, moe_stream_t stream);
+
+/* moe_decoder_workspace_size / moe_decoder_forward: n_layers decoder layers
+ * in order, each  resid += w_o . Attn(RMSNorm0(resid));
+ *                 resid += MoE(RMSNorm0(resid))  (as moe_stack_forward).
+ * attn->d_model == moe->d_model; moe: bf16 weights and input, out_dtype F32
+ * (the fp32 residual stream).  Per-layer tensors come as HOST arrays of
+ * n_layers DEVICE pointers. */
+moe_status moe_decoder_workspace_size(const moe_sa_dims *attn, const moe_dims *moe,
+                                      int32_t max_tokens, size_t *bytes);
+moe_status moe_decoder_forward(const moe_sa_dims *attn, const moe_dims *moe, int32_t n_layers,
+                               int32_t T, const int32_t *seq, const int32_t *pos,
+                               int32_t n_seq, int32_t max_len, float *resid,
+                               const void *const *w_qkv, const void *const *w_o,
+                               const void *const *w_router, const void *const *w1,
+                               const void *const *v1, const void *const *w2,
+                               void *const *k_cache, void *const *v_cache, float eps,
+                               void *ws, size_t ws_bytes, moe_stream_t stream);
 
 #ifdef __cplusplus
 }

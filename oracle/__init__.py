@@ -262,19 +262,23 @@ class OracleLib:
         """Decoder layers x <- x + SA(x); x <- x + MoE(RMSNorm0(x)), in order.
         layers: sequence of (w_qkv, w_o, w_r, w1, v1, w2); caches: list of
         (k_cache, v_cache) fp64 per layer.  Returns the residual stream after
-        the last layer and the updated caches."""
+        the last layer, the updated caches and the routing gaps [n_layers, T]
+        (as ``stack_tokens``)."""
         x = _c(x0_64, np.float64)
-        out_caches = []
+        out_caches, gaps = [], []
         for (w_qkv, w_o, w_r, w1, v1, w2), (kc, vc) in zip(layers, caches):
             x, kc, vc = self.sa_forward(x, w_qkv, w_o, dtype, n_heads, n_kv_heads, base, eps,
                                         seq, pos, kc, vc)
-            x = self.moe_block(x, (w_r, w1, v1, w2), dtype, top_k, eps)
+            x, g = self.moe_block(x, (w_r, w1, v1, w2), dtype, top_k, eps)
             out_caches.append((kc, vc))
-        return x, out_caches
+            gaps.append(g)
+        return x, out_caches, np.array(gaps)
 
-    def moe_block(self, x64, layer, dtype: str, top_k: int, eps: float) -> np.ndarray:
+    def moe_block(self, x64, layer, dtype: str, top_k: int, eps: float):
         """x + MoE(RMSNorm0(x)) on the fp64 residual stream x [T, D], the
-        normalised input stored in bf16 when the weights are (reading C9)."""
+        normalised input stored in bf16 when the weights are (reading C9).
+        Returns the new stream and each token's routing gap (K-th minus
+        (K+1)-th logit over the logit RMS; +inf when K = E)."""
         x = _c(x64, np.float64)
         xn = self.rmsnorm0(x, eps)
         if dtype == "bf16":
@@ -282,7 +286,12 @@ class OracleLib:
         w_r, w1, v1, w2 = layer
         out, _, _ = self.layer_tokens(xn, w_r, w1, v1, w2, dtype, top_k, residual=x,
                                       x_dtype="f64")
-        return out
+        logits = self.router_logits(xn, w_r, dtype, x_dtype="f64")
+        if top_k >= logits.shape[1]:
+            return out, np.full(logits.shape[0], np.inf)
+        srt = -np.sort(-logits, axis=1)
+        rms = np.sqrt(np.mean(logits * logits, axis=1))
+        return out, (srt[:, top_k - 1] - srt[:, top_k]) / rms
 
     def layer_dense_masked(self, x, w_r, w1, v1, w2, dtype: str,
                            top_k: int) -> np.ndarray:

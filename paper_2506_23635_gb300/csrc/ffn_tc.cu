@@ -423,7 +423,7 @@ bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, ui
 template <int MODE, class C>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUtensorMap &b1,
                         const int32_t *offsets, int E, int S, int Kdim, int Nw, uint32_t a_bytes,
-                        bf16 *h_out, float *y_out, cudaStream_t st) {
+                        bf16 *h_out, float *y_out, cudaStream_t st, const char *name = nullptr) {
     const void *kern = (const void *)k_gemm_tc<MODE, C>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
@@ -432,7 +432,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUten
     CUtensorMap ma = a, mb0 = b0, mb1 = b1;
     void *args[] = {&ma, &mb0, &mb1, &offsets, &E, &S, &Kdim, &Nw, &a_bytes, &h_out, &y_out,
                     &err};
-    LaunchScope ls(MODE == kUp ? "gemm_up_glu_tc" : "gemm_down_tc", st);
+    LaunchScope ls(name ? name : MODE == kUp ? "gemm_up_glu_tc" : "gemm_down_tc", st);
     return launch_pdl(kern, dim3(device_info().sm_count), dim3(kThreadsTc), C::kSmem, st, args);
 }
 
@@ -486,7 +486,8 @@ cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, co
 }
 
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
-                                const void *w2, float *y_sorted, cudaStream_t st) {
+                                const void *w2, float *y_sorted, cudaStream_t st,
+                                const char *name) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
     const uint32_t arows = a_box_rows(T);
     CUtensorMap a, b0;
@@ -494,7 +495,7 @@ cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const i
         !make_map(&b0, w2, (uint64_t)E * D, (uint64_t)F, DownWide::BN))
         return cudaErrorInvalidValue;
     return launch_gemm<kDown, DownWide>(a, b0, b0, offsets, E, S, F, D, arows * BK * 2, nullptr,
-                                        y_sorted, st);
+                                        y_sorted, st, name);
 }
 
 }  // namespace moe

@@ -769,6 +769,15 @@ LaunchScope::~LaunchScope() {
     P.pending.push_back({kind_of(P, name), P.begin_of_slot[slot], b});
 }
 
+moe_status injected_failure(const char *entry) {
+    const char *v = getenv("MOE_INJECT_FAILURE");
+    if (!v) return MOE_OK;
+    const size_t n = strlen(entry);
+    if (strncmp(v, entry, n) != 0 || v[n] != ':') return MOE_OK;
+    const int code = atoi(v + n + 1);
+    return (code > 0 && code <= MOE_ERR_DEVICE_INDEX) ? (moe_status)code : MOE_OK;
+}
+
 WsLayout ws_layout(const moe_dims &d, int64_t T) {
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
     const size_t S = (size_t)T * d.top_k;
@@ -800,24 +809,6 @@ namespace {
 
 bool dt_ok(int32_t v) { return v == MOE_F32 || v == MOE_BF16; }
 
-// Host-side fault injection for callers' error paths: MOE_INJECT_FAILURE
-// "<entry point>:<status>" makes that entry return the status at once,
-// before anything is validated or launched.  Read on every call (tests set
-// it per process); nothing is injected when it is unset.
-moe_status injected(const char *entry) {
-    const char *v = getenv("MOE_INJECT_FAILURE");
-    if (!v) return MOE_OK;
-    const size_t n = strlen(entry);
-    if (strncmp(v, entry, n) != 0 || v[n] != ':') return MOE_OK;
-    const int code = atoi(v + n + 1);
-    return (code > 0 && code <= MOE_ERR_DEVICE_INDEX) ? (moe_status)code : MOE_OK;
-}
-
-#define MOE_INJECT(name)                                \
-    do {                                                \
-        moe_status inj_ = injected(name);               \
-        if (inj_ != MOE_OK) return inj_;                \
-    } while (0)
 
 moe_status check_dims(const moe_dims *d) {
     if (!d) return MOE_ERR_INVALID_ARG;

@@ -134,6 +134,18 @@ struct DeviceInfo {
 // Per-device facts, looked up once per device (current device).
 const DeviceInfo &device_info();
 
+// Host-side fault injection for callers' error paths: MOE_INJECT_FAILURE
+// "<entry point>:<status>" makes that entry return the status at once,
+// before anything is validated or launched.  Read on every call (tests set
+// it per process); nothing is injected when it is unset.
+moe_status injected_failure(const char *entry);
+
+#define MOE_INJECT(name)                                 \
+    do {                                                 \
+        moe_status inj_ = ::moe::injected_failure(name); \
+        if (inj_ != MOE_OK) return inj_;                 \
+    } while (0)
+
 // Launch bookkeeping: counts every launch and, when profiling is on,
 // brackets it with CUDA events on its stream.
 struct LaunchScope {
@@ -188,8 +200,10 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
 cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
                               const int32_t *offsets, const void *w1, const void *v1, void *h,
                               cudaStream_t st);
+// name: the profiling name of the launch (default "gemm_down_tc").
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
-                                const void *w2, float *y_sorted, cudaStream_t st);
+                                const void *w2, float *y_sorted, cudaStream_t st,
+                                const char *name = nullptr);
 
 // Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
 // kStreamMaxSlots slots; the GLU hidden vectors h are bf16.  Batches of at
@@ -200,9 +214,11 @@ bool stream_path_ok(const moe_dims &d, int T);
 cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
                                  const int32_t *offsets, const void *w1, const void *v1, void *h,
                                  cudaStream_t st);
+// name: the profiling name of the launch (default "down_combine_stream" /
+// "down_stream").
 cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                const int32_t *inv_perm, const void *w2, const float *gate,
                                const void *residual, void *out, float *y_sorted, bool fused,
-                               cudaStream_t st);
+                               cudaStream_t st, const char *name = nullptr);
 
 }  // namespace moe

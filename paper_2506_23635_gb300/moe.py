@@ -32,6 +32,8 @@ EXPORTS = (
     "moe_selftest_wait_timeout", "moe_dense_workspace_size", "moe_layer_forward_dense",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
     "moe_profile_reset", "moe_profile_read",
+    "moe_sa_workspace_size", "moe_sa_qkv", "moe_sa_attend", "moe_sa_forward",
+    "moe_decoder_workspace_size", "moe_decoder_forward",
 )
 
 
@@ -50,6 +52,17 @@ class Dims(ctypes.Structure):
     def __repr__(self):
         return (f"Dims(D={self.d_model}, F={self.ffn_hidden}, E={self.n_experts}, "
                 f"K={self.top_k}, w={self.w_dtype}, x={self.x_dtype}, out={self.out_dtype})")
+
+
+class SaDims(ctypes.Structure):
+    """moe_sa_dims: the self-attention block's shape."""
+    _fields_ = [("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("rope_base", ctypes.c_float)]
+
+    def __repr__(self):
+        return (f"SaDims(D={self.d_model}, Hq={self.n_heads}, Hkv={self.n_kv_heads}, "
+                f"dh={self.head_dim}, base={self.rope_base})")
 
 
 class KernelStat(ctypes.Structure):
@@ -75,6 +88,7 @@ def lib() -> ctypes.CDLL:
     L = ctypes.CDLL(path)
     P, I32, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
     DP = ctypes.POINTER(Dims)
+    SP = ctypes.POINTER(SaDims)
     sigs = {
         "moe_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
         "moe_route": [DP, I32, P, P, P, P, P, P],
@@ -96,6 +110,13 @@ def lib() -> ctypes.CDLL:
         "moe_profile_reset": [],
         "moe_profile_read": [ctypes.POINTER(KernelStat), I32],
         "moe_launch_count": [],
+        "moe_sa_workspace_size": [SP, I32, ctypes.POINTER(SZ)],
+        "moe_sa_qkv": [SP, I32, P, P, P, P, I32, I32, P, P, P, P, SZ, P],
+        "moe_sa_attend": [SP, I32, P, P, P, I32, I32, P, P, P, P, SZ, P],
+        "moe_sa_forward": [SP, I32, P, P, I32, I32, P, P, P, P, P, ctypes.c_float, P, SZ, P],
+        "moe_decoder_workspace_size": [SP, DP, I32, ctypes.POINTER(SZ)],
+        "moe_decoder_forward": [SP, DP, I32, I32, P, P, I32, I32, P] + [ctypes.POINTER(P)] * 8
+                               + [ctypes.c_float, P, SZ, P],
     }
     for name, args in sigs.items():
         fn = getattr(L, name)
@@ -334,3 +355,104 @@ def profile_read() -> dict:
 
 def status_string(code: int) -> str:
     return lib().moe_status_string(code).decode()
+
+
+# ---- self-attention block and whole decoder layers --------------------------
+
+
+def sa_dims(d_model: int, n_heads: int, n_kv_heads: int, head_dim: int = 128,
+            rope_base: float = 500000.0) -> SaDims:
+    return SaDims(d_model, n_heads, n_kv_heads, head_dim, rope_base)
+
+
+def sa_workspace_size(a: SaDims, max_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().moe_sa_workspace_size(ctypes.byref(a), max_tokens, ctypes.byref(n)),
+           "moe_sa_workspace_size")
+    return int(n.value)
+
+
+def _sa_ws(a: SaDims, T: int, device, ws):
+    if ws is None:
+        ws = torch.empty(max(sa_workspace_size(a, T), 256), dtype=torch.uint8, device=device)
+    return ws
+
+
+def sa_qkv(a: SaDims, x_norm, w_qkv, seq, pos, k_cache, v_cache, q=None, ws=None, stream=None):
+    """Rotated queries q [T, Hq, dh] (fp32); the T tokens' keys and values
+    written into the caches [n_seq, Hkv, max_len, dh] at (seq[t], pos[t])."""
+    T = x_norm.shape[0]
+    n_seq, _, max_len, _ = k_cache.shape
+    if q is None:
+        q = torch.empty((T, a.n_heads, a.head_dim), dtype=torch.float32, device=x_norm.device)
+    ws = _sa_ws(a, T, x_norm.device, ws)
+    _check(lib().moe_sa_qkv(ctypes.byref(a), T, _ptr(x_norm), _ptr(w_qkv), _ptr(seq), _ptr(pos),
+                            n_seq, max_len, _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(ws),
+                            ws.numel(), _stream(stream)), "moe_sa_qkv")
+    return q
+
+
+def sa_attend(a: SaDims, q, seq, pos, k_cache, v_cache, ctx=None, ws=None, stream=None):
+    """ctx [T, Hq * dh] (bf16): causal attention of each token over positions
+    0..pos[t] of its sequence."""
+    T = q.shape[0]
+    n_seq, _, max_len, _ = k_cache.shape
+    if ctx is None:
+        ctx = torch.empty((T, a.n_heads * a.head_dim), dtype=torch.bfloat16, device=q.device)
+    ws = _sa_ws(a, T, q.device, ws)
+    _check(lib().moe_sa_attend(ctypes.byref(a), T, _ptr(q), _ptr(seq), _ptr(pos), n_seq,
+                               max_len, _ptr(k_cache), _ptr(v_cache), _ptr(ctx), _ptr(ws),
+                               ws.numel(), _stream(stream)), "moe_sa_attend")
+    return ctx
+
+
+def sa_forward(a: SaDims, resid, w_qkv, w_o, seq, pos, k_cache, v_cache, eps: float = STACK_EPS,
+               ws=None, stream=None):
+    """resid <- resid + W_o . Attn(RMSNorm0(resid)) in place (fp32 [T, D])."""
+    T = resid.shape[0]
+    n_seq, _, max_len, _ = k_cache.shape
+    ws = _sa_ws(a, T, resid.device, ws)
+    _check(lib().moe_sa_forward(ctypes.byref(a), T, _ptr(seq), _ptr(pos), n_seq, max_len,
+                                _ptr(resid), _ptr(w_qkv), _ptr(w_o), _ptr(k_cache),
+                                _ptr(v_cache), eps, _ptr(ws), ws.numel(), _stream(stream)),
+           "moe_sa_forward")
+    return resid
+
+
+def decoder_workspace_size(a: SaDims, d: Dims, max_tokens: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().moe_decoder_workspace_size(ctypes.byref(a), ctypes.byref(d), max_tokens,
+                                            ctypes.byref(n)), "moe_decoder_workspace_size")
+    return int(n.value)
+
+
+class DecoderWeights:
+    """Device pointers of every decoder layer's tensors as C arrays: per
+    layer (w_qkv, w_o, w_r, w1, v1, w2, k_cache, v_cache).  The tensors must
+    outlive this object's use."""
+
+    def __init__(self, layers):
+        n = len(layers)
+        self.n = n
+        self.tensors = layers
+        arr = lambda i: (ctypes.c_void_p * n)(*[ctypes.c_void_p(l[i].data_ptr()) for l in layers])
+        (self.w_qkv, self.w_o, self.w_r, self.w1, self.v1, self.w2, self.k_cache,
+         self.v_cache) = (arr(i) for i in range(8))
+        self.n_seq, _, self.max_len, _ = layers[0][6].shape
+
+
+def decoder_forward(a: SaDims, d: Dims, weights: DecoderWeights, resid, seq, pos,
+                    eps: float = STACK_EPS, ws=None, stream=None):
+    """Every decoder layer in order, in place on resid (fp32 [T, D]):
+    resid += W_o . Attn(RMSNorm0(resid)); resid += MoE(RMSNorm0(resid))."""
+    T = resid.shape[0]
+    if ws is None:
+        ws = torch.empty(max(decoder_workspace_size(a, d, T), 256), dtype=torch.uint8,
+                         device=resid.device)
+    W = weights
+    _check(lib().moe_decoder_forward(ctypes.byref(a), ctypes.byref(d), W.n, T, _ptr(seq),
+                                     _ptr(pos), W.n_seq, W.max_len, _ptr(resid), W.w_qkv, W.w_o,
+                                     W.w_r, W.w1, W.v1, W.w2, W.k_cache, W.v_cache, eps,
+                                     _ptr(ws), ws.numel(), _stream(stream)),
+           "moe_decoder_forward")
+    return resid

@@ -26,7 +26,13 @@ def bounds(dtype: str):
     return (REL_L2, MAX_ABS_OF_RMS) if dtype == "bf16" else (REL_L2_F32, MAX_ABS_OF_RMS_F32)
 
 
-def assert_parity(got, want, dtype: str = "bf16", what: str = ""):
+def assert_parity(got, want, dtype: str = "bf16", what: str = "", stored_bf16: bool = False):
+    """rel L2 and max abs bounds of the path's dtype.  stored_bf16: the
+    compared tensor is an intermediate that the path stores in bf16, so each
+    element may also carry one bf16 rounding (2^-8 of its magnitude) beyond
+    the max abs bound -- rows of very different magnitude (an attention
+    output that is one value row next to one that averages thousands) make
+    a bound on the RMS alone meaningless for them."""
     rel_l2, max_abs = bounds(dtype)
     g = np.asarray(got, np.float64)
     w = np.asarray(want, np.float64)
@@ -38,7 +44,12 @@ def assert_parity(got, want, dtype: str = "bf16", what: str = ""):
     rms = float(np.sqrt(np.mean(w * w))) if w.size else 0.0
     mx = float(np.max(np.abs(err))) if err.size else 0.0
     assert rel <= rel_l2, f"{what}: rel L2 {rel:.3e} > {rel_l2}"
-    assert mx <= max_abs * rms + 1e-30, f"{what}: max abs {mx:.3e} > {max_abs}*RMS ({rms:.3e})"
+    if stored_bf16:
+        lim = max_abs * rms + 2.0 ** -8 * np.abs(w) + 1e-30
+        worst = float(np.max(np.abs(err) - lim)) if err.size else 0.0
+        assert worst <= 0, f"{what}: an element exceeds {max_abs}*RMS + one bf16 rounding"
+    else:
+        assert mx <= max_abs * rms + 1e-30, f"{what}: max abs {mx:.3e} > {max_abs}*RMS ({rms:.3e})"
     return rel, mx / rms if rms else 0.0
 
 

@@ -552,4 +552,29 @@ def pin_sa_bf16_storage(orc):
         assert np.array_equal(gen.to_f64(gen.store(c, "bf16"), "bf16"), c), "cache not bf16"
 
 
+def pin_decoder_layer_composition(orc):
+    """A decoder layer whose output projection is zero is the MoE stack
+    layer alone (pinned above); with it, the layer is the self-attention
+    block followed by that stack layer."""
+    rng = np.random.default_rng(67)
+    D, Hq, Hkv, dh = 32, 4, 2, 8
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh)
+    (w_r, w1, v1, w2), = _stack_layers(69, 1, D=D)
+    x0 = gen.store(rng.normal(size=(3, D)), "f32")
+    seq = np.array([0, 1, 1], np.int32)
+    pos = np.array([3, 5, 6], np.int32)
+    zero_o = gen.store(np.zeros((D, Hq * dh)), "f32")
+    got, _, gaps = orc.decoder_layers(gen.to_f64(x0, "f32"), [(w_qkv, zero_o, w_r, w1, v1, w2)],
+                                      "f32", Hq, Hkv, 1000.0, 1e-6, 2, seq, pos, [(kc, vc)])
+    want, wgaps = orc.stack_tokens(x0, [(w_r, w1, v1, w2)], "f32", 2, 1e-6)
+    _close(got, want, 1e-12, 1e-14, "decoder layer with zero output projection")
+    _close(gaps, wgaps, 1e-12, 0, "routing gaps")
+    got, _, _ = orc.decoder_layers(gen.to_f64(x0, "f32"), [(w_qkv, w_o, w_r, w1, v1, w2)],
+                                   "f32", Hq, Hkv, 1000.0, 1e-6, 2, seq, pos, [(kc, vc)])
+    mid, _, _ = orc.sa_forward(gen.to_f64(x0, "f32"), w_qkv, w_o, "f32", Hq, Hkv, 1000.0, 1e-6,
+                               seq, pos, kc, vc)
+    want, _ = orc.stack_tokens(mid, [(w_r, w1, v1, w2)], "f64", 2, 1e-6)
+    _close(got, want, 1e-12, 1e-14, "decoder layer = attention block then stack layer")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -164,3 +164,61 @@ def test_fault_injection_env(lib):
     out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
                          timeout=120)
     assert list(map(int, out.stdout.split())) == [5, 1]
+
+
+@no_gpu
+def test_attention_and_decoder_validation(lib):
+    """The self-attention and decoder entry points reject bad shapes,
+    pointers and workspaces before touching the device."""
+    L = lib.lib()
+    a = lib.sa_dims(6144, 48, 8)
+    n = ctypes.c_size_t(0)
+    size = lambda dims, T=1: L.moe_sa_workspace_size(ctypes.byref(dims), T, ctypes.byref(n))
+    assert size(a) == 0 and n.value > 0
+    one = n.value
+    assert size(a, 2048) == 0 and n.value > one
+    assert size(lib.sa_dims(6144, 48, 8, head_dim=64)) == 2
+    assert size(lib.sa_dims(6144, 48, 7)) == 1          # 7 does not divide 48
+    assert size(lib.sa_dims(6144, 48, 4)) == 2          # 12 query heads per group
+    assert size(lib.sa_dims(6144, 48, 8, rope_base=1.0)) == 1
+    assert size(lib.sa_dims(6100, 48, 8)) == 1          # D not a multiple of 8
+    assert size(a, 65537) == 1
+    fwd = lambda T, resid=A, ws=A, nb=one, seq=A, n_seq=1, ln=8: L.moe_sa_forward(
+        ctypes.byref(a), T, seq, A, n_seq, ln, resid, A, A, A, A, 1e-6, ws, nb, None)
+    assert fwd(0) == 0
+    assert fwd(1, resid=None) == 1
+    assert fwd(1, seq=None) == 1
+    assert fwd(1, n_seq=0) == 1
+    assert fwd(1, ln=0) == 1
+    assert fwd(1, resid=MIS) == 1
+    assert fwd(1, ws=None) == 3
+    assert fwd(1, nb=one - 1) == 3
+    assert L.moe_sa_attend(ctypes.byref(a), 1, A, A, A, 1, 8, A, A, None, A, one, None) == 1
+    assert L.moe_sa_qkv(ctypes.byref(a), 1, A, A, A, A, 1, 8, A, A, A, A, 0, None) == 3
+    d = lib.dims(**DBRX, out_dtype=torch.float32)
+    P = ctypes.c_void_p
+    arr = (P * 1)(A)
+    dec = lambda dims, attn=a: L.moe_decoder_forward(
+        ctypes.byref(attn), ctypes.byref(dims), 1, 1, A, A, 1, 8, A, arr, arr, arr, arr, arr,
+        arr, arr, arr, 1e-6, A, 1 << 30, None)
+    assert dec(lib.dims(**DBRX)) == 1                   # the residual stream must be fp32
+    assert dec(d, attn=lib.sa_dims(4096, 32, 8)) == 1   # widths differ
+    assert L.moe_decoder_workspace_size(ctypes.byref(a), ctypes.byref(d), 8, ctypes.byref(n)) == 0
+    assert n.value >= one
+
+
+def test_fault_injection_reaches_the_attention_entries(lib):
+    code = (
+        "import ctypes, sys; sys.path.insert(0, %r)\n"
+        "from paper_2506_23635_gb300 import moe\n"
+        "L = moe.lib(); a = moe.sa_dims(256, 4, 2)\n"
+        "print(L.moe_sa_forward(ctypes.byref(a), 1, None, None, 1, 8, None, None, None, None,\n"
+        "                       None, 1e-6, None, 0, None))\n" % ROOT)
+    import subprocess
+    import sys
+    for env_value, want in (("moe_sa_forward:5", 5), ("moe_sa_qkv:5", 1)):
+        env = dict(os.environ, MOE_INJECT_FAILURE=env_value)
+        out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True,
+                             env=env, timeout=120)
+        assert out.returncode == 0, out.stderr
+        assert int(out.stdout) == want
