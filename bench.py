@@ -62,6 +62,17 @@ WORKLOADS = {
 }
 PREFILL_MIN_TOKENS = 512
 
+# whole decoder layers (the DBRX self-attention block in front of the MoE
+# layer), decode at context 2048: name -> (MoE shape, sequences per step)
+DECODER_WORKLOADS = {
+    "dbrx-decoder-t1": (gen.DBRX, 1),
+    "dbrx-decoder-t8": (gen.DBRX, 8),
+    # 4 DBRX-shaped experts resident (1.9 GB in all): the small case for ncu
+    # captures of the attention block's kernels
+    "dbrx4-decoder-t8": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 8),
+}
+METRIC_DECODER = "Decoder-layer us/token-step (DBRX-shaped attention + MoE, decode at context 2048)"
+
 
 def parse():
     p = argparse.ArgumentParser()
@@ -69,7 +80,8 @@ def parse():
     p.add_argument("--steps", type=int, default=4000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", choices=sorted(WORKLOADS), default="dbrx-decode-t1")
+    p.add_argument("--workload", choices=sorted(WORKLOADS) + sorted(DECODER_WORKLOADS),
+                   default="dbrx-decode-t1")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-extra", action="store_true",
                    help="skip the prefill and decode-sweep side measurements")
@@ -413,7 +425,7 @@ def measure_extra(layer, workload, steps, warmup):
     return r
 
 
-def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True):
+def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True, decoder=True):
     """The 16-layer DBRX-shaped stack (about 101 GB of bf16 weights resident,
     each layer independently seeded), x_{l+1} = x_l + MoE_l(RMSNorm0(x_l)) with
     an fp32 residual stream; decode at batch 1 and 8 for 64 consecutive steps,
@@ -490,7 +502,124 @@ def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True):
             except Exception as exc:  # report, keep the plain numbers
                 r["graph"] = {"error": str(exc)[:200]}
         res[f"batch{T}"] = r
+    if decoder:
+        res["decoder"] = _decoder_stack(moe, dev, layers, d, n_layers, steps, batches)
     del layers, sw
+    torch.cuda.empty_cache()
+    return res
+
+
+def _decoder_stack(moe, dev, moe_layers, d, n_layers, steps, batches, ctx_len=2048):
+    """The same 16 MoE layers as full decoder layers: a DBRX self-attention
+    block (D_qkv = 8,192) in front of each.  Batch T = T sequences decoding
+    64 consecutive positions ending at ctx_len - 1 (caches pre-filled with
+    synthetic earlier entries)."""
+    import torch
+
+    a_shape = gen.DBRX_ATTN
+    a = moe.sa_dims(a_shape.d_model, a_shape.n_heads, a_shape.n_kv_heads, a_shape.head_dim,
+                    a_shape.rope_base)
+    D = a_shape.d_model
+    out = {"layers": n_layers, "context_end": ctx_len, "steps": steps}
+    attn_w = [gen.device_attn_weights(a_shape, SEED + 7, dev, layer=l) for l in range(n_layers)]
+    stream = torch.cuda.current_stream(dev)
+    for T in batches:
+        caches = [gen.device_kv_cache(a_shape, T, ctx_len, SEED + 7, dev, layer=l)
+                  for l in range(n_layers)]
+        W = moe.DecoderWeights([attn_w[l] + moe_layers[l] + caches[l] for l in range(n_layers)])
+        xs = torch.stack([gen.host_to_torch(gen.host_normal((T, D), 1.0, "bf16", SEED, "dec-x",
+                                                            T, s), "bf16", dev).float()
+                          for s in range(steps)])
+        seq = torch.arange(T, dtype=torch.int32, device=dev)
+        pos = [torch.full((T,), ctx_len - steps + s, dtype=torch.int32, device=dev)
+               for s in range(steps)]
+        resid = torch.empty((T, D), dtype=torch.float32, device=dev)
+        ws = torch.empty(moe.decoder_workspace_size(a, d, T), dtype=torch.uint8, device=dev)
+
+        def step(s):
+            resid.copy_(xs[s % steps])
+            moe.decoder_forward(a, d, W, resid, seq, pos[s % steps], ws=ws, stream=stream)
+
+        for s in range(3):
+            step(s)
+        moe.check_device_errors(stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(steps):
+            step(s)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        moe.check_device_errors(stream)
+        ms = e0.elapsed_time(e1) / steps
+        out[f"batch{T}"] = {"ms_per_step": round(ms, 4), "us_per_token_step": round(ms * 1e3 / T, 2),
+                            "tokens_per_s": round(T / (ms / 1e3), 1)}
+        del W, caches
+        torch.cuda.empty_cache()
+    del attn_w
+    return out
+
+
+def sa_bytes(a, T, ctx_len):
+    """Bytes one self-attention block must move per decode step: W_qkv and
+    W_o once, every token's cached keys and values over its context, the new
+    keys/values and the activations (fp32 residual in and out, bf16 ctx)."""
+    D, Hq, Hkv, dh = a.d_model, a.n_heads, a.n_kv_heads, a.head_dim
+    nr = (Hq + 2 * Hkv) * dh
+    return (nr * D * 2 + D * Hq * dh * 2 + T * ctx_len * Hkv * dh * 2 * 2
+            + T * (2 * D * 4 + Hq * dh * 2 + 2 * Hkv * dh * 2))
+
+
+def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5):
+    """One DBRX-shaped decoder layer (the self-attention block with D_qkv =
+    8,192 in front of this MoE layer) in decode: T sequences, one new token
+    each, at position ctx_len - 1 of a KV cache filled with synthetic earlier
+    entries; fp32 residual stream."""
+    import torch
+
+    moe, dev = layer.moe, layer.dev
+    a_shape = gen.DBRX_ATTN
+    a = moe.sa_dims(a_shape.d_model, a_shape.n_heads, a_shape.n_kv_heads, a_shape.head_dim,
+                    a_shape.rope_base)
+    d32 = moe.dims(layer.shape.d_model, layer.shape.ffn_hidden, layer.shape.n_experts,
+                   layer.shape.top_k, torch.bfloat16, torch.bfloat16, torch.float32)
+    w_qkv, w_o = gen.device_attn_weights(a_shape, SEED, dev)
+    kc, vc = gen.device_kv_cache(a_shape, T, ctx_len, SEED, dev)
+    xs_host, w_r_host = token_pool(layer.shape, T, SEED, 16)
+    w_r = gen.host_to_torch(w_r_host, "bf16", dev)
+    xs = gen.host_to_torch(xs_host, "bf16", dev).float()
+    w1, v1, w2 = layer.w
+    W = moe.DecoderWeights([(w_qkv, w_o, w_r, w1, v1, w2, kc, vc)])
+    seq = torch.arange(T, dtype=torch.int32, device=dev)
+    pos = torch.full((T,), ctx_len - 1, dtype=torch.int32, device=dev)
+    resid = torch.empty((T, layer.shape.d_model), dtype=torch.float32, device=dev)
+    ws = torch.empty(moe.decoder_workspace_size(a, d32, T), dtype=torch.uint8, device=dev)
+
+    def step(i):
+        resid.copy_(xs[i % 16])
+        moe.decoder_forward(a, d32, W, resid, seq, pos, ws=ws, stream=layer.stream)
+
+    for i in range(warmup):
+        step(i)
+    ms, launches, kstats = layer.time_steps(step, steps)
+    sa_names = ("sa_prenorm", "qkv_stream", "qkv_rows_tc", "qkv_gemm_tc", "rope_cache",
+                "attention", "attn_merge", "o_stream", "o_rows_tc", "o_gemm_tc", "residual_add")
+    sa_ms = sum(v[1] for k, v in kstats.items() if k in sa_names) / steps
+    b = sa_bytes(a, T, ctx_len)
+    peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
+    kv = T * ctx_len * a.n_kv_heads * a.head_dim * 4
+    att = kstats.get("attention")
+    res = {"tokens_per_step": T, "context": ctx_len, "ms_per_step": round(ms, 4),
+           "launches_per_step": launches / steps,
+           "attention_block": {"us_per_step": round(sa_ms * 1e3, 2),
+                               "algorithmic_bytes": b,
+                               "achieved_gbs": round(b / (sa_ms / 1e3) / 1e9, 1),
+                               "frac_of_hbm": round(b / (sa_ms / 1e3) / 1e9 / peak, 4)},
+           "kernels": kernel_table(kstats)}
+    if att:
+        s_att = att[1] / att[0] / 1e3
+        res["attention_block"]["kv_read_gbs"] = round(kv / s_att / 1e9, 1)
+    del W, w_qkv, w_o, kc, vc
     torch.cuda.empty_cache()
     return res
 
@@ -520,6 +649,36 @@ def measure_dense(layer, T, steps=100, warmup=3):
             "kernels": kernel_table(kstats)}
 
 
+def run_decoder(args, moe, dev, dist, rank, world):
+    """A whole decoder layer as the measured step (device-resident inputs);
+    one JSON line with the step time per token and the attention block's
+    share and roofline."""
+    shape, T = DECODER_WORKLOADS[args.workload]
+    layer = Layer(moe, shape, dev, dist)
+    r = measure_decoder_layer(layer, T, steps=args.steps, warmup=max(3, args.warmup))
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+    line = {
+        "metric": METRIC_DECODER, "value": round(r["ms_per_step"] * 1e3 / T, 3),
+        "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
+        "ms_per_step": r["ms_per_step"], "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,0.02^2) bf16 weights, N(0,1) tokens, KV cache "
+                "pre-filled with synthetic entries)",
+        "config": {"workload": args.workload, "d_model": shape.d_model,
+                   "ffn_hidden": shape.ffn_hidden, "n_experts": shape.n_experts,
+                   "top_k": shape.top_k, "sequences_per_step": T, "context": r["context"],
+                   "attention": "48 query / 8 key-value heads of 128 (D_qkv = 8192)"},
+        "attention_block": r["attention_block"], "kernels": r["kernels"],
+        "gpu_launches": int(r["launches_per_step"] * args.steps),
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
 def run_ours(args):
     import torch
 
@@ -529,6 +688,8 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dist = init_dist(world, "nccl")
     dev = torch.device("cuda", local)
+    if args.workload in DECODER_WORKLOADS:
+        return run_decoder(args, moe, dev, dist, rank, world)
     shape, T = WORKLOADS[args.workload]
     D, F, E, K = shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k
     prefill = T >= PREFILL_MIN_TOKENS
@@ -591,6 +752,7 @@ def run_ours(args):
         extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5)
                                  for t in (2, 4, 8, 16, 32, 64)]
         extra["busy_full_loading"] = [measure_dense(layer, t) for t in (1, 8)]
+        extra["decoder_layer"] = [measure_decoder_layer(layer, t) for t in (1, 8)]
         extra["stack"] = measure_stack(moe, dev)
 
     if rank != 0:
@@ -696,7 +858,8 @@ def run_reference(args):
         return
     import oracle
 
-    shape, T = WORKLOADS[args.workload]
+    decoder = args.workload in DECODER_WORKLOADS
+    shape, T = DECODER_WORKLOADS[args.workload] if decoder else WORKLOADS[args.workload]
     prefill = T >= PREFILL_MIN_TOKENS
     pool = 1 if prefill else POOL
     xs_host, w_r_host = token_pool(shape, T, SEED, pool)
@@ -716,9 +879,20 @@ def run_reference(args):
         w1, v1, w2 = gen.host_expert_weights(shape, SEED)
         src = "host-drawn seeded weights"
     chunk = 16
+    if decoder:  # the attention block's weights and caches, host-drawn
+        a_shape, ctx_len = gen.DBRX_ATTN, 2048
+        w_qkv, w_o = gen.host_attn_weights(a_shape, SEED)
+        kc, vc = (gen.to_f64(c, "bf16") for c in gen.host_kv_cache(a_shape, T, ctx_len, SEED))
+        seq = np.arange(T, dtype=np.int32)
+        pos = np.full(T, ctx_len - 1, np.int32)
 
     def one(i):
-        if prefill:
+        if decoder:
+            x = gen.to_f64(xs_host[i % pool], shape.dtype)
+            oracle.decoder_layers(x, [(w_qkv, w_o, w_r_host, w1, v1, w2)], shape.dtype,
+                                  a_shape.n_heads, a_shape.n_kv_heads, a_shape.rope_base, 1e-6,
+                                  shape.top_k, seq, pos, [(kc, vc)])
+        elif prefill:
             t0 = (i * chunk) % T
             toks = np.arange(t0, t0 + chunk, dtype=np.int32)
             oracle.layer_tokens(xs_host[0], w_r_host, w1, v1, w2, shape.dtype, shape.top_k,
@@ -743,7 +917,7 @@ def run_reference(args):
         value = round(flops / (ms / 1e3) / 1e12, 6)
         sample = f"{steps} steps of {chunk} of the {T} tokens (of {args.steps} requested)"
     else:
-        metric, unit, hib = METRIC, UNIT, False
+        metric, unit, hib = (METRIC_DECODER if decoder else METRIC), UNIT, False
         value = round(ms * 1e3 / T, 1)
         sample = f"{steps} token-steps of {T} token(s) (of {args.steps} requested)"
     line = {

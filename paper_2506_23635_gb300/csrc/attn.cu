@@ -15,15 +15,18 @@
 //                  two projections run on the MoE layer's own projection
 //                  kernels with E = K = 1;
 //   projection     W_qkv . x: the row-streaming kernel for one token, the
-//                  tcgen05 GEMM otherwise (fp32 out);
-//   k_rope_cache   rotary embedding of q and k (angles in fp64), k and v
-//                  written to the cache in bf16;
+//                  tcgen05 kernel with the weights as the M operand for up to
+//                  64 tokens, the grouped tcgen05 GEMM beyond (fp32 out);
+//   k_rope_cache   rotary embedding of q and k (angles formed and reduced in
+//                  fp64, evaluated in fp32), k and v written to the cache in
+//                  bf16;
 //   k_attn_partial one CTA per (token, key/value head, position split): the
 //                  group's query heads against its positions, online softmax,
 //                  partial (max, sum, weighted values) per split;
 //   k_attn_merge   merges the splits, ctx in bf16;
 //   projection     W_o . ctx added to the residual (fused into the streaming
-//                  kernel for one token; GEMM + k_residual_add otherwise).
+//                  kernel for one token; a tcgen05 kernel + k_residual_add
+//                  otherwise).
 #include <math.h>
 
 #include <algorithm>
@@ -37,18 +40,38 @@ constexpr int kHeadDim = 128;
 constexpr int kMaxGroup = 8;       // query heads per key/value head
 constexpr int kAttnThreads = 128;  // 4 warps
 constexpr int kAttnWarps = kAttnThreads / 32;
-constexpr int kPosInFlight = 4;    // positions a warp loads before using them
-constexpr int kSplitTarget = 320;  // CTAs a decode step's attention aims for
-constexpr int kMaxSplit = 32;
+constexpr int kPosInFlight = 8;    // positions a warp loads before using them
+constexpr int kSplitTarget = 304;     // CTAs a decode step's attention aims for at least
+constexpr int kSplitPositions = 128;  // cache positions per split it aims for at most
+constexpr int kMaxSplit = 64;
+constexpr int kMaxSplitCtas = 4096;   // bound on T * Hkv * splits (sizes the workspace)
 constexpr int kMaxSaTokens = 65536;
 
-int n_split_for(int T, int Hkv) {
-    const int tg = T * Hkv;
-    return std::max(1, std::min(kMaxSplit, (kSplitTarget + tg - 1) / tg));
+// Most position splits a call of T tokens may use (the workspace holds this many).
+int split_cap(int T, int Hkv) {
+    const int tg = std::max(1, T * Hkv);
+    return std::max(1, std::min(kMaxSplit, kMaxSplitCtas / tg));
 }
+
+// Splits per (token, key/value head): enough CTAs to cover the SMs and at
+// most kSplitPositions cache positions per split, within split_cap.
+int n_split_for(int T, int Hkv, int max_len) {
+    const int tg = std::max(1, T * Hkv);
+    const int by_ctas = (kSplitTarget + tg - 1) / tg;
+    const int by_len = (max_len + kSplitPositions - 1) / kSplitPositions;
+    return std::max(1, std::min(split_cap(T, Hkv), std::max(by_ctas, by_len)));
+}
+
+// Rotary angular rates base^(-2i/dh), i < dh/2, computed on the host in
+// double precision and passed by value.
+struct RopeRates {
+    double w[kHeadDim / 2];
+};
 
 // ---- kernels --------------------------------------------------------------------
 
+// The trivial dispatch of the one-"expert" projections (offsets {0, T},
+// identity permutation, unit gates).
 __device__ __forceinline__ void write_trivial_dispatch(int T, int32_t *offsets, int32_t *ident,
                                                        float *ones) {
     for (int i = threadIdx.x; i < T; i += blockDim.x) {
@@ -61,16 +84,21 @@ __device__ __forceinline__ void write_trivial_dispatch(int T, int32_t *offsets, 
     }
 }
 
-__global__ void __launch_bounds__(256)
+// One 1024-thread block per token: every thread's loads of the row are in
+// flight together.
+constexpr int kNormThreads = 1024;
+
+__global__ void __launch_bounds__(kNormThreads)
 k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ xn, float eps,
              int32_t *offsets, int32_t *ident, float *ones) {
     ptx::grid_dependency_wait();
-    __shared__ float red[8];
+    __shared__ float red[kNormThreads / 32];
     const int t = blockIdx.x;
     if (t == 0) write_trivial_dispatch(T, offsets, ident, ones);
     const float4 *r = reinterpret_cast<const float4 *>(resid + (size_t)t * D);
     const int nv = D >> 2;
     float ss = 0.f;
+#pragma unroll 4
     for (int i = threadIdx.x; i < nv; i += blockDim.x) {
         const float4 v = r[i];
         ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
@@ -80,9 +108,10 @@ k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ x
     __syncthreads();
     float tot = 0.f;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) tot += red[w];
+    for (int w = 0; w < kNormThreads / 32; ++w) tot += red[w];
     const float s = 1.0f / sqrtf(tot / (float)D + eps);
     __nv_bfloat162 *o = reinterpret_cast<__nv_bfloat162 *>(xn + (size_t)t * D);
+#pragma unroll 4
     for (int i = threadIdx.x; i < nv; i += blockDim.x) {
         const float4 v = r[i];
         o[2 * i] = __floats2bfloat162_rn(v.x * s, v.y * s);
@@ -97,49 +126,46 @@ k_sa_setup(int T, int32_t *offsets, int32_t *ident, float *ones) {
 }
 
 // qkv [T, (Hq + 2 Hkv) 128] fp32 -> q [T, Hq, 128] fp32 (rotated); rotated
-// keys and the values to the caches [n_seq, Hkv, L, 128] in bf16.
-__global__ void __launch_bounds__(128)
-k_rope_cache(int Hq, int Hkv, int n_seq, int L, double base, const int32_t *__restrict__ seq,
+// keys and the values to the caches [n_seq, Hkv, L, 128] in bf16.  One
+// 64-thread block per (head row of qkv, token): thread i turns the pair
+// (i, i + 64) of a query or key head, or copies two value elements.
+__global__ void __launch_bounds__(kHeadDim / 2)
+k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *__restrict__ seq,
              const int32_t *__restrict__ pos, const float *__restrict__ qkv, float *__restrict__ q,
              bf16 *__restrict__ kc, bf16 *__restrict__ vc, unsigned *err) {
     ptx::grid_dependency_wait();
     constexpr int H2 = kHeadDim / 2;
-    __shared__ float cs[H2], sn[H2];
-    const int t = blockIdx.x;
+    const int hr = blockIdx.x, t = blockIdx.y, i = threadIdx.x;
     const int sq = seq[t], p = pos[t];
     const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
-    if (!ok && threadIdx.x == 0) set_error(err, kErrIndex);
-    if (threadIdx.x < H2) {
-        // the angle of pair i is pos * base^(-2i/dh); fp64 keeps it exact to
-        // well below fp32 resolution at any cache position
-        const double w = pow(base, -2.0 * (double)threadIdx.x / (double)kHeadDim);
-        double s, c;
-        sincos((double)(ok ? p : 0) * w, &s, &c);
-        cs[threadIdx.x] = (float)c;
-        sn[threadIdx.x] = (float)s;
-    }
-    __syncthreads();
+    if (!ok && hr == 0 && i == 0) set_error(err, kErrIndex);
     const int nq = Hq * kHeadDim, nkv = Hkv * kHeadDim;
-    const float *row = qkv + (size_t)t * (nq + 2 * nkv);
-    float *qo = q + (size_t)t * nq;
-    for (int i = threadIdx.x; i < Hq * H2; i += blockDim.x) {
-        const int h = i / H2, k = i - h * H2;
-        const float a = row[h * kHeadDim + k], b = row[h * kHeadDim + k + H2];
-        qo[h * kHeadDim + k] = a * cs[k] - b * sn[k];
-        qo[h * kHeadDim + k + H2] = b * cs[k] + a * sn[k];
+    const float *row = qkv + (size_t)t * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
+    const float a = row[i], b = row[i + H2];
+    if (hr >= Hq + Hkv) {  // a value head: stored as it is
+        if (!ok) return;
+        bf16 *vd = vc + (((size_t)sq * Hkv + (hr - Hq - Hkv)) * L + p) * kHeadDim;
+        vd[i] = __float2bfloat16_rn(a);
+        vd[i + H2] = __float2bfloat16_rn(b);
+        return;
     }
-    if (!ok) return;
-    for (int i = threadIdx.x; i < Hkv * H2; i += blockDim.x) {
-        const int g = i / H2, k = i - g * H2;
-        const float a = row[nq + g * kHeadDim + k], b = row[nq + g * kHeadDim + k + H2];
-        bf16 *kd = kc + (((size_t)sq * Hkv + g) * L + p) * kHeadDim;
-        kd[k] = __float2bfloat16_rn(a * cs[k] - b * sn[k]);
-        kd[k + H2] = __float2bfloat16_rn(b * cs[k] + a * sn[k]);
-    }
-    for (int i = threadIdx.x; i < nkv; i += blockDim.x) {
-        const int g = i / kHeadDim, k = i - g * kHeadDim;
-        vc[(((size_t)sq * Hkv + g) * L + p) * kHeadDim + k] =
-            __float2bfloat16_rn(row[nq + nkv + i]);
+    // the angle of pair i is pos * rate_i, formed and reduced to [-pi, pi]
+    // in fp64 (exact to far below fp32 resolution at any cache position),
+    // then evaluated in fp32
+    constexpr double kTwoPi = 6.283185307179586;
+    const double ang = (double)(ok ? p : 0) * rates.w[i];
+    const double red = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);
+    float sn, cs;
+    sincosf((float)red, &sn, &cs);
+    const float x0 = a * cs - b * sn, x1 = b * cs + a * sn;
+    if (hr < Hq) {
+        float *qo = q + (size_t)t * nq + (size_t)hr * kHeadDim;
+        qo[i] = x0;
+        qo[i + H2] = x1;
+    } else if (ok) {
+        bf16 *kd = kc + (((size_t)sq * Hkv + (hr - Hq)) * L + p) * kHeadDim;
+        kd[i] = __float2bfloat16_rn(x0);
+        kd[i + H2] = __float2bfloat16_rn(x1);
     }
 }
 
@@ -257,22 +283,46 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
     }
 }
 
-// ctx[t, h*128 + d] = merged weighted values / merged sum, over the splits.
-__global__ void __launch_bounds__(kHeadDim)
+// ctx[t, h*128 + d] = merged weighted values / merged sum, over the splits:
+// ctx = sum_s e^(M_s - M) A_s[d] / sum_s e^(M_s - M) L_s.  The splits'
+// (max, sum) pairs are read once into shared memory; kMergeGroups groups of
+// 128 threads each sum every kMergeGroups-th split of their dimension with
+// independent loads, and the groups' sums are added in group order.
+constexpr int kMergeGroups = 4;
+
+__global__ void __launch_bounds__(kHeadDim * kMergeGroups)
 k_attn_merge(int n_split, const float *__restrict__ part_ml, const float *__restrict__ part_acc,
              bf16 *__restrict__ ctx) {
+    static_assert(kMaxSplit <= kHeadDim * kMergeGroups, "one thread per split");
     ptx::grid_dependency_wait();
-    const int th = blockIdx.x, d = threadIdx.x;
+    __shared__ float sm[kMaxSplit], sl[kMaxSplit], sc[kMaxSplit];
+    __shared__ float sa[kMergeGroups][kHeadDim], sls[kMergeGroups][kHeadDim];
+    const int th = blockIdx.x, tid = threadIdx.x;
+    const int d = tid % kHeadDim, grp = tid / kHeadDim;
     const float *ml = part_ml + (size_t)th * n_split * 2;
+    if (tid < n_split) {
+        sm[tid] = ml[2 * tid];
+        sl[tid] = ml[2 * tid + 1];
+    }
+    __syncthreads();
     float M = -INFINITY;
-    for (int s = 0; s < n_split; ++s) M = fmaxf(M, ml[2 * s]);
+    for (int k = 0; k < n_split; ++k) M = fmaxf(M, sm[k]);
+    if (tid < n_split) sc[tid] = M != -INFINITY ? expf(sm[tid] - M) : 0.f;
+    __syncthreads();
     float Ls = 0.f, A = 0.f;
-    if (M != -INFINITY) {
-        for (int s = 0; s < n_split; ++s) {
-            const float c = expf(ml[2 * s] - M);
-            Ls = fmaf(ml[2 * s + 1], c, Ls);
-            A = fmaf(part_acc[((size_t)th * n_split + s) * kHeadDim + d], c, A);
-        }
+    const float *pa = part_acc + (size_t)th * n_split * kHeadDim + d;
+#pragma unroll 4
+    for (int k = grp; k < n_split; k += kMergeGroups) {
+        Ls = fmaf(sl[k], sc[k], Ls);
+        A = fmaf(pa[(size_t)k * kHeadDim], sc[k], A);
+    }
+    sa[grp][d] = A;
+    sls[grp][d] = Ls;
+    __syncthreads();
+    if (grp != 0) return;
+    for (int g = 1; g < kMergeGroups; ++g) {
+        A += sa[g][d];
+        Ls += sls[g][d];
     }
     ctx[(size_t)th * kHeadDim + d] = __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
 }
@@ -304,8 +354,7 @@ SaWs sa_ws(const moe_sa_dims &d, int64_t T) {
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
     const size_t nq = (size_t)d.n_heads * kHeadDim;
     const size_t nr = nq + 2 * (size_t)d.n_kv_heads * kHeadDim;
-    const size_t parts = (size_t)T * d.n_heads * n_split_for((int)std::max<int64_t>(T, 1),
-                                                             d.n_kv_heads);
+    const size_t parts = (size_t)T * d.n_heads * split_cap((int)T, d.n_kv_heads);
     SaWs L{};
     size_t o = 0;
     L.offsets = o; o += up(2 * 4);
@@ -390,23 +439,29 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
         e = launch_down_stream(pd, 1, xn, offsets, at<int32_t>(c.ws, c.L.ident), w_qkv,
                                at<float>(c.ws, c.L.ones), nullptr, nullptr, qkv, false, c.st,
                                "qkv_stream");
+    else if (c.T <= kRowsMaxTokens)
+        e = launch_gemm_rows_tc(c.T, c.d.d_model, c.nr(), xn, w_qkv, qkv, c.st, "qkv_rows_tc");
     else
         e = launch_gemm_down_tc(pd, c.T, xn, offsets, w_qkv, qkv, c.st, "qkv_gemm_tc");
     if (e != cudaSuccess) return e;
     int Hq = c.d.n_heads, Hkv = c.d.n_kv_heads, ns = n_seq, Lv = L;
-    double base = (double)c.d.rope_base;
+    RopeRates rates;
+    for (int i = 0; i < kHeadDim / 2; ++i)
+        rates.w[i] = pow((double)c.d.rope_base, -2.0 * i / (double)kHeadDim);
     const float *qkvc = qkv;
     bf16 *kcp = static_cast<bf16 *>(kc), *vcp = static_cast<bf16 *>(vc);
     unsigned *err = device_info().err;
-    void *args[] = {&Hq, &Hkv, &ns, &Lv, &base, &seq, &pos, &qkvc, &q, &kcp, &vcp, &err};
+    void *args[] = {&Hq, &Hkv, &ns, &Lv, &rates, &seq, &pos, &qkvc, &q, &kcp, &vcp, &err};
     LaunchScope ls("rope_cache", c.st);
-    return launch_pdl((const void *)k_rope_cache, dim3(c.T), dim3(128), 0, c.st, args);
+    return launch_pdl((const void *)k_rope_cache, dim3(Hq + 2 * Hkv, c.T), dim3(kHeadDim / 2), 0,
+                      c.st, args);
 }
 
+// Attention over the caches: per-split partials, then their merge.
 cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const int32_t *pos,
                    int n_seq, int L, const void *kc, const void *vc, void *ctx) {
     const int Hq = c.d.n_heads, Hkv = c.d.n_kv_heads, G = Hq / Hkv;
-    int ns = n_split_for(c.T, Hkv);
+    int ns = n_split_for(c.T, Hkv, L);
     float *ml = at<float>(c.ws, c.L.part_ml), *acc = at<float>(c.ws, c.L.part_acc);
     const void *kern = nullptr;
     switch (G) {
@@ -423,7 +478,7 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     const bf16 *kcp = static_cast<const bf16 *>(kc), *vcp = static_cast<const bf16 *>(vc);
     {
         void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &seq, &pos, &q, &kcp, &vcp, &ml, &acc};
-        LaunchScope ls("attn_partial", c.st);
+        LaunchScope ls("attention", c.st);
         cudaError_t e = launch_pdl(kern, dim3(ns, c.T * Hkv), dim3(kAttnThreads), 0, c.st, args);
         if (e != cudaSuccess) return e;
     }
@@ -431,7 +486,8 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     bf16 *cp = static_cast<bf16 *>(ctx);
     void *args[] = {&ns, &mlc, &accc, &cp};
     LaunchScope ls("attn_merge", c.st);
-    return launch_pdl((const void *)k_attn_merge, dim3(c.T * Hq), dim3(kHeadDim), 0, c.st, args);
+    return launch_pdl((const void *)k_attn_merge, dim3(c.T * Hq), dim3(kHeadDim * kMergeGroups), 0,
+                      c.st, args);
 }
 
 // resid += W_o . ctx
@@ -444,7 +500,10 @@ cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *r
         return launch_down_stream(pd, 1, ctx, offsets, ident, w_o, ones, resid, resid, nullptr,
                                   true, c.st, "o_stream");
     float *y = at<float>(c.ws, c.L.qkv);
-    cudaError_t e = launch_gemm_down_tc(pd, c.T, ctx, offsets, w_o, y, c.st, "o_gemm_tc");
+    cudaError_t e = c.T <= kRowsMaxTokens
+                        ? launch_gemm_rows_tc(c.T, c.nq(), c.d.d_model, ctx, w_o, y, c.st,
+                                              "o_rows_tc")
+                        : launch_gemm_down_tc(pd, c.T, ctx, offsets, w_o, y, c.st, "o_gemm_tc");
     if (e != cudaSuccess) return e;
     long long n4 = (long long)c.T * c.d.d_model / 4;
     const long long cap = (long long)device_info().sm_count * 8;
@@ -543,7 +602,7 @@ moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq
         float *ones = at<float>(ws, c.L.ones);
         void *args[] = {&Tv, &D, &rc, &xn, &eps, &off, &id, &ones};
         LaunchScope ls("sa_prenorm", c.st);
-        if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(256), 0, c.st, args) !=
+        if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(kNormThreads), 0, c.st, args) !=
             cudaSuccess)
             return MOE_ERR_CUDA;
     }

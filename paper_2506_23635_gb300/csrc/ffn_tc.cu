@@ -46,6 +46,7 @@ constexpr int kMaxStages = 8;
 constexpr int kThreadsTc = 192;
 constexpr uint32_t kStageA = BM * BK * 2;  // 16 KB
 constexpr size_t kTcHeaderBytes = 2048;
+constexpr int kMaxSwapStages = 12;
 
 enum Mode { kUp = 0, kDown = 1 };
 
@@ -369,6 +370,154 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
 }
 
+// ---- one weight matrix against a few token rows (weights as the M operand) -------
+//
+// y[j, n] = x[j, :] . W[n, :] for j < T <= 64 tokens and the Nw rows of one
+// matrix W [Nw, Kdim].  A decode batch fills at most 64 of the 128 slot rows
+// of the MMA above, and a single matrix has few 256-row tiles; here the
+// weights are the A operand instead (128 rows per tile, one tile per CTA)
+// and the tokens the B operand (NTOK = T rounded up to 16 columns), so every
+// stage is 16 KB of weights plus NTOK x 128 B of tokens and up to 12 stages
+// stay in flight.  The weight loads of the first stages are issued before the
+// kernel waits for the previous grid (weights do not depend on it).
+template <int NTOK>
+struct SwapCfg {
+    static constexpr uint32_t kStageW = BM * BK * 2;     // 16 KB of weights
+    static constexpr uint32_t kStageX = NTOK * BK * 2;   // token rows
+    static constexpr uint32_t kStageBytes = kStageW + kStageX;
+    static constexpr int kStages =
+        (int)((227 * 1024 - 1024 - kTcHeaderBytes) / kStageBytes) < 12
+            ? (int)((227 * 1024 - 1024 - kTcHeaderBytes) / kStageBytes)
+            : 12;
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kTcHeaderBytes;
+    static constexpr uint32_t kTmemCols = 64;
+    // kind::f16: bf16 A and B, fp32 D, both K-major, N = NTOK, M = 128
+    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                                       ((uint32_t)(NTOK >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    static_assert(NTOK % 16 == 0 && NTOK >= 16 && NTOK <= 64, "token columns");
+    static_assert(kStageBytes % 1024 == 0, "stages stay 1024-byte aligned");
+    static_assert(kStages >= 4 && kStages <= kMaxSwapStages, "stages");
+    static_assert(kSmem <= 227 * 1024, "shared memory");
+};
+
+struct SwapHeader {
+    uint64_t full[kMaxSwapStages];
+    uint64_t empty[kMaxSwapStages];
+    uint64_t tfull;
+    uint32_t tmem_base;
+};
+static_assert(sizeof(SwapHeader) <= kTcHeaderBytes, "swap kernel header too large");
+
+template <int NTOK>
+__global__ void __launch_bounds__(kThreadsTc, 1)
+k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+            int T, int Kdim, int Nw, float *__restrict__ y_out, unsigned *err) {
+    using C = SwapCfg<NTOK>;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    constexpr int kStages = C::kStages;
+    SwapHeader *hd = reinterpret_cast<SwapHeader *>(smem + kStages * C::kStageBytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nk = (Kdim + BK - 1) / BK;
+    const int n0 = blockIdx.x * BM;  // first weight row of this CTA's tile
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&hd->full[s], 1);
+            ptx::mbar_init(&hd->empty[s], 1);
+        }
+        ptx::mbar_init(&hd->tfull, 1);
+        ptx::fence_barrier_init();
+        ptx::prefetch_tmap(&tmW);
+        ptx::prefetch_tmap(&tmX);
+    }
+    if (warp == 1) tmem_alloc(&hd->tmem_base, C::kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = hd->tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            const uint64_t pol_w = ptx::policy_evict_first();
+            const uint64_t pol_x = ptx::policy_evict_last();
+            const int early = nk < kStages ? nk : kStages;
+            // weights of the first stages: independent of earlier kernels
+            for (int kb = 0; kb < early; ++kb) {
+                ptx::mbar_arrive_expect_tx(&hd->full[kb], C::kStageBytes);
+                ptx::tma_load_2d(smem + kb * C::kStageBytes, &tmW, kb * BK, n0, &hd->full[kb],
+                                 pol_w);
+            }
+            ptx::grid_dependency_wait();  // the token rows come from the previous kernel
+            for (int kb = 0; kb < early; ++kb)
+                ptx::tma_load_2d(smem + kb * C::kStageBytes + C::kStageW, &tmX, kb * BK, 0,
+                                 &hd->full[kb], pol_x);
+            int issued = early;
+            for (int kb = early; kb < nk; ++kb) {
+                const uint32_t s = kb % kStages, ph = (kb / kStages) & 1;
+                if (!ptx::mbar_wait(&hd->empty[s], ph ^ 1, err)) break;
+                unsigned char *st = smem + s * C::kStageBytes;
+                ptx::mbar_arrive_expect_tx(&hd->full[s], C::kStageBytes);
+                ptx::tma_load_2d(st, &tmW, kb * BK, n0, &hd->full[s], pol_w);
+                ptx::tma_load_2d(st + C::kStageW, &tmX, kb * BK, 0, &hd->full[s], pol_x);
+                issued = kb + 1;
+            }
+            // let loads still in flight land before the block can exit
+            for (int k = (issued > kStages ? issued - kStages : 0); k < issued; ++k)
+                ptx::mbar_wait(&hd->full[k % kStages], (k / kStages) & 1, err);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            bool ok = true;
+            for (int kb = 0; kb < nk; ++kb) {
+                const uint32_t s = kb % kStages, ph = (kb / kStages) & 1;
+                if (!(ok = ptx::mbar_wait(&hd->full[s], ph, err))) break;
+                tc_fence_after();
+                const uint32_t sa = ptx::smem_u32(smem + s * C::kStageBytes);
+                const uint64_t adesc = smem_desc(sa), bdesc = smem_desc(sa + C::kStageW);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    mma_bf16(tmem, adesc + 2 * kk, bdesc + 2 * kk, C::kIdesc,
+                             (kb | kk) != 0 ? 1u : 0u);
+                mma_commit(&hd->empty[s]);
+            }
+            // tfull flips once every MMA issued here has completed; wait for it
+            // here too, so tensor memory is never freed under a running MMA
+            mma_commit(&hd->tfull);
+            (void)ok;
+            ptx::mbar_wait(&hd->tfull, 0, err);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        ptx::grid_dependency_wait();
+        const int q = warp & 3;
+        const int n = n0 + q * 32 + lane;  // weight row = output column
+        if (ptx::mbar_wait(&hd->tfull, 0, err)) {
+            tc_fence_after();
+            const uint32_t base = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < NTOK; c += 32) {
+                float v[32];
+                tmem_ld32(base + c, v);
+                tmem_ld_wait();
+                if (n < Nw) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (c + j < NTOK && c + j < T) y_out[(size_t)(c + j) * Nw + n] = v[j];
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, C::kTmemCols);
+}
+
 // ---- gather of the A operand: x_sorted[j, :] = x[perm[j] / K, :] ----------------
 
 __global__ void __launch_bounds__(256)
@@ -451,6 +600,21 @@ uint32_t a_box_rows(int T) {
     return (uint32_t)((T + 15) / 16 * 16);
 }
 
+template <int NTOK>
+cudaError_t launch_swap(const CUtensorMap &w, const CUtensorMap &x, int T, int Kdim, int Nw,
+                        float *y, cudaStream_t st, const char *name) {
+    using C = SwapCfg<NTOK>;
+    const void *kern = (const void *)k_gemm_swap<NTOK>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)C::kSmem);
+    if (e != cudaSuccess) return e;
+    unsigned *err = device_info().err;
+    CUtensorMap mw = w, mx = x;
+    void *args[] = {&mw, &mx, &T, &Kdim, &Nw, &y, &err};
+    LaunchScope ls(name ? name : "gemm_rows_tc", st);
+    return launch_pdl(kern, dim3((Nw + BM - 1) / BM), dim3(kThreadsTc), C::kSmem, st, args);
+}
+
 }  // namespace
 
 bool tc_path_ok(const moe_dims &d) {
@@ -496,6 +660,20 @@ cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const i
         return cudaErrorInvalidValue;
     return launch_gemm<kDown, DownWide>(a, b0, b0, offsets, E, S, F, D, arows * BK * 2, nullptr,
                                         y_sorted, st, name);
+}
+
+cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, float *y,
+                                cudaStream_t st, const char *name) {
+    if (T < 1 || T > kRowsMaxTokens) return cudaErrorInvalidValue;
+    const int ntok = (T + 15) / 16 * 16;
+    const uint32_t xrows = ntok <= 16 ? 16 : ntok <= 32 ? 32 : 64;
+    CUtensorMap mw, mx;
+    if (!make_map(&mw, w, (uint64_t)Nw, (uint64_t)Kdim, BM) ||
+        !make_map(&mx, x, (uint64_t)T, (uint64_t)Kdim, xrows))
+        return cudaErrorInvalidValue;
+    if (xrows == 16) return launch_swap<16>(mw, mx, T, Kdim, Nw, y, st, name);
+    if (xrows == 32) return launch_swap<32>(mw, mx, T, Kdim, Nw, y, st, name);
+    return launch_swap<64>(mw, mx, T, Kdim, Nw, y, st, name);
 }
 
 }  // namespace moe

@@ -200,6 +200,11 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
 cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
                               const int32_t *offsets, const void *w1, const void *v1, void *h,
                               cudaStream_t st);
+// One bf16 weight matrix w [Nw, Kdim] against T <= kRowsMaxTokens token rows
+// x [T, Kdim]: y [T, Nw] = x . w^T in fp32, weights as the MMA's M operand.
+constexpr int kRowsMaxTokens = 64;
+cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, float *y,
+                                cudaStream_t st, const char *name = nullptr);
 // name: the profiling name of the launch (default "gemm_down_tc").
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
