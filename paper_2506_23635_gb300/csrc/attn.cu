@@ -11,12 +11,12 @@
 // Kernels, in launch order:
 //   k_sa_prenorm   RMSNorm0 of the fp32 residual -> bf16 rows; block 0 also
 //                  writes the trivial dispatch of a one-"expert" projection
-//                  (offsets {0, T}, identity permutation, unit gates), so the
-//                  two projections run on the MoE layer's own projection
-//                  kernels with E = K = 1;
-//   projection     W_qkv . x: the row-streaming kernel for one token, the
-//                  tcgen05 kernel with the weights as the M operand for up to
-//                  64 tokens, the grouped tcgen05 GEMM beyond (fp32 out);
+//                  (offsets {0, T}), for the grouped GEMM of prefill batches;
+//                  it lets the projection launch at once (the projection's
+//                  weight loads do not depend on it);
+//   projection     W_qkv . x: the tcgen05 kernel with the weights as the M
+//                  operand (split reduction) for up to 64 tokens, the grouped
+//                  tcgen05 GEMM with E = 1 beyond (fp32 out);
 //   k_rope_cache   rotary embedding of q and k (angles formed and reduced in
 //                  fp64, evaluated in fp32), k and v written to the cache in
 //                  bf16;
@@ -24,9 +24,8 @@
 //                  group's query heads against its positions, online softmax,
 //                  partial (max, sum, weighted values) per split;
 //   k_attn_merge   merges the splits, ctx in bf16;
-//   projection     W_o . ctx added to the residual (fused into the streaming
-//                  kernel for one token; a tcgen05 kernel + k_residual_add
-//                  otherwise).
+//   projection     W_o . ctx (the same two kernels), its partial sums added to
+//                  the residual by k_residual_add.
 #include <math.h>
 
 #include <algorithm>
@@ -40,9 +39,8 @@ constexpr int kHeadDim = 128;
 constexpr int kMaxGroup = 8;       // query heads per key/value head
 constexpr int kAttnThreads = 128;  // 4 warps
 constexpr int kAttnWarps = kAttnThreads / 32;
-constexpr int kPosInFlight = 8;    // positions a warp loads before using them
-constexpr int kSplitTarget = 304;     // CTAs a decode step's attention aims for at least
-constexpr int kSplitPositions = 128;  // cache positions per split it aims for at most
+constexpr int kSplitTarget = 152;     // CTAs a decode step's attention aims for at least
+constexpr int kSplitPositions = 128;  // cache positions per split (a 32-position tile per warp)
 constexpr int kMaxSplit = 64;
 constexpr int kMaxSplitCtas = 4096;   // bound on T * Hkv * splits (sizes the workspace)
 constexpr int kMaxSaTokens = 65536;
@@ -70,14 +68,8 @@ struct RopeRates {
 
 // ---- kernels --------------------------------------------------------------------
 
-// The trivial dispatch of the one-"expert" projections (offsets {0, T},
-// identity permutation, unit gates).
-__device__ __forceinline__ void write_trivial_dispatch(int T, int32_t *offsets, int32_t *ident,
-                                                       float *ones) {
-    for (int i = threadIdx.x; i < T; i += blockDim.x) {
-        ident[i] = i;
-        ones[i] = 1.f;
-    }
+// The trivial dispatch of a one-"expert" projection: offsets {0, T}.
+__device__ __forceinline__ void write_trivial_dispatch(int T, int32_t *offsets) {
     if (threadIdx.x == 0) {
         offsets[0] = 0;
         offsets[1] = T;
@@ -90,11 +82,14 @@ constexpr int kNormThreads = 1024;
 
 __global__ void __launch_bounds__(kNormThreads)
 k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ xn, float eps,
-             int32_t *offsets, int32_t *ident, float *ones) {
+             int32_t *offsets) {
+    // the projection after this kernel may start now: its weight loads do
+    // not depend on anything here
+    ptx::launch_dependents();
     ptx::grid_dependency_wait();
     __shared__ float red[kNormThreads / 32];
     const int t = blockIdx.x;
-    if (t == 0) write_trivial_dispatch(T, offsets, ident, ones);
+    if (t == 0) write_trivial_dispatch(T, offsets);
     const float4 *r = reinterpret_cast<const float4 *>(resid + (size_t)t * D);
     const int nv = D >> 2;
     float ss = 0.f;
@@ -120,19 +115,21 @@ k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ x
 }
 
 __global__ void __launch_bounds__(256)
-k_sa_setup(int T, int32_t *offsets, int32_t *ident, float *ones) {
+k_sa_setup(int T, int32_t *offsets) {
     ptx::grid_dependency_wait();
-    write_trivial_dispatch(T, offsets, ident, ones);
+    write_trivial_dispatch(T, offsets);
 }
 
-// qkv [T, (Hq + 2 Hkv) 128] fp32 -> q [T, Hq, 128] fp32 (rotated); rotated
-// keys and the values to the caches [n_seq, Hkv, L, 128] in bf16.  One
+// qkv [T, (Hq + 2 Hkv) 128] fp32 (the sum of n_part partial projections
+// part_stride floats apart) -> q [T, Hq, 128] fp32 (rotated); rotated keys
+// and the values to the caches [n_seq, Hkv, L, 128] in bf16.  One
 // 64-thread block per (head row of qkv, token): thread i turns the pair
 // (i, i + 64) of a query or key head, or copies two value elements.
 __global__ void __launch_bounds__(kHeadDim / 2)
 k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *__restrict__ seq,
-             const int32_t *__restrict__ pos, const float *__restrict__ qkv, float *__restrict__ q,
-             bf16 *__restrict__ kc, bf16 *__restrict__ vc, unsigned *err) {
+             const int32_t *__restrict__ pos, const float *__restrict__ qkv, int n_part,
+             long long part_stride, float *__restrict__ q, bf16 *__restrict__ kc,
+             bf16 *__restrict__ vc, unsigned *err) {
     ptx::grid_dependency_wait();
     constexpr int H2 = kHeadDim / 2;
     const int hr = blockIdx.x, t = blockIdx.y, i = threadIdx.x;
@@ -141,7 +138,11 @@ k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *
     if (!ok && hr == 0 && i == 0) set_error(err, kErrIndex);
     const int nq = Hq * kHeadDim, nkv = Hkv * kHeadDim;
     const float *row = qkv + (size_t)t * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
-    const float a = row[i], b = row[i + H2];
+    float a = 0.f, b = 0.f;  // the projection's partial sums, added in order
+    for (int k = 0; k < n_part; ++k) {
+        a += row[k * part_stride + i];
+        b += row[k * part_stride + i + H2];
+    }
     if (hr >= Hq + Hkv) {  // a value head: stored as it is
         if (!ok) return;
         bf16 *vd = vc + (((size_t)sq * Hkv + (hr - Hq - Hkv)) * L + p) * kHeadDim;
@@ -169,16 +170,37 @@ k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *
     }
 }
 
+// 8-byte asynchronous global -> shared copy (per thread) and its group wait.
+__device__ __forceinline__ void cp_async8(void *dst_smem, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(ptx::smem_u32(dst_smem)),
+                 "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void unpack4(uint2 u, float (&o)[4]) {
     unpack_bf16x2(u.x, o[0], o[1]);
     unpack_bf16x2(u.y, o[2], o[3]);
 }
 
-// One CTA per (split s, token t, key/value head g).  Lane l owns dims
-// [4l, 4l+4) of the G query heads of the group; warp w takes positions
-// j0 + w*P + i*(4P) + u (P = kPosInFlight) of the split's range [j0, j1).
-// Partial results per (t, query head, s): max score, sum of exp, and the
-// exp-weighted sum of values, all relative to that max.
+// One CTA per (split s, token t, key/value head g); the split covers cache
+// positions [j0, j1) of token t's sequence.  Each warp takes tiles of 32
+// positions (tile i of warp w starts at j0 + 32*(w + kAttnWarps*i)):
+//   scores: lane l owns position l of the tile and computes the full dot
+//     products with the G query heads (queries pre-scaled in shared memory),
+//     so no cross-lane reduction per position;
+//   softmax: per head, one warp max and one warp sum per tile update the
+//     running (max m, sum l) and rescale the accumulator;
+//   values: lane l owns dims [4l, 4l+4); for each position of the tile the
+//     head weights are broadcast from the owning lane and the value row is
+//     read coalesced.
+// Partial results per (t, query head, s): m, l, and the weighted value sum
+// (relative to m).
 template <int G>
 __global__ void __launch_bounds__(kAttnThreads)
 k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__restrict__ seq,
@@ -186,8 +208,10 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
                const bf16 *__restrict__ kc, const bf16 *__restrict__ vc,
                float *__restrict__ part_ml, float *__restrict__ part_acc) {
     ptx::grid_dependency_wait();
+    __shared__ __align__(16) float qs[G][kHeadDim];
     __shared__ float sm_m[kAttnWarps][G], sm_l[kAttnWarps][G];
     __shared__ float sm_acc[kAttnWarps][G][kHeadDim];
+    __shared__ __align__(16) bf16 vtile[kAttnWarps][32][kHeadDim];  // each warp's value tile
     const int s = blockIdx.x, tg = blockIdx.y;
     const int t = tg / Hkv, g = tg - t * Hkv;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -197,55 +221,90 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
     const int chunk = (n + n_split - 1) / n_split;
     const int j0 = min(n, s * chunk), j1 = min(n, j0 + chunk);
     const float scale = 1.0f / sqrtf((float)kHeadDim);
+    for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x)
+        qs[i / kHeadDim][i % kHeadDim] = q[((size_t)t * Hq + g * G) * kHeadDim + i] * scale;
+    __syncthreads();
 
-    float qv[G][4], m[G], l[G], acc[G][4];
+    float m[G], l[G], acc[G][4];
 #pragma unroll
     for (int h = 0; h < G; ++h) {
-        const float4 v = *reinterpret_cast<const float4 *>(
-            q + ((size_t)t * Hq + g * G + h) * kHeadDim + lane * 4);
-        qv[h][0] = v.x * scale;
-        qv[h][1] = v.y * scale;
-        qv[h][2] = v.z * scale;
-        qv[h][3] = v.w * scale;
         m[h] = -INFINITY;
         l[h] = 0.f;
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[h][i] = 0.f;
     }
     const size_t base = ok ? ((size_t)sq * Hkv + g) * L * kHeadDim : 0;
-    const bf16 *kb = kc + base + lane * 4;
-    const bf16 *vb = vc + base + lane * 4;
-    constexpr int P = kPosInFlight;
-    for (int j = j0 + warp * P; j < j1; j += kAttnWarps * P) {
-        uint2 kr[P], vr[P];
+    const bf16 *kb = kc + base;
+    const bf16 *vb = vc + base;
+    for (int jt = j0 + warp * 32; jt < j1; jt += kAttnWarps * 32) {
+        const int jl = jt + lane;  // this lane's position
+        const bool live = jl < j1;
+        const int nt = min(32, j1 - jt);
+        // the tile's value rows land in shared memory while the scores are
+        // computed: lane l copies bytes [8l, 8l+8) of every row
+        __syncwarp();
+        for (int u = 0; u < nt; ++u)
+            cp_async8(&vtile[warp][u][lane * 4], vb + (size_t)(jt + u) * kHeadDim + lane * 4);
+        cp_async_commit();
+        float sc[G];
 #pragma unroll
-        for (int u = 0; u < P; ++u) {
-            if (j + u < j1) {
-                kr[u] = __ldg(reinterpret_cast<const uint2 *>(kb + (size_t)(j + u) * kHeadDim));
-                vr[u] = __ldg(reinterpret_cast<const uint2 *>(vb + (size_t)(j + u) * kHeadDim));
+        for (int h = 0; h < G; ++h) sc[h] = 0.f;
+        if (live) {
+            const uint4 *kr = reinterpret_cast<const uint4 *>(kb + (size_t)jl * kHeadDim);
+#pragma unroll
+            for (int c = 0; c < kHeadDim / 32; ++c) {  // 32 dims per step
+                uint4 u[4];
+#pragma unroll
+                for (int v = 0; v < 4; ++v) u[v] = __ldg(kr + c * 4 + v);
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    float k8[8];
+                    unpack_bf16x2(u[v].x, k8[0], k8[1]);
+                    unpack_bf16x2(u[v].y, k8[2], k8[3]);
+                    unpack_bf16x2(u[v].z, k8[4], k8[5]);
+                    unpack_bf16x2(u[v].w, k8[6], k8[7]);
+                    const int d0 = c * 32 + v * 8;
+#pragma unroll
+                    for (int h = 0; h < G; ++h) {
+                        const float4 qa = *reinterpret_cast<const float4 *>(&qs[h][d0]);
+                        const float4 qb = *reinterpret_cast<const float4 *>(&qs[h][d0 + 4]);
+                        sc[h] = fmaf(qa.x, k8[0], sc[h]);
+                        sc[h] = fmaf(qa.y, k8[1], sc[h]);
+                        sc[h] = fmaf(qa.z, k8[2], sc[h]);
+                        sc[h] = fmaf(qa.w, k8[3], sc[h]);
+                        sc[h] = fmaf(qb.x, k8[4], sc[h]);
+                        sc[h] = fmaf(qb.y, k8[5], sc[h]);
+                        sc[h] = fmaf(qb.z, k8[6], sc[h]);
+                        sc[h] = fmaf(qb.w, k8[7], sc[h]);
+                    }
+                }
             }
         }
+        float w[G];
 #pragma unroll
-        for (int u = 0; u < P; ++u) {
-            if (j + u >= j1) break;
-            float k4[4], v4[4];
-            unpack4(kr[u], k4);
-            unpack4(vr[u], v4);
-            float sc[G];
+        for (int h = 0; h < G; ++h) {
+            float tm = live ? sc[h] : -INFINITY;
 #pragma unroll
-            for (int h = 0; h < G; ++h)
-                sc[h] = qv[h][0] * k4[0] + qv[h][1] * k4[1] + qv[h][2] * k4[2] + qv[h][3] * k4[3];
+            for (int o = 16; o > 0; o >>= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, o));
+            const float mn = fmaxf(m[h], tm);  // finite: the tile has a live lane
+            const float corr = expf(m[h] - mn);  // 0 while m is -inf
+            w[h] = live ? expf(sc[h] - mn) : 0.f;
+            l[h] = l[h] * corr + warp_sum(w[h]);
 #pragma unroll
-            for (int h = 0; h < G; ++h) sc[h] = warp_sum(sc[h]);
+            for (int i = 0; i < 4; ++i) acc[h][i] *= corr;
+            m[h] = mn;
+        }
+        cp_async_wait_all();
+        __syncwarp();
+#pragma unroll 4
+        for (int u = 0; u < nt; ++u) {
+            float v4[4];
+            unpack4(*reinterpret_cast<const uint2 *>(&vtile[warp][u][lane * 4]), v4);
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                const float mn = fmaxf(m[h], sc[h]);
-                const float corr = expf(m[h] - mn);  // 0 while m is -inf
-                const float w = expf(sc[h] - mn);
-                l[h] = l[h] * corr + w;
+                const float wu = __shfl_sync(0xffffffffu, w[h], u);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) acc[h][i] = fmaf(w, v4[i], acc[h][i] * corr);
-                m[h] = mn;
+                for (int i = 0; i < 4; ++i) acc[h][i] = fmaf(wu, v4[i], acc[h][i]);
             }
         }
     }
@@ -294,6 +353,7 @@ __global__ void __launch_bounds__(kHeadDim * kMergeGroups)
 k_attn_merge(int n_split, const float *__restrict__ part_ml, const float *__restrict__ part_acc,
              bf16 *__restrict__ ctx) {
     static_assert(kMaxSplit <= kHeadDim * kMergeGroups, "one thread per split");
+    ptx::launch_dependents();  // the output projection may start streaming its weights
     ptx::grid_dependency_wait();
     __shared__ float sm[kMaxSplit], sl[kMaxSplit], sc[kMaxSplit];
     __shared__ float sa[kMergeGroups][kHeadDim], sls[kMergeGroups][kHeadDim];
@@ -327,15 +387,24 @@ k_attn_merge(int n_split, const float *__restrict__ part_ml, const float *__rest
     ctx[(size_t)th * kHeadDim + d] = __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
 }
 
+// resid += y_0 + ... + y_{n_part-1} (partial projections n4 float4 apart,
+// added in order before the residual).
 __global__ void __launch_bounds__(256)
-k_residual_add(long long n4, float *__restrict__ resid, const float *__restrict__ y) {
+k_residual_add(long long n4, int n_part, float *__restrict__ resid, const float *__restrict__ y) {
     ptx::grid_dependency_wait();
     float4 *r = reinterpret_cast<float4 *>(resid);
     const float4 *a = reinterpret_cast<const float4 *>(y);
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
          i += (long long)gridDim.x * blockDim.x) {
+        float4 w = a[i];
+        for (int k = 1; k < n_part; ++k) {
+            const float4 u = a[k * n4 + i];
+            w.x += u.x;
+            w.y += u.y;
+            w.z += u.z;
+            w.w += u.w;
+        }
         float4 v = r[i];
-        const float4 w = a[i];
         v.x += w.x;
         v.y += w.y;
         v.z += w.z;
@@ -347,25 +416,25 @@ k_residual_add(long long n4, float *__restrict__ resid, const float *__restrict_
 // ---- host ------------------------------------------------------------------------
 
 struct SaWs {
-    size_t offsets, ident, ones, xn, qkv, q, part_ml, part_acc, ctx, total;
+    size_t offsets, xn, qkv, q, part_ml, part_acc, ctx, total;
 };
 
 SaWs sa_ws(const moe_sa_dims &d, int64_t T) {
     auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
     const size_t nq = (size_t)d.n_heads * kHeadDim;
     const size_t nr = nq + 2 * (size_t)d.n_kv_heads * kHeadDim;
-    const size_t parts = (size_t)T * d.n_heads * split_cap((int)T, d.n_kv_heads);
+    const size_t splits = (size_t)T * d.n_heads * split_cap((int)T, d.n_kv_heads);
     SaWs L{};
     size_t o = 0;
     L.offsets = o; o += up(2 * 4);
-    L.ident = o; o += up((size_t)T * 4);
-    L.ones = o; o += up((size_t)T * 4);
     L.xn = o; o += up((size_t)T * d.d_model * 2);
-    // projection outputs: qkv first, later the output projection's rows
-    L.qkv = o; o += up((size_t)T * std::max(nr, (size_t)d.d_model) * 4);
+    // projection outputs (partial sums of a split reduction for up to
+    // kRowsMaxTokens tokens): qkv first, later the output projection's rows
+    const size_t parts = T <= kRowsMaxTokens ? kRowsMaxParts : 1;
+    L.qkv = o; o += up(parts * T * std::max(nr, (size_t)d.d_model) * 4);
     L.q = o; o += up((size_t)T * nq * 4);
-    L.part_ml = o; o += up(parts * 2 * 4);
-    L.part_acc = o; o += up(parts * kHeadDim * 4);
+    L.part_ml = o; o += up(splits * 2 * 4);
+    L.part_acc = o; o += up(splits * kHeadDim * 4);
     L.ctx = o; o += up((size_t)T * nq * 2);
     L.total = o;
     return L;
@@ -422,10 +491,6 @@ struct SaCall {
     SaWs L;
     int nq() const { return d.n_heads * kHeadDim; }
     int nr() const { return (d.n_heads + 2 * d.n_kv_heads) * kHeadDim; }
-    bool streamed() const {
-        return T == 1 && stream_path_ok(proj_dims(nr(), d.d_model), 1) &&
-               stream_path_ok(proj_dims(d.d_model, nq()), 1);
-    }
 };
 
 // W_qkv . xn -> qkv (fp32), then the rotary embedding and the cache writes.
@@ -435,15 +500,16 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
     const int32_t *offsets = at<int32_t>(c.ws, c.L.offsets);
     float *qkv = at<float>(c.ws, c.L.qkv);
     cudaError_t e;
-    if (c.streamed())
-        e = launch_down_stream(pd, 1, xn, offsets, at<int32_t>(c.ws, c.L.ident), w_qkv,
-                               at<float>(c.ws, c.L.ones), nullptr, nullptr, qkv, false, c.st,
-                               "qkv_stream");
-    else if (c.T <= kRowsMaxTokens)
-        e = launch_gemm_rows_tc(c.T, c.d.d_model, c.nr(), xn, w_qkv, qkv, c.st, "qkv_rows_tc");
-    else
+    int n_part = 1;
+    if (c.T <= kRowsMaxTokens) {
+        n_part = gemm_rows_parts(c.d.d_model, c.nr());
+        e = launch_gemm_rows_tc(c.T, c.d.d_model, c.nr(), xn, w_qkv, n_part, qkv, c.st,
+                                "qkv_rows_tc");
+    } else {
         e = launch_gemm_down_tc(pd, c.T, xn, offsets, w_qkv, qkv, c.st, "qkv_gemm_tc");
+    }
     if (e != cudaSuccess) return e;
+    long long pstride = (long long)c.T * c.nr();
     int Hq = c.d.n_heads, Hkv = c.d.n_kv_heads, ns = n_seq, Lv = L;
     RopeRates rates;
     for (int i = 0; i < kHeadDim / 2; ++i)
@@ -451,7 +517,8 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
     const float *qkvc = qkv;
     bf16 *kcp = static_cast<bf16 *>(kc), *vcp = static_cast<bf16 *>(vc);
     unsigned *err = device_info().err;
-    void *args[] = {&Hq, &Hkv, &ns, &Lv, &rates, &seq, &pos, &qkvc, &q, &kcp, &vcp, &err};
+    void *args[] = {&Hq,  &Hkv, &ns,  &Lv,  &rates, &seq, &pos,
+                    &qkvc, &n_part, &pstride, &q, &kcp, &vcp, &err};
     LaunchScope ls("rope_cache", c.st);
     return launch_pdl((const void *)k_rope_cache, dim3(Hq + 2 * Hkv, c.T), dim3(kHeadDim / 2), 0,
                       c.st, args);
@@ -494,22 +561,21 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
 cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *resid) {
     const moe_dims pd = proj_dims(c.d.d_model, c.nq());
     const int32_t *offsets = at<int32_t>(c.ws, c.L.offsets);
-    const int32_t *ident = at<int32_t>(c.ws, c.L.ident);
-    const float *ones = at<float>(c.ws, c.L.ones);
-    if (c.streamed())  // the residual element is read before the same thread writes it
-        return launch_down_stream(pd, 1, ctx, offsets, ident, w_o, ones, resid, resid, nullptr,
-                                  true, c.st, "o_stream");
     float *y = at<float>(c.ws, c.L.qkv);
-    cudaError_t e = c.T <= kRowsMaxTokens
-                        ? launch_gemm_rows_tc(c.T, c.nq(), c.d.d_model, ctx, w_o, y, c.st,
-                                              "o_rows_tc")
-                        : launch_gemm_down_tc(pd, c.T, ctx, offsets, w_o, y, c.st, "o_gemm_tc");
+    int n_part = 1;
+    cudaError_t e;
+    if (c.T <= kRowsMaxTokens) {
+        n_part = gemm_rows_parts(c.nq(), c.d.d_model);
+        e = launch_gemm_rows_tc(c.T, c.nq(), c.d.d_model, ctx, w_o, n_part, y, c.st, "o_rows_tc");
+    } else {
+        e = launch_gemm_down_tc(pd, c.T, ctx, offsets, w_o, y, c.st, "o_gemm_tc");
+    }
     if (e != cudaSuccess) return e;
     long long n4 = (long long)c.T * c.d.d_model / 4;
     const long long cap = (long long)device_info().sm_count * 8;
     const int grid = (int)std::max(1LL, std::min((n4 + 255) / 256, cap));
     const float *yc = y;
-    void *args[] = {&n4, &resid, &yc};
+    void *args[] = {&n4, &n_part, &resid, &yc};
     LaunchScope ls("residual_add", c.st);
     return launch_pdl((const void *)k_residual_add, dim3(grid), dim3(256), 0, c.st, args);
 }
@@ -522,9 +588,8 @@ moe_status check_ws(const moe_sa_dims *d, int T, void *ws, size_t ws_bytes) {
 
 moe_status setup_dispatch(const SaCall &c) {
     int Tv = c.T;
-    int32_t *off = at<int32_t>(c.ws, c.L.offsets), *id = at<int32_t>(c.ws, c.L.ident);
-    float *ones = at<float>(c.ws, c.L.ones);
-    void *args[] = {&Tv, &off, &id, &ones};
+    int32_t *off = at<int32_t>(c.ws, c.L.offsets);
+    void *args[] = {&Tv, &off};
     LaunchScope ls("sa_setup", c.st);
     return cuda_status(launch_pdl((const void *)k_sa_setup, dim3(1), dim3(256), 0, c.st, args));
 }
@@ -556,7 +621,7 @@ moe_status moe_sa_qkv(const moe_sa_dims *dims, int32_t T, const void *x_norm, co
         return MOE_ERR_INVALID_ARG;
     if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
     SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
-    if (!c.streamed() && !tc_path_ok(proj_dims(c.nr(), dims->d_model))) return MOE_ERR_UNSUPPORTED;
+    if (!tc_path_ok(proj_dims(c.nr(), dims->d_model))) return MOE_ERR_UNSUPPORTED;
     if ((s = setup_dispatch(c)) != MOE_OK) return s;
     return cuda_status(qkv_rope(c, x_norm, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache));
 }
@@ -589,8 +654,8 @@ moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq
         return MOE_ERR_INVALID_ARG;
     if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
     SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
-    if (!c.streamed() && (!tc_path_ok(proj_dims(c.nr(), dims->d_model)) ||
-                          !tc_path_ok(proj_dims(dims->d_model, c.nq()))))
+    if (!tc_path_ok(proj_dims(c.nr(), dims->d_model)) ||
+        !tc_path_ok(proj_dims(dims->d_model, c.nq())))
         return MOE_ERR_UNSUPPORTED;
     bf16 *xn = at<bf16>(ws, c.L.xn);
     float *q = at<float>(ws, c.L.q);
@@ -598,9 +663,8 @@ moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq
     {
         int Tv = T, D = dims->d_model;
         const float *rc = resid;
-        int32_t *off = at<int32_t>(ws, c.L.offsets), *id = at<int32_t>(ws, c.L.ident);
-        float *ones = at<float>(ws, c.L.ones);
-        void *args[] = {&Tv, &D, &rc, &xn, &eps, &off, &id, &ones};
+        int32_t *off = at<int32_t>(ws, c.L.offsets);
+        void *args[] = {&Tv, &D, &rc, &xn, &eps, &off};
         LaunchScope ls("sa_prenorm", c.st);
         if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(kNormThreads), 0, c.st, args) !=
             cudaSuccess)

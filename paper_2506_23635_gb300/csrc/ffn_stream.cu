@@ -408,8 +408,7 @@ cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const 
 template <typename TO, typename TR, bool FUSED>
 cudaError_t down_stream_impl(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                              const int32_t *inv_perm, const void *w2, const float *gate,
-                             const void *residual, void *out, float *y_sorted, cudaStream_t st,
-                             const char *name) {
+                             const void *residual, void *out, float *y_sorted, cudaStream_t st) {
     const int grid = std::min(device_info().sm_count, d.d_model);
     DownPlan p;
     if (!plan_down(d, T, grid, p)) return cudaErrorInvalidValue;
@@ -426,22 +425,22 @@ cudaError_t down_stream_impl(const moe_dims &d, int T, const void *h, const int3
     unsigned *err = device_info().err;
     void *args[] = {&D, &F, &E, &K, &Tv, &hp, &offsets, &inv_perm, &w2p, &gate, &rp, &op,
                     &y_sorted, &ns, &rows_max, &err};
-    LaunchScope ls(name ? name : FUSED ? "down_combine_stream" : "down_stream", st);
+    LaunchScope ls(FUSED ? "down_combine_stream" : "down_stream", st);
     return launch_pdl(kern, dim3(grid), dim3((p.n_stages + 1) * 32), p.smem, st, args);
 }
 
 cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                const int32_t *inv_perm, const void *w2, const float *gate,
                                const void *residual, void *out, float *y_sorted, bool fused,
-                               cudaStream_t st, const char *name) {
+                               cudaStream_t st) {
     if (!fused)
         return down_stream_impl<float, bf16, false>(d, T, h, offsets, inv_perm, w2, gate, nullptr,
-                                                    nullptr, y_sorted, st, name);
+                                                    nullptr, y_sorted, st);
     if (d.out_dtype == MOE_BF16)
         return down_stream_impl<bf16, bf16, true>(d, T, h, offsets, inv_perm, w2, gate, residual,
-                                                  out, nullptr, st, name);
+                                                  out, nullptr, st);
     return down_stream_impl<float, float, true>(d, T, h, offsets, inv_perm, w2, gate, residual, out,
-                                               nullptr, st, name);
+                                               nullptr, st);
 }
 
 }  // namespace moe

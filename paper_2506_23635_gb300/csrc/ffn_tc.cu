@@ -375,11 +375,14 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
 // y[j, n] = x[j, :] . W[n, :] for j < T <= 64 tokens and the Nw rows of one
 // matrix W [Nw, Kdim].  A decode batch fills at most 64 of the 128 slot rows
 // of the MMA above, and a single matrix has few 256-row tiles; here the
-// weights are the A operand instead (128 rows per tile, one tile per CTA)
-// and the tokens the B operand (NTOK = T rounded up to 16 columns), so every
-// stage is 16 KB of weights plus NTOK x 128 B of tokens and up to 12 stages
-// stay in flight.  The weight loads of the first stages are issued before the
-// kernel waits for the previous grid (weights do not depend on it).
+// weights are the A operand instead (128 rows per tile) and the tokens the B
+// operand (NTOK = T rounded up to 16 columns), so every stage is 16 KB of
+// weights plus NTOK x 128 B of tokens and up to 12 stages stay in flight.
+// Loaded HBM latency is ~3.5 us, so streaming at the HBM rate needs ~25 MB in
+// flight: the reduction is split over gridDim.y CTAs per tile (split z writes
+// its partial sums to y_out + z*T*Nw; the caller adds the parts in order).
+// The weight loads of the first stages are issued before the kernel waits
+// for the previous grid (weights do not depend on it).
 template <int NTOK>
 struct SwapCfg {
     static constexpr uint32_t kStageW = BM * BK * 2;     // 16 KB of weights
@@ -419,8 +422,11 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
     constexpr int kStages = C::kStages;
     SwapHeader *hd = reinterpret_cast<SwapHeader *>(smem + kStages * C::kStageBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nk = (Kdim + BK - 1) / BK;
+    const int nk_all = (Kdim + BK - 1) / BK;
+    const int kb0 = (int)((long long)nk_all * blockIdx.y / gridDim.y);
+    const int nk = (int)((long long)nk_all * (blockIdx.y + 1) / gridDim.y) - kb0;
     const int n0 = blockIdx.x * BM;  // first weight row of this CTA's tile
+    y_out += (size_t)blockIdx.y * T * Nw;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -447,12 +453,12 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
             // weights of the first stages: independent of earlier kernels
             for (int kb = 0; kb < early; ++kb) {
                 ptx::mbar_arrive_expect_tx(&hd->full[kb], C::kStageBytes);
-                ptx::tma_load_2d(smem + kb * C::kStageBytes, &tmW, kb * BK, n0, &hd->full[kb],
+                ptx::tma_load_2d(smem + kb * C::kStageBytes, &tmW, (kb0 + kb) * BK, n0, &hd->full[kb],
                                  pol_w);
             }
             ptx::grid_dependency_wait();  // the token rows come from the previous kernel
             for (int kb = 0; kb < early; ++kb)
-                ptx::tma_load_2d(smem + kb * C::kStageBytes + C::kStageW, &tmX, kb * BK, 0,
+                ptx::tma_load_2d(smem + kb * C::kStageBytes + C::kStageW, &tmX, (kb0 + kb) * BK, 0,
                                  &hd->full[kb], pol_x);
             int issued = early;
             for (int kb = early; kb < nk; ++kb) {
@@ -460,8 +466,8 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
                 if (!ptx::mbar_wait(&hd->empty[s], ph ^ 1, err)) break;
                 unsigned char *st = smem + s * C::kStageBytes;
                 ptx::mbar_arrive_expect_tx(&hd->full[s], C::kStageBytes);
-                ptx::tma_load_2d(st, &tmW, kb * BK, n0, &hd->full[s], pol_w);
-                ptx::tma_load_2d(st + C::kStageW, &tmX, kb * BK, 0, &hd->full[s], pol_x);
+                ptx::tma_load_2d(st, &tmW, (kb0 + kb) * BK, n0, &hd->full[s], pol_w);
+                ptx::tma_load_2d(st + C::kStageW, &tmX, (kb0 + kb) * BK, 0, &hd->full[s], pol_x);
                 issued = kb + 1;
             }
             // let loads still in flight land before the block can exit
@@ -496,7 +502,10 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         ptx::grid_dependency_wait();
         const int q = warp & 3;
         const int n = n0 + q * 32 + lane;  // weight row = output column
-        if (ptx::mbar_wait(&hd->tfull, 0, err)) {
+        if (nk <= 0) {  // an empty share of the reduction: its part is zero
+            if (n < Nw)
+                for (int j = 0; j < T; ++j) y_out[(size_t)j * Nw + n] = 0.f;
+        } else if (ptx::mbar_wait(&hd->tfull, 0, err)) {
             tc_fence_after();
             const uint32_t base = tmem + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
@@ -602,7 +611,7 @@ uint32_t a_box_rows(int T) {
 
 template <int NTOK>
 cudaError_t launch_swap(const CUtensorMap &w, const CUtensorMap &x, int T, int Kdim, int Nw,
-                        float *y, cudaStream_t st, const char *name) {
+                        int parts, float *y, cudaStream_t st, const char *name) {
     using C = SwapCfg<NTOK>;
     const void *kern = (const void *)k_gemm_swap<NTOK>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -612,7 +621,8 @@ cudaError_t launch_swap(const CUtensorMap &w, const CUtensorMap &x, int T, int K
     CUtensorMap mw = w, mx = x;
     void *args[] = {&mw, &mx, &T, &Kdim, &Nw, &y, &err};
     LaunchScope ls(name ? name : "gemm_rows_tc", st);
-    return launch_pdl(kern, dim3((Nw + BM - 1) / BM), dim3(kThreadsTc), C::kSmem, st, args);
+    return launch_pdl(kern, dim3((Nw + BM - 1) / BM, parts), dim3(kThreadsTc), C::kSmem, st,
+                      args);
 }
 
 }  // namespace
@@ -662,18 +672,25 @@ cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const i
                                         y_sorted, st, name);
 }
 
-cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, float *y,
-                                cudaStream_t st, const char *name) {
-    if (T < 1 || T > kRowsMaxTokens) return cudaErrorInvalidValue;
+int gemm_rows_parts(int Kdim, int Nw) {
+    const int tiles = (Nw + BM - 1) / BM, nk = (Kdim + BK - 1) / BK;
+    const int by_sms = std::max(1, device_info().sm_count / std::max(1, tiles));
+    return std::max(1, std::min({kRowsMaxParts, by_sms, nk}));
+}
+
+cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, int parts,
+                                float *y, cudaStream_t st, const char *name) {
+    if (T < 1 || T > kRowsMaxTokens || parts < 1 || parts > kRowsMaxParts)
+        return cudaErrorInvalidValue;
     const int ntok = (T + 15) / 16 * 16;
     const uint32_t xrows = ntok <= 16 ? 16 : ntok <= 32 ? 32 : 64;
     CUtensorMap mw, mx;
     if (!make_map(&mw, w, (uint64_t)Nw, (uint64_t)Kdim, BM) ||
         !make_map(&mx, x, (uint64_t)T, (uint64_t)Kdim, xrows))
         return cudaErrorInvalidValue;
-    if (xrows == 16) return launch_swap<16>(mw, mx, T, Kdim, Nw, y, st, name);
-    if (xrows == 32) return launch_swap<32>(mw, mx, T, Kdim, Nw, y, st, name);
-    return launch_swap<64>(mw, mx, T, Kdim, Nw, y, st, name);
+    if (xrows == 16) return launch_swap<16>(mw, mx, T, Kdim, Nw, parts, y, st, name);
+    if (xrows == 32) return launch_swap<32>(mw, mx, T, Kdim, Nw, parts, y, st, name);
+    return launch_swap<64>(mw, mx, T, Kdim, Nw, parts, y, st, name);
 }
 
 }  // namespace moe

@@ -201,10 +201,15 @@ cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
                               const int32_t *offsets, const void *w1, const void *v1, void *h,
                               cudaStream_t st);
 // One bf16 weight matrix w [Nw, Kdim] against T <= kRowsMaxTokens token rows
-// x [T, Kdim]: y [T, Nw] = x . w^T in fp32, weights as the MMA's M operand.
+// x [T, Kdim]: y = x . w^T in fp32, weights as the MMA's M operand, the
+// reduction split into `parts` (<= kRowsMaxParts) shares whose partial sums
+// land in y + p*T*Nw for p < parts (the caller adds them in order).
+// gemm_rows_parts: the split that keeps the SMs streaming for this shape.
 constexpr int kRowsMaxTokens = 64;
-cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, float *y,
-                                cudaStream_t st, const char *name = nullptr);
+constexpr int kRowsMaxParts = 4;
+int gemm_rows_parts(int Kdim, int Nw);
+cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, int parts,
+                                float *y, cudaStream_t st, const char *name = nullptr);
 // name: the profiling name of the launch (default "gemm_down_tc").
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
@@ -219,11 +224,9 @@ bool stream_path_ok(const moe_dims &d, int T);
 cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
                                  const int32_t *offsets, const void *w1, const void *v1, void *h,
                                  cudaStream_t st);
-// name: the profiling name of the launch (default "down_combine_stream" /
-// "down_stream").
 cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                const int32_t *inv_perm, const void *w2, const float *gate,
                                const void *residual, void *out, float *y_sorted, bool fused,
-                               cudaStream_t st, const char *name = nullptr);
+                               cudaStream_t st);
 
 }  // namespace moe
