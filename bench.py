@@ -570,11 +570,12 @@ def sa_bytes(a, T, ctx_len):
             + T * (2 * D * 4 + Hq * dh * 2 + 2 * Hkv * dh * 2))
 
 
-def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5):
+def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5, prefill=False):
     """One DBRX-shaped decoder layer (the self-attention block with D_qkv =
-    8,192 in front of this MoE layer) in decode: T sequences, one new token
+    8,192 in front of this MoE layer).  Decode: T sequences, one new token
     each, at position ctx_len - 1 of a KV cache filled with synthetic earlier
-    entries; fp32 residual stream."""
+    entries.  Prefill: one sequence, positions 0..T-1 (causal).  fp32
+    residual stream."""
     import torch
 
     moe, dev = layer.moe, layer.dev
@@ -584,19 +585,27 @@ def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5):
     d32 = moe.dims(layer.shape.d_model, layer.shape.ffn_hidden, layer.shape.n_experts,
                    layer.shape.top_k, torch.bfloat16, torch.bfloat16, torch.float32)
     w_qkv, w_o = gen.device_attn_weights(a_shape, SEED, dev)
-    kc, vc = gen.device_kv_cache(a_shape, T, ctx_len, SEED, dev)
-    xs_host, w_r_host = token_pool(layer.shape, T, SEED, 16)
+    if prefill:
+        ctx_len = T
+    n_seq = 1 if prefill else T
+    pool = 4 if prefill else 16
+    kc, vc = gen.device_kv_cache(a_shape, n_seq, ctx_len, SEED, dev)
+    xs_host, w_r_host = token_pool(layer.shape, T, SEED, pool)
     w_r = gen.host_to_torch(w_r_host, "bf16", dev)
     xs = gen.host_to_torch(xs_host, "bf16", dev).float()
     w1, v1, w2 = layer.w
     W = moe.DecoderWeights([(w_qkv, w_o, w_r, w1, v1, w2, kc, vc)])
-    seq = torch.arange(T, dtype=torch.int32, device=dev)
-    pos = torch.full((T,), ctx_len - 1, dtype=torch.int32, device=dev)
+    if prefill:
+        seq = torch.zeros(T, dtype=torch.int32, device=dev)
+        pos = torch.arange(T, dtype=torch.int32, device=dev)
+    else:
+        seq = torch.arange(T, dtype=torch.int32, device=dev)
+        pos = torch.full((T,), ctx_len - 1, dtype=torch.int32, device=dev)
     resid = torch.empty((T, layer.shape.d_model), dtype=torch.float32, device=dev)
     ws = torch.empty(moe.decoder_workspace_size(a, d32, T), dtype=torch.uint8, device=dev)
 
     def step(i):
-        resid.copy_(xs[i % 16])
+        resid.copy_(xs[i % pool])
         moe.decoder_forward(a, d32, W, resid, seq, pos, ws=ws, stream=layer.stream)
 
     for i in range(warmup):
@@ -609,6 +618,17 @@ def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5):
     peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
     kv = T * ctx_len * a.n_kv_heads * a.head_dim * 4
     att = kstats.get("attention")
+    if prefill:  # tensor work: projections 2*T*(8192 + 6144)*6144, attention ~2*2*T^2/2*48*128
+        sa_flops = 2.0 * T * (a_shape.qkv_rows + a.d_model) * a.d_model \
+            + 2.0 * T * (T + 1) * a.n_heads * a.head_dim
+        res = {"tokens_per_step": T, "mode": "prefill (one sequence, causal)",
+               "ms_per_step": round(ms, 4), "launches_per_step": launches / steps,
+               "attention_block": {"us_per_step": round(sa_ms * 1e3, 2),
+                                   "tflops": round(sa_flops / (sa_ms / 1e3) / 1e12, 1)},
+               "kernels": kernel_table(kstats)}
+        del W, w_qkv, w_o, kc, vc
+        torch.cuda.empty_cache()
+        return res
     res = {"tokens_per_step": T, "context": ctx_len, "ms_per_step": round(ms, 4),
            "launches_per_step": launches / steps,
            "attention_block": {"us_per_step": round(sa_ms * 1e3, 2),
@@ -753,6 +773,8 @@ def run_ours(args):
                                  for t in (2, 4, 8, 16, 32, 64)]
         extra["busy_full_loading"] = [measure_dense(layer, t) for t in (1, 8)]
         extra["decoder_layer"] = [measure_decoder_layer(layer, t) for t in (1, 8)]
+        extra["decoder_prefill"] = [measure_decoder_layer(layer, t, steps=20, warmup=3,
+                                                          prefill=True) for t in (128, 2048)]
         extra["stack"] = measure_stack(moe, dev)
 
     if rank != 0:

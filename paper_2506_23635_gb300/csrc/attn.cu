@@ -23,7 +23,11 @@
 //   k_attn_partial one CTA per (token, key/value head, position split): the
 //                  group's query heads against its positions, online softmax,
 //                  partial (max, sum, weighted values) per split;
-//   k_attn_merge   merges the splits, ctx in bf16;
+//   k_attn_merge   merges the splits, ctx in bf16 (a single split writes ctx
+//                  itself); in moe_sa_forward, calls of 128 tokens or more
+//                  first run the tensor-core prefill attention (attn_tc.cu)
+//                  on every full 128-token tile of consecutive positions of
+//                  one sequence, and the kernels above only on the rest;
 //   projection     W_o . ctx (the same two kernels), its partial sums added to
 //                  the residual by k_residual_add.
 #include <math.h>
@@ -122,17 +126,21 @@ k_sa_setup(int T, int32_t *offsets) {
 
 // qkv [T, (Hq + 2 Hkv) 128] fp32 (the sum of n_part partial projections
 // part_stride floats apart) -> q [T, Hq, 128] fp32 (rotated); rotated keys
-// and the values to the caches [n_seq, Hkv, L, 128] in bf16.  One
-// 64-thread block per (head row of qkv, token): thread i turns the pair
+// and the values to the caches [n_seq, Hkv, L, 128] in bf16.  A block holds
+// kRopeRows head rows of one token, 64 threads each: thread i turns the pair
 // (i, i + 64) of a query or key head, or copies two value elements.
-__global__ void __launch_bounds__(kHeadDim / 2)
+constexpr int kRopeRows = 4;  // head rows per block
+
+__global__ void __launch_bounds__(kRopeRows * kHeadDim / 2)
 k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *__restrict__ seq,
              const int32_t *__restrict__ pos, const float *__restrict__ qkv, int n_part,
-             long long part_stride, float *__restrict__ q, bf16 *__restrict__ kc,
-             bf16 *__restrict__ vc, unsigned *err) {
+             long long part_stride, float *__restrict__ q, bf16 *__restrict__ q16,
+             bf16 *__restrict__ kc, bf16 *__restrict__ vc, unsigned *err) {
     ptx::grid_dependency_wait();
     constexpr int H2 = kHeadDim / 2;
-    const int hr = blockIdx.x, t = blockIdx.y, i = threadIdx.x;
+    const int hr = blockIdx.x * kRopeRows + threadIdx.x / H2, t = blockIdx.y;
+    const int i = threadIdx.x % H2;
+    if (hr >= Hq + 2 * Hkv) return;
     const int sq = seq[t], p = pos[t];
     const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
     if (!ok && hr == 0 && i == 0) set_error(err, kErrIndex);
@@ -163,6 +171,11 @@ k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *
         float *qo = q + (size_t)t * nq + (size_t)hr * kHeadDim;
         qo[i] = x0;
         qo[i + H2] = x1;
+        if (q16) {  // the tensor-core attention's copy
+            bf16 *qh = q16 + (size_t)t * nq + (size_t)hr * kHeadDim;
+            qh[i] = __float2bfloat16_rn(x0);
+            qh[i + H2] = __float2bfloat16_rn(x1);
+        }
     } else if (ok) {
         bf16 *kd = kc + (((size_t)sq * Hkv + (hr - Hq)) * L + p) * kHeadDim;
         kd[i] = __float2bfloat16_rn(x0);
@@ -206,7 +219,8 @@ __global__ void __launch_bounds__(kAttnThreads)
 k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__restrict__ seq,
                const int32_t *__restrict__ pos, const float *__restrict__ q,
                const bf16 *__restrict__ kc, const bf16 *__restrict__ vc,
-               float *__restrict__ part_ml, float *__restrict__ part_acc) {
+               float *__restrict__ part_ml, float *__restrict__ part_acc,
+               bf16 *__restrict__ ctx, const int *__restrict__ tile_ok) {
     ptx::grid_dependency_wait();
     __shared__ __align__(16) float qs[G][kHeadDim];
     __shared__ float sm_m[kAttnWarps][G], sm_l[kAttnWarps][G];
@@ -214,6 +228,7 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
     __shared__ __align__(16) bf16 vtile[kAttnWarps][32][kHeadDim];  // each warp's value tile
     const int s = blockIdx.x, tg = blockIdx.y;
     const int t = tg / Hkv, g = tg - t * Hkv;
+    if (tile_ok && tile_ok[t / kAttnTcTile]) return;  // the tensor-core kernel has it
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sq = seq[t], p = pos[t];
     const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
@@ -333,6 +348,11 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
                 A = fmaf(sm_acc[w][h][d], c, A);
             }
         }
+        if (n_split == 1) {  // the only split: this is the result
+            ctx[((size_t)t * Hq + g * G + h) * kHeadDim + d] =
+                __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
+            continue;
+        }
         const size_t o = ((size_t)t * Hq + g * G + h) * n_split + s;
         if (d == 0) {
             part_ml[2 * o] = M;
@@ -416,7 +436,7 @@ k_residual_add(long long n4, int n_part, float *__restrict__ resid, const float 
 // ---- host ------------------------------------------------------------------------
 
 struct SaWs {
-    size_t offsets, xn, qkv, q, part_ml, part_acc, ctx, total;
+    size_t offsets, xn, qkv, q, q16, tile_ok, part_ml, part_acc, ctx, total;
 };
 
 SaWs sa_ws(const moe_sa_dims &d, int64_t T) {
@@ -433,6 +453,8 @@ SaWs sa_ws(const moe_sa_dims &d, int64_t T) {
     const size_t parts = T <= kRowsMaxTokens ? kRowsMaxParts : 1;
     L.qkv = o; o += up(parts * T * std::max(nr, (size_t)d.d_model) * 4);
     L.q = o; o += up((size_t)T * nq * 4);
+    L.q16 = o; o += up((size_t)T * nq * 2);
+    L.tile_ok = o; o += up((size_t)(T + kAttnTcTile - 1) / kAttnTcTile * 4);
     L.part_ml = o; o += up(splits * 2 * 4);
     L.part_acc = o; o += up(splits * kHeadDim * 4);
     L.ctx = o; o += up((size_t)T * nq * 2);
@@ -494,8 +516,13 @@ struct SaCall {
 };
 
 // W_qkv . xn -> qkv (fp32), then the rotary embedding and the cache writes.
+// Whether the call's attention takes the tensor-core prefill kernel for its
+// full 128-token tiles (the CUDA-core kernel keeps the others).
+bool tc_attention(int T) { return T >= kAttnTcTile && attn_prefill_tc_ok(); }
+
 cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const int32_t *seq,
-                     const int32_t *pos, int n_seq, int L, float *q, void *kc, void *vc) {
+                     const int32_t *pos, int n_seq, int L, float *q, void *kc, void *vc,
+                     bf16 *q16 = nullptr) {
     const moe_dims pd = proj_dims(c.nr(), c.d.d_model);
     const int32_t *offsets = at<int32_t>(c.ws, c.L.offsets);
     float *qkv = at<float>(c.ws, c.L.qkv);
@@ -517,18 +544,28 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
     const float *qkvc = qkv;
     bf16 *kcp = static_cast<bf16 *>(kc), *vcp = static_cast<bf16 *>(vc);
     unsigned *err = device_info().err;
-    void *args[] = {&Hq,  &Hkv, &ns,  &Lv,  &rates, &seq, &pos,
-                    &qkvc, &n_part, &pstride, &q, &kcp, &vcp, &err};
+    void *args[] = {&Hq,     &Hkv,     &ns, &Lv,  &rates, &seq, &pos, &qkvc,
+                    &n_part, &pstride, &q,  &q16, &kcp,   &vcp,  &err};
     LaunchScope ls("rope_cache", c.st);
-    return launch_pdl((const void *)k_rope_cache, dim3(Hq + 2 * Hkv, c.T), dim3(kHeadDim / 2), 0,
-                      c.st, args);
+    const int rows = Hq + 2 * Hkv;
+    return launch_pdl((const void *)k_rope_cache, dim3((rows + kRopeRows - 1) / kRopeRows, c.T),
+                      dim3(kRopeRows * kHeadDim / 2), 0, c.st, args);
 }
 
 // Attention over the caches: per-split partials, then their merge.
 cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const int32_t *pos,
-                   int n_seq, int L, const void *kc, const void *vc, void *ctx) {
+                   int n_seq, int L, const void *kc, const void *vc, void *ctx,
+                   const bf16 *q16 = nullptr) {
     const int Hq = c.d.n_heads, Hkv = c.d.n_kv_heads, G = Hq / Hkv;
     int ns = n_split_for(c.T, Hkv, L);
+    int *tile_ok = nullptr;
+    if (q16) {  // full prefill tiles on the tensor cores, the rest below (one split)
+        tile_ok = at<int>(c.ws, c.L.tile_ok);
+        cudaError_t e = launch_attn_prefill_tc(c.T, Hq, Hkv, n_seq, L, seq, pos, q16, kc, vc, ctx,
+                                               tile_ok, c.st);
+        if (e != cudaSuccess) return e;
+        ns = 1;
+    }
     float *ml = at<float>(c.ws, c.L.part_ml), *acc = at<float>(c.ws, c.L.part_acc);
     const void *kern = nullptr;
     switch (G) {
@@ -543,14 +580,16 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     }
     int Hqv = Hq, Hkvv = Hkv, nsq = n_seq, Lv = L;
     const bf16 *kcp = static_cast<const bf16 *>(kc), *vcp = static_cast<const bf16 *>(vc);
+    bf16 *cp = static_cast<bf16 *>(ctx);
     {
-        void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &seq, &pos, &q, &kcp, &vcp, &ml, &acc};
+        const int *tok = tile_ok;
+        void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &seq, &pos, &q, &kcp, &vcp, &ml, &acc, &cp,
+                        &tok};
         LaunchScope ls("attention", c.st);
         cudaError_t e = launch_pdl(kern, dim3(ns, c.T * Hkv), dim3(kAttnThreads), 0, c.st, args);
-        if (e != cudaSuccess) return e;
+        if (e != cudaSuccess || ns == 1) return e;
     }
     const float *mlc = ml, *accc = acc;
-    bf16 *cp = static_cast<bf16 *>(ctx);
     void *args[] = {&ns, &mlc, &accc, &cp};
     LaunchScope ls("attn_merge", c.st);
     return launch_pdl((const void *)k_attn_merge, dim3(c.T * Hq), dim3(kHeadDim * kMergeGroups), 0,
@@ -670,8 +709,9 @@ moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq
             cudaSuccess)
             return MOE_ERR_CUDA;
     }
-    cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache);
-    if (e == cudaSuccess) e = attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx);
+    bf16 *q16 = tc_attention(T) ? at<bf16>(ws, c.L.q16) : nullptr;
+    cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache, q16);
+    if (e == cudaSuccess) e = attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx, q16);
     if (e == cudaSuccess) e = out_proj(c, ctx, w_o, resid);
     return cuda_status(e);
 }

@@ -36,10 +36,12 @@
 
 #include <mutex>
 
-#include "ptx.cuh"
+#include "tc.cuh"
 
 namespace moe {
 namespace {
+
+using namespace tc;
 
 constexpr int BM = 128, BK = 64;
 constexpr int kMaxStages = 8;
@@ -82,76 +84,6 @@ struct TcHeader {
     int tprefix[257];  // tile prefix over experts
 };
 static_assert(sizeof(TcHeader) <= kTcHeaderBytes, "tcgen05 kernel header too large");
-
-// ---- tcgen05 wrappers --------------------------------------------------------
-
-__device__ __forceinline__ void tmem_alloc(uint32_t *holder, uint32_t cols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     ptx::smem_u32(holder)),
-                 "r"(cols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols)
-                 : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// D[tmem] (+)= A[smem] * B[smem]^T, both K-major, one instruction of K=16.
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                         uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-// Arrive on an mbarrier once all earlier tcgen05 ops of this thread finish.
-__device__ __forceinline__ void mma_commit(uint64_t *bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-            ptx::smem_u32(bar))
-        : "memory");
-}
-
-// 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31])
-        : "r"(taddr)
-        : "memory");
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void tmem_ld_wait() {
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-// Shared-memory matrix descriptor: K-major operand written by TMA with the
-// 128-byte swizzle; 8-row groups 1024 bytes apart; descriptor version 1.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
-           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
 
 // ---- tile schedule -------------------------------------------------------------
 
@@ -372,12 +304,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
 
 // ---- one weight matrix against a few token rows (weights as the M operand) -------
 //
-// y[j, n] = x[j, :] . W[n, :] for j < T <= 64 tokens and the Nw rows of one
-// matrix W [Nw, Kdim].  A decode batch fills at most 64 of the 128 slot rows
-// of the MMA above, and a single matrix has few 256-row tiles; here the
-// weights are the A operand instead (128 rows per tile) and the tokens the B
-// operand (NTOK = T rounded up to 16 columns), so every stage is 16 KB of
-// weights plus NTOK x 128 B of tokens and up to 12 stages stay in flight.
+// y[j, n] = x[j, :] . W[n, :] for j < T <= 128 tokens and the Nw rows of one
+// matrix W [Nw, Kdim].  A decode batch fills few of the 128 slot rows of the
+// MMA above, and a single matrix has few 256-row tiles; here the weights are
+// the A operand instead (128 rows per tile) and the tokens the B operand
+// (NTOK = 16, 32, 64 or 128 columns), so every stage is 16 KB of weights
+// plus NTOK x 128 B of tokens and 6-12 stages stay in flight.
 // Loaded HBM latency is ~3.5 us, so streaming at the HBM rate needs ~25 MB in
 // flight: the reduction is split over gridDim.y CTAs per tile (split z writes
 // its partial sums to y_out + z*T*Nw; the caller adds the parts in order).
@@ -393,13 +325,14 @@ struct SwapCfg {
             ? (int)((227 * 1024 - 1024 - kTcHeaderBytes) / kStageBytes)
             : 12;
     static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kTcHeaderBytes;
-    static constexpr uint32_t kTmemCols = 64;
+    static constexpr uint32_t kTmemCols = NTOK < 32 ? 32 : NTOK;
     // kind::f16: bf16 A and B, fp32 D, both K-major, N = NTOK, M = 128
     static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
                                        ((uint32_t)(NTOK >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-    static_assert(NTOK % 16 == 0 && NTOK >= 16 && NTOK <= 64, "token columns");
+    static_assert(NTOK % 16 == 0 && NTOK >= 16 && NTOK <= 128, "token columns");
     static_assert(kStageBytes % 1024 == 0, "stages stay 1024-byte aligned");
     static_assert(kStages >= 4 && kStages <= kMaxSwapStages, "stages");
+    static_assert((kTmemCols & (kTmemCols - 1)) == 0, "tensor memory is allocated in powers of two");
     static_assert(kSmem <= 227 * 1024, "shared memory");
 };
 
@@ -548,36 +481,6 @@ k_gather_rows(int S, int D, int K, const bf16 *__restrict__ x, const int32_t *__
     }
 }
 
-// ---- host: tensor maps -----------------------------------------------------------
-
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    });
-    return fn;
-}
-
-// 2-D bf16 row-major [rows, cols] tensor, box {64 columns, box_rows}, 128-byte
-// swizzle, zero fill outside the tensor.
-bool make_map(CUtensorMap *m, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
-    auto fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[2] = {cols, rows};
-    cuuint64_t strides[1] = {cols * 2};
-    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
-    cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
-              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int MODE, class C>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUtensorMap &b1,
                         const int32_t *offsets, int E, int S, int Kdim, int Nw, uint32_t a_bytes,
@@ -683,14 +586,15 @@ cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const vo
     if (T < 1 || T > kRowsMaxTokens || parts < 1 || parts > kRowsMaxParts)
         return cudaErrorInvalidValue;
     const int ntok = (T + 15) / 16 * 16;
-    const uint32_t xrows = ntok <= 16 ? 16 : ntok <= 32 ? 32 : 64;
+    const uint32_t xrows = ntok <= 16 ? 16 : ntok <= 32 ? 32 : ntok <= 64 ? 64 : 128;
     CUtensorMap mw, mx;
     if (!make_map(&mw, w, (uint64_t)Nw, (uint64_t)Kdim, BM) ||
         !make_map(&mx, x, (uint64_t)T, (uint64_t)Kdim, xrows))
         return cudaErrorInvalidValue;
     if (xrows == 16) return launch_swap<16>(mw, mx, T, Kdim, Nw, parts, y, st, name);
     if (xrows == 32) return launch_swap<32>(mw, mx, T, Kdim, Nw, parts, y, st, name);
-    return launch_swap<64>(mw, mx, T, Kdim, Nw, parts, y, st, name);
+    if (xrows == 64) return launch_swap<64>(mw, mx, T, Kdim, Nw, parts, y, st, name);
+    return launch_swap<128>(mw, mx, T, Kdim, Nw, parts, y, st, name);
 }
 
 }  // namespace moe

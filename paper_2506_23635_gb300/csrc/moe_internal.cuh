@@ -205,11 +205,22 @@ cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
 // reduction split into `parts` (<= kRowsMaxParts) shares whose partial sums
 // land in y + p*T*Nw for p < parts (the caller adds them in order).
 // gemm_rows_parts: the split that keeps the SMs streaming for this shape.
-constexpr int kRowsMaxTokens = 64;
+constexpr int kRowsMaxTokens = 128;
 constexpr int kRowsMaxParts = 4;
 int gemm_rows_parts(int Kdim, int Nw);
 cudaError_t launch_gemm_rows_tc(int T, int Kdim, int Nw, const void *x, const void *w, int parts,
                                 float *y, cudaStream_t st, const char *name = nullptr);
+// Causal attention of prefill tiles on the tensor cores (attn_tc.cu): every
+// 128-token tile of the call whose tokens are positions p0..p0+127 of one
+// sequence; tile_ok[i] = 1 for the tiles it handled (the others are left to
+// the CUDA-core kernel).  q16 [T, Hq*128] bf16 queries (rotated, unscaled),
+// caches [n_seq, Hkv, L, 128] bf16, head_dim 128.
+constexpr int kAttnTcTile = 128;
+bool attn_prefill_tc_ok();
+cudaError_t launch_attn_prefill_tc(int T, int Hq, int Hkv, int n_seq, int L, const int32_t *seq,
+                                   const int32_t *pos, const void *q16, const void *k_cache,
+                                   const void *v_cache, void *ctx, int *tile_ok, cudaStream_t st);
+
 // name: the profiling name of the launch (default "gemm_down_tc").
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,

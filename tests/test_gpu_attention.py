@@ -43,6 +43,8 @@ def _tokens(kind, n_seq, L, rng):
     if kind == "prefill":
         n = min(L, 70)
         return np.zeros(n, np.int32), np.arange(n, dtype=np.int32)
+    if kind == "chunk300":  # positions 37..336 of sequence 1: two full 128-token tiles + 44
+        return np.ones(300, np.int32), np.arange(37, 337, dtype=np.int32)
     # a chunk of sequence 0 after 10 cached positions, plus decode tokens
     seq = np.concatenate([np.zeros(20, np.int32), np.arange(1, n_seq, dtype=np.int32)])
     pos = np.concatenate([np.arange(10, 30, dtype=np.int32),
@@ -50,9 +52,11 @@ def _tokens(kind, n_seq, L, rng):
     return seq, pos
 
 
-# (D, Hq, Hkv, n_seq, max_len, tokens): groups of 2, 6, 1 and 8 query heads
-# per key/value head; one token (row-streaming projections) and batches
-# (tensor-core projections); position splits with ragged ends.
+# (D, Hq, Hkv, n_seq, max_len, tokens): groups of 2, 6, 1, 8 and 3 query
+# heads per key/value head; one token and batches of up to 128 tokens (the
+# tensor-core kernel with the weights as the M operand), beyond 128 the
+# grouped tensor-core GEMM (DBRX test below); position splits with ragged
+# ends, and a single split.
 CASES = [
     (256, 4, 2, 3, 64, "decode1"),
     (256, 4, 2, 6, 300, "decode"),
@@ -60,6 +64,8 @@ CASES = [
     (512, 4, 4, 5, 200, "mixed"),
     (1024, 8, 1, 4, 2500, "decode"),
     (384, 3, 1, 1, 1100, "decode1"),
+    (512, 8, 4, 1, 100, "prefill"),  # one position split per token: ctx written directly
+    (256, 4, 2, 2, 400, "chunk300"),  # tensor-core prefill tiles + a CUDA-core tail
 ]
 
 
