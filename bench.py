@@ -67,11 +67,15 @@ PREFILL_MIN_TOKENS = 512
 DECODER_WORKLOADS = {
     "dbrx-decoder-t1": (gen.DBRX, 1),
     "dbrx-decoder-t8": (gen.DBRX, 8),
-    # 4 DBRX-shaped experts resident (1.9 GB in all): the small case for ncu
-    # captures of the attention block's kernels
+    # prefill of one sequence (the paper's prompts are 128 tokens)
+    "dbrx-decoder-prefill-t128": (gen.DBRX, 128),
+    "dbrx-decoder-prefill-t2048": (gen.DBRX, 2048),
+    # 4 DBRX-shaped experts resident (about 2 GB in all): the small cases for
+    # ncu captures of the attention block's kernels
     "dbrx4-decoder-t8": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 8),
+    "dbrx4-decoder-prefill-t2048": (gen.LayerShape(6144, 10752, 4, 4, "bf16"), 2048),
 }
-METRIC_DECODER = "Decoder-layer us/token-step (DBRX-shaped attention + MoE, decode at context 2048)"
+METRIC_DECODER = "Decoder-layer us/token-step (DBRX-shaped attention + MoE)"
 
 
 def parse():
@@ -611,8 +615,8 @@ def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5, prefill=F
     for i in range(warmup):
         step(i)
     ms, launches, kstats = layer.time_steps(step, steps)
-    sa_names = ("sa_prenorm", "qkv_rows_tc", "qkv_gemm_tc", "rope_cache", "attention",
-                "attn_merge", "o_rows_tc", "o_gemm_tc", "residual_add")
+    sa_names = ("sa_prenorm", "qkv_rows_tc", "qkv_gemm_tc", "rope_cache", "attention_tc",
+                "attention", "attn_merge", "o_rows_tc", "o_gemm_tc", "residual_add")
     sa_ms = sum(v[1] for k, v in kstats.items() if k in sa_names) / steps
     b = sa_bytes(a, T, ctx_len)
     peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
@@ -674,8 +678,10 @@ def run_decoder(args, moe, dev, dist, rank, world):
     one JSON line with the step time per token and the attention block's
     share and roofline."""
     shape, T = DECODER_WORKLOADS[args.workload]
+    prefill = "prefill" in args.workload
     layer = Layer(moe, shape, dev, dist)
-    r = measure_decoder_layer(layer, T, steps=args.steps, warmup=max(3, args.warmup))
+    r = measure_decoder_layer(layer, T, steps=args.steps, warmup=max(3, args.warmup),
+                              prefill=prefill)
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
@@ -689,7 +695,8 @@ def run_decoder(args, moe, dev, dist, rank, world):
                 "pre-filled with synthetic entries)",
         "config": {"workload": args.workload, "d_model": shape.d_model,
                    "ffn_hidden": shape.ffn_hidden, "n_experts": shape.n_experts,
-                   "top_k": shape.top_k, "sequences_per_step": T, "context": r["context"],
+                   "top_k": shape.top_k, "tokens_per_step": T,
+                   "mode": r.get("mode", f"decode, {T} sequences at context {r.get('context')}"),
                    "attention": "48 query / 8 key-value heads of 128 (D_qkv = 8192)"},
         "attention_block": r["attention_block"], "kernels": r["kernels"],
         "gpu_launches": int(r["launches_per_step"] * args.steps),
@@ -882,7 +889,7 @@ def run_reference(args):
 
     decoder = args.workload in DECODER_WORKLOADS
     shape, T = DECODER_WORKLOADS[args.workload] if decoder else WORKLOADS[args.workload]
-    prefill = T >= PREFILL_MIN_TOKENS
+    prefill = "prefill" in args.workload if decoder else T >= PREFILL_MIN_TOKENS
     pool = 1 if prefill else POOL
     xs_host, w_r_host = token_pool(shape, T, SEED, pool)
     try:
@@ -902,18 +909,25 @@ def run_reference(args):
         src = "host-drawn seeded weights"
     chunk = 16
     if decoder:  # the attention block's weights and caches, host-drawn
-        a_shape, ctx_len = gen.DBRX_ATTN, 2048
+        a_shape = gen.DBRX_ATTN
+        ctx_len = T if prefill else 2048
         w_qkv, w_o = gen.host_attn_weights(a_shape, SEED)
-        kc, vc = (gen.to_f64(c, "bf16") for c in gen.host_kv_cache(a_shape, T, ctx_len, SEED))
-        seq = np.arange(T, dtype=np.int32)
+        kc, vc = (gen.to_f64(c, "bf16")
+                  for c in gen.host_kv_cache(a_shape, 1 if prefill else T, ctx_len, SEED))
+        seq = np.arange(T, dtype=np.int32) if not prefill else np.zeros(chunk, np.int32)
         pos = np.full(T, ctx_len - 1, np.int32)
 
     def one(i):
         if decoder:
-            x = gen.to_f64(xs_host[i % pool], shape.dtype)
-            oracle.decoder_layers(x, [(w_qkv, w_o, w_r_host, w1, v1, w2)], shape.dtype,
+            if prefill:  # a chunk of 16 consecutive positions over synthetic earlier entries
+                t0 = (i * chunk) % T
+                x, p = xs_host[0][t0:t0 + chunk], np.arange(t0, t0 + chunk, dtype=np.int32)
+            else:
+                x, p = xs_host[i % pool], pos
+            oracle.decoder_layers(gen.to_f64(x, shape.dtype),
+                                  [(w_qkv, w_o, w_r_host, w1, v1, w2)], shape.dtype,
                                   a_shape.n_heads, a_shape.n_kv_heads, a_shape.rope_base, 1e-6,
-                                  shape.top_k, seq, pos, [(kc, vc)])
+                                  shape.top_k, seq, p, [(kc, vc)])
         elif prefill:
             t0 = (i * chunk) % T
             toks = np.arange(t0, t0 + chunk, dtype=np.int32)
@@ -933,7 +947,12 @@ def run_reference(args):
         one(i)
     dt = time.perf_counter() - t0
     ms = dt / steps * 1e3
-    if prefill:
+    if decoder and prefill:
+        metric, unit, hib = METRIC_DECODER, UNIT, False
+        value = round(ms * 1e3 / chunk, 1)
+        sample = (f"{steps} steps of {chunk} consecutive of the {T} positions over synthetic "
+                  f"earlier cache entries (of {args.steps} requested)")
+    elif prefill:
         flops = 2.0 * chunk * shape.top_k * 3 * shape.d_model * shape.ffn_hidden
         metric, unit, hib = METRIC_PREFILL, "TFLOP/s", True
         value = round(flops / (ms / 1e3) / 1e12, 6)

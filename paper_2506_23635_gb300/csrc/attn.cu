@@ -129,57 +129,87 @@ k_sa_setup(int T, int32_t *offsets) {
 // and the values to the caches [n_seq, Hkv, L, 128] in bf16.  A block holds
 // kRopeRows head rows of one token, 64 threads each: thread i turns the pair
 // (i, i + 64) of a query or key head, or copies two value elements.
-constexpr int kRopeRows = 4;  // head rows per block
+constexpr int kRopeRows = 16;  // head rows per block
+constexpr int kRopeTokens = 8;  // tokens per block, one after the other
 
 __global__ void __launch_bounds__(kRopeRows * kHeadDim / 2)
-k_rope_cache(int Hq, int Hkv, int n_seq, int L, RopeRates rates, const int32_t *__restrict__ seq,
-             const int32_t *__restrict__ pos, const float *__restrict__ qkv, int n_part,
-             long long part_stride, float *__restrict__ q, bf16 *__restrict__ q16,
-             bf16 *__restrict__ kc, bf16 *__restrict__ vc, unsigned *err) {
+k_rope_cache(int T, int Hq, int Hkv, int n_seq, int L, RopeRates rates,
+             const int32_t *__restrict__ seq, const int32_t *__restrict__ pos,
+             const float *__restrict__ qkv, int n_part, long long part_stride,
+             float *__restrict__ q, bf16 *__restrict__ q16, bf16 *__restrict__ kc,
+             bf16 *__restrict__ vc, unsigned *err) {
     ptx::grid_dependency_wait();
     constexpr int H2 = kHeadDim / 2;
-    const int hr = blockIdx.x * kRopeRows + threadIdx.x / H2, t = blockIdx.y;
+    static_assert(kRopeTokens * H2 <= kRopeRows * H2, "one thread per (token, pair)");
+    __shared__ float cs_s[kRopeTokens][H2], sn_s[kRopeTokens][H2];
+    __shared__ int seq_s[kRopeTokens], pos_s[kRopeTokens];
+    const int hr = blockIdx.x * kRopeRows + threadIdx.x / H2;
     const int i = threadIdx.x % H2;
-    if (hr >= Hq + 2 * Hkv) return;
-    const int sq = seq[t], p = pos[t];
-    const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
-    if (!ok && hr == 0 && i == 0) set_error(err, kErrIndex);
     const int nq = Hq * kHeadDim, nkv = Hkv * kHeadDim;
-    const float *row = qkv + (size_t)t * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
-    float a = 0.f, b = 0.f;  // the projection's partial sums, added in order
-    for (int k = 0; k < n_part; ++k) {
-        a += row[k * part_stride + i];
-        b += row[k * part_stride + i + H2];
-    }
-    if (hr >= Hq + Hkv) {  // a value head: stored as it is
-        if (!ok) return;
-        bf16 *vd = vc + (((size_t)sq * Hkv + (hr - Hq - Hkv)) * L + p) * kHeadDim;
-        vd[i] = __float2bfloat16_rn(a);
-        vd[i + H2] = __float2bfloat16_rn(b);
-        return;
-    }
-    // the angle of pair i is pos * rate_i, formed and reduced to [-pi, pi]
-    // in fp64 (exact to far below fp32 resolution at any cache position),
-    // then evaluated in fp32
-    constexpr double kTwoPi = 6.283185307179586;
-    const double ang = (double)(ok ? p : 0) * rates.w[i];
-    const double red = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);
-    float sn, cs;
-    sincosf((float)red, &sn, &cs);
-    const float x0 = a * cs - b * sn, x1 = b * cs + a * sn;
-    if (hr < Hq) {
-        float *qo = q + (size_t)t * nq + (size_t)hr * kHeadDim;
-        qo[i] = x0;
-        qo[i + H2] = x1;
-        if (q16) {  // the tensor-core attention's copy
-            bf16 *qh = q16 + (size_t)t * nq + (size_t)hr * kHeadDim;
-            qh[i] = __float2bfloat16_rn(x0);
-            qh[i + H2] = __float2bfloat16_rn(x1);
+    const int tb = blockIdx.y * kRopeTokens;
+    const int nt = min(kRopeTokens, T - tb);
+    // the angles of every token of the block: pair i of token tb+u turns by
+    // pos * rate_i, formed and reduced to [-pi, pi] in fp64 (exact to far
+    // below fp32 resolution at any cache position), evaluated in fp32
+    if (threadIdx.x < nt * H2) {
+        const int u = threadIdx.x / H2, k = threadIdx.x % H2;
+        const int sq = seq[tb + u], p = pos[tb + u];
+        const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
+        if (k == 0) {
+            seq_s[u] = ok ? sq : -1;
+            pos_s[u] = p;
+            if (!ok && blockIdx.x == 0) set_error(err, kErrIndex);
         }
-    } else if (ok) {
-        bf16 *kd = kc + (((size_t)sq * Hkv + (hr - Hq)) * L + p) * kHeadDim;
-        kd[i] = __float2bfloat16_rn(x0);
-        kd[i + H2] = __float2bfloat16_rn(x1);
+        constexpr double kTwoPi = 6.283185307179586;
+        const double ang = (double)(ok ? p : 0) * rates.w[k];
+        const double red = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);
+        sincosf((float)red, &sn_s[u][k], &cs_s[u][k]);
+    }
+    __syncthreads();
+    if (hr >= Hq + 2 * Hkv) return;
+    // every token's pair first (independent loads in flight together), the
+    // projection's partial sums added in order
+    float av[kRopeTokens], bv[kRopeTokens];
+#pragma unroll
+    for (int u = 0; u < kRopeTokens; ++u) {
+        av[u] = 0.f;
+        bv[u] = 0.f;
+        if (u < nt) {
+            const float *row = qkv + (size_t)(tb + u) * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
+            for (int k = 0; k < n_part; ++k) {
+                av[u] += row[k * part_stride + i];
+                bv[u] += row[k * part_stride + i + H2];
+            }
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kRopeTokens; ++u) {
+        if (u >= nt) break;
+        const int t = tb + u, sq = seq_s[u], p = pos_s[u];
+        const float a = av[u], b = bv[u];
+        if (hr >= Hq + Hkv) {  // a value head: stored as it is
+            if (sq < 0) continue;
+            bf16 *vd = vc + (((size_t)sq * Hkv + (hr - Hq - Hkv)) * L + p) * kHeadDim;
+            vd[i] = __float2bfloat16_rn(a);
+            vd[i + H2] = __float2bfloat16_rn(b);
+            continue;
+        }
+        const float cs = cs_s[u][i], sn = sn_s[u][i];
+        const float x0 = a * cs - b * sn, x1 = b * cs + a * sn;
+        if (hr < Hq) {
+            float *qo = q + (size_t)t * nq + (size_t)hr * kHeadDim;
+            qo[i] = x0;
+            qo[i + H2] = x1;
+            if (q16) {  // the tensor-core attention's copy
+                bf16 *qh = q16 + (size_t)t * nq + (size_t)hr * kHeadDim;
+                qh[i] = __float2bfloat16_rn(x0);
+                qh[i + H2] = __float2bfloat16_rn(x1);
+            }
+        } else if (sq >= 0) {
+            bf16 *kd = kc + (((size_t)sq * Hkv + (hr - Hq)) * L + p) * kHeadDim;
+            kd[i] = __float2bfloat16_rn(x0);
+            kd[i + H2] = __float2bfloat16_rn(x1);
+        }
     }
 }
 
@@ -544,11 +574,13 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
     const float *qkvc = qkv;
     bf16 *kcp = static_cast<bf16 *>(kc), *vcp = static_cast<bf16 *>(vc);
     unsigned *err = device_info().err;
-    void *args[] = {&Hq,     &Hkv,     &ns, &Lv,  &rates, &seq, &pos, &qkvc,
-                    &n_part, &pstride, &q,  &q16, &kcp,   &vcp,  &err};
+    int Tv = c.T;
+    void *args[] = {&Tv,     &Hq,      &Hkv, &ns,  &Lv,  &rates, &seq, &pos,
+                    &qkvc,   &n_part,  &pstride, &q, &q16, &kcp, &vcp, &err};
     LaunchScope ls("rope_cache", c.st);
     const int rows = Hq + 2 * Hkv;
-    return launch_pdl((const void *)k_rope_cache, dim3((rows + kRopeRows - 1) / kRopeRows, c.T),
+    return launch_pdl((const void *)k_rope_cache,
+                      dim3((rows + kRopeRows - 1) / kRopeRows, (c.T + kRopeTokens - 1) / kRopeTokens),
                       dim3(kRopeRows * kHeadDim / 2), 0, c.st, args);
 }
 

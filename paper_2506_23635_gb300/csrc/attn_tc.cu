@@ -5,21 +5,25 @@
 // head h), key/value head g = h / (Hq/Hkv), over cache positions 0 .. p0+127
 // in key/value tiles of 128 positions:
 //
-//   warp 0      TMA: the tile's bf16 queries once, then the key and value
-//               tiles of positions [128j, 128j+128) into a two-stage ring;
+//   warp 0      TMA: the tile's bf16 queries once, then the key tiles of
+//               positions [128j, 128j+128) into a two-stage ring and the value
+//               tiles into one stage (free again once transposed);
 //   warp 1      tensor memory (512 columns: two score buffers and one output
 //               tile) and the MMAs: S_j = Q K_j^T (M = 128 queries, N = 128
 //               positions, K = 128 dims) into score buffer j % 2, and once
 //               the softmax warps have written P_j and V_j^T,
 //               O_j = P_j V_j (M = 128 queries, N = 128 dims, K = 128
 //               positions) into the output tile;
-//   warps 2-5   one thread per query row: fold O_{j-1} into the row's fp32
-//               accumulator (registers), transpose V_j into the K-major V^T
-//               tile (positions past the tile's last query are written as
-//               zero), then the online softmax of S_j (causal mask, base-2
-//               exponent of the 1/sqrt(128)-scaled scores) and the bf16
-//               probabilities P_j, both written in the 128-byte-swizzled
-//               K-major layout the MMA reads.
+//   warps 2-9   two threads per query row, each owning 64 of the 128 score
+//               columns and of the 128 output dims: fold O_{j-1} into the
+//               row's fp32 accumulator (registers), transpose V_j into the
+//               K-major V^T tile with ldmatrix.trans / stmatrix (positions
+//               past the tile's last query are written as zero), then the
+//               online softmax of S_j (causal mask, base-2 exponent of the
+//               1/sqrt(128)-scaled scores; the two halves of a row exchange
+//               their maxima through shared memory) and the bf16
+//               probabilities P_j, written in the 128-byte-swizzled K-major
+//               layout the MMA reads.
 //
 // Every wait is bounded (ptx.cuh).  Tiles that do not satisfy the layout
 // condition record tile_ok = 0 and are left to the CUDA-core kernel.
@@ -34,17 +38,19 @@ using namespace tc;
 
 constexpr int kFa = 128;                 // queries per tile, positions per key/value tile
 constexpr int kHeadDimFa = 128;
-constexpr int kFaThreads = 192;          // 6 warps
+constexpr int kFaSoftmaxWarps = 8;       // two threads per query row
+constexpr int kFaThreads = (2 + kFaSoftmaxWarps) * 32;
 constexpr uint32_t kHalfBytes = kFa * 128;     // one 64-column half of a 128-row tile
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;  // 32 KB
-// shared memory: Q, K[2], V[2], V^T, P (each a 32 KB tile), then the header
+// shared memory: Q, K[2], V, V^T, P (each a 32 KB tile), then the header
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kTileBytes;
 constexpr uint32_t kOffV = 3 * kTileBytes;
-constexpr uint32_t kOffVt = 5 * kTileBytes;
-constexpr uint32_t kOffP = 6 * kTileBytes;
-constexpr uint32_t kOffHdr = 7 * kTileBytes;
-constexpr size_t kFaSmem = 1024 + kOffHdr + 256;
+constexpr uint32_t kOffVt = 4 * kTileBytes;
+constexpr uint32_t kOffP = 5 * kTileBytes;
+constexpr uint32_t kOffHdr = 6 * kTileBytes;
+constexpr uint32_t kOffRed = kOffHdr + 256;  // row max / sum exchange: [2][2][128] floats
+constexpr size_t kFaSmem = 1024 + kOffRed + 2 * 2 * kFa * 4;
 static_assert(kFaSmem <= 227 * 1024, "shared memory");
 // kind::f16 instruction descriptor: bf16 A and B, fp32 D, K-major, N = M = 128
 constexpr uint32_t kFaIdesc =
@@ -53,11 +59,13 @@ constexpr uint32_t kFaTmemCols = 512;  // S[0] 0..127, S[1] 128..255, O 256..383
 
 struct FaHeader {
     uint64_t q_full;
-    uint64_t kv_full[2];
+    uint64_t kv_full[2];   // key tile j in stage j % 2
     uint64_t kv_empty[2];
+    uint64_t v_full;       // value tile j (one stage)
+    uint64_t v_empty;      // the softmax warps have transposed it (one arrival each)
     uint64_t s_full[2];
-    uint64_t s_free[2];  // the softmax warps have read score buffer b (4 arrivals)
-    uint64_t p_ready;    // P_j and V_j^T written (4 arrivals)
+    uint64_t s_free[2];  // the softmax warps have read score buffer b (one arrival each)
+    uint64_t p_ready;    // P_j and V_j^T written (one arrival per softmax warp)
     uint64_t o_full;
     uint64_t done;
     uint32_t tmem_base;
@@ -68,6 +76,27 @@ static_assert(sizeof(FaHeader) <= 256, "flash-attention header");
 // 128 x 128 bf16 tile: two 64-column halves, K-major, 128-byte swizzle.
 __device__ __forceinline__ uint32_t tile_offset(uint32_t r, uint32_t k) {
     return (k >> 6) * kHalfBytes + swizzle_offset(r, k & 63u);
+}
+
+// Four 8x8 bf16 blocks, transposed on the way into registers / stored as is.
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+__device__ __forceinline__ void stsm_x4(uint32_t addr, const uint32_t (&r)[4]) {
+    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(addr),
+                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
+                 : "memory");
+}
+
+// 2^x on the special-function unit (the probabilities are rounded to bf16
+// right after, far coarser than its error).
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
 __device__ __forceinline__ void issue_128x128x128(uint32_t d_tmem, uint32_t a_smem, uint32_t b_smem) {
@@ -102,9 +131,11 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             ptx::mbar_init(&hd->kv_full[b], 1);
             ptx::mbar_init(&hd->kv_empty[b], 1);
             ptx::mbar_init(&hd->s_full[b], 1);
-            ptx::mbar_init(&hd->s_free[b], 4);
+            ptx::mbar_init(&hd->s_free[b], kFaSoftmaxWarps);
         }
-        ptx::mbar_init(&hd->p_ready, 4);
+        ptx::mbar_init(&hd->p_ready, kFaSoftmaxWarps);
+        ptx::mbar_init(&hd->v_full, 1);
+        ptx::mbar_init(&hd->v_empty, kFaSoftmaxWarps);
         ptx::mbar_init(&hd->o_full, 1);
         ptx::mbar_init(&hd->done, 1);
         ptx::fence_barrier_init();
@@ -144,22 +175,27 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                                  &hd->q_full, pol);
             const int row0 = (sq * Hkv + g) * L;
             int issued = 0;
+            int v_issued = 0;
             for (int j = 0; j < n_kv; ++j) {
                 const int b = j & 1;
                 if (!ptx::mbar_wait(&hd->kv_empty[b], ((j >> 1) & 1) ^ 1, err)) break;
-                ptx::mbar_arrive_expect_tx(&hd->kv_full[b], 2 * kTileBytes);
-                for (int half = 0; half < 2; ++half) {
+                ptx::mbar_arrive_expect_tx(&hd->kv_full[b], kTileBytes);
+                for (int half = 0; half < 2; ++half)
                     ptx::tma_load_2d(smem + kOffK + b * kTileBytes + half * kHalfBytes, &tmK,
                                      half * 64, row0 + j * kFa, &hd->kv_full[b], pol);
-                    ptx::tma_load_2d(smem + kOffV + b * kTileBytes + half * kHalfBytes, &tmV,
-                                     half * 64, row0 + j * kFa, &hd->kv_full[b], pol);
-                }
                 issued = j + 1;
+                if (!ptx::mbar_wait(&hd->v_empty, (j & 1) ^ 1, err)) break;
+                ptx::mbar_arrive_expect_tx(&hd->v_full, kTileBytes);
+                for (int half = 0; half < 2; ++half)
+                    ptx::tma_load_2d(smem + kOffV + half * kHalfBytes, &tmV, half * 64,
+                                     row0 + j * kFa, &hd->v_full, pol);
+                v_issued = j + 1;
             }
             // let loads still in flight land before the block can exit
             ptx::mbar_wait(&hd->q_full, 0, err);
             for (int j = (issued > 2 ? issued - 2 : 0); j < issued; ++j)
                 ptx::mbar_wait(&hd->kv_full[j & 1], (j >> 1) & 1, err);
+            if (v_issued > 0) ptx::mbar_wait(&hd->v_full, (v_issued - 1) & 1, err);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -173,6 +209,7 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                     tc_fence_after();
                     issue_128x128x128(tmem + b * kFa, sbase + kOffQ, sbase + kOffK + b * kTileBytes);
                     mma_commit(&hd->s_full[b]);
+                    mma_commit(&hd->kv_empty[b]);  // key tile j read once these finish
                 }
                 if (j >= 1) {  // O_{j-1} = P_{j-1} V_{j-1}
                     const int jp = j - 1;
@@ -180,7 +217,6 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                     tc_fence_after();
                     issue_128x128x128(tmem + 2 * kFa, sbase + kOffP, sbase + kOffVt);
                     mma_commit(&hd->o_full);
-                    mma_commit(&hd->kv_empty[jp & 1]);
                 }
             }
             mma_commit(&hd->done);
@@ -189,95 +225,116 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         __syncwarp();
     } else if (ok) {
         // ------------------------------------------------------------ softmax
-        const int q = warp & 3;             // tensor-memory lane quarter
-        const int r = q * 32 + lane;        // query row of the tile
-        const int st = (warp - 2) * 32 + lane;  // 0..127: the V^T row this thread writes
+        const int q = warp & 3;                  // tensor-memory lane quarter
+        const int r = q * 32 + lane;             // query row of the tile
+        const int w8 = warp - 2;                 // 0..7
+        const int hf = w8 >> 2;                  // column half: scores and output dims
+        const int c0 = hf * 64;
         const int qpos = p0 + r;
-        const int last = p0 + kFa - 1;      // the tile's last query position
+        const int last = p0 + kFa - 1;           // the tile's last query position
         const float sl2 = 1.4426950408889634f / sqrtf((float)kHeadDimFa);
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        float o[128];
+        float *red = reinterpret_cast<float *>(smem + kOffRed);  // [2 buffers][2 halves][128]
+        float o[64];
 #pragma unroll
-        for (int i = 0; i < 128; ++i) o[i] = 0.f;
-        float m = -INFINITY, l = 0.f, corr = 1.f;
+        for (int i = 0; i < 64; ++i) o[i] = 0.f;
+        float m = -INFINITY, l = 0.f, corr = 1.f;  // l: this half's share of the row sum
+        // every softmax warp runs every iteration and reaches every named
+        // barrier: a wait that gave up (recorded in err) turns the later waits
+        // into no-ops instead of leaving the loop early
         bool good = true;
-        for (int j = 0; j < n_kv && good; ++j) {
+        for (int j = 0; j < n_kv; ++j) {
             const int b = j & 1;
             if (j >= 1) {  // fold O_{j-1}; then P, V^T and the output tile are free
-                if (!(good = ptx::mbar_wait(&hd->o_full, (j - 1) & 1, err))) break;
+                good = good && ptx::mbar_wait(&hd->o_full, (j - 1) & 1, err);
                 tc_fence_after();
 #pragma unroll
-                for (int c = 0; c < 128; c += 32) {
+                for (int c = 0; c < 64; c += 32) {
                     float v[32];
-                    tmem_ld32(tmem + lane_base + 2 * kFa + c, v);
+                    tmem_ld32(tmem + lane_base + 2 * kFa + c0 + c, v);
                     tmem_ld_wait();
 #pragma unroll
                     for (int i = 0; i < 32; ++i) o[c + i] = fmaf(o[c + i], corr, v[i]);
                 }
             }
-            // V_j -> V^T (row = dim st, column = position), zero past `last`
-            if (!(good = ptx::mbar_wait(&hd->kv_full[b], (j >> 1) & 1, err))) break;
+            // V_j -> V^T (row = dim, column = position), zero past `last`: warp
+            // w8 transposes position blocks 2w8, 2w8+1, four 8x8 blocks (dims
+            // 32k..32k+31) per ldmatrix.trans / stmatrix pair
+            good = good && ptx::mbar_wait(&hd->v_full, j & 1, err);
             {
-                const unsigned char *vs = smem + kOffV + b * kTileBytes;
-                unsigned char *vt = smem + kOffVt;
-                const int d = st;
-#pragma unroll 2
-                for (int p8 = 0; p8 < kFa; p8 += 8) {
-                    uint32_t w[4];
+                const uint32_t vs = sbase + kOffV, vt = sbase + kOffVt;
+                const bool clip = j * kFa + kFa - 1 > last;
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int pa = p8 + 2 * e, pb = pa + 1;
-                        const uint16_t va = *reinterpret_cast<const uint16_t *>(vs + tile_offset(pa, d));
-                        const uint16_t vb = *reinterpret_cast<const uint16_t *>(vs + tile_offset(pb, d));
-                        const uint32_t lo = j * kFa + pa <= last ? va : 0u;
-                        const uint32_t hi = j * kFa + pb <= last ? vb : 0u;
-                        w[e] = lo | (hi << 16);
+                for (int pbi = 0; pbi < 2; ++pbi) {
+                    const int pb = w8 * 2 + pbi;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int db = 4 * k + (lane >> 3);  // this lane's block for the addresses
+                        uint32_t rr[4];
+                        ldsm_x4_trans(vs + tile_offset(8 * pb + (lane & 7), 8 * db), rr);
+                        if (clip) {  // register i holds positions 8pb + 2(lane%4) and +1
+                            const int pa = j * kFa + 8 * pb + 2 * (lane & 3);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                if (pa > last) rr[i] &= 0xffff0000u;
+                                if (pa + 1 > last) rr[i] &= 0x0000ffffu;
+                            }
+                        }
+                        stsm_x4(vt + tile_offset(8 * db + (lane & 7), 8 * pb), rr);
                     }
-                    *reinterpret_cast<uint4 *>(vt + tile_offset(d, p8)) = make_uint4(w[0], w[1], w[2], w[3]);
                 }
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&hd->v_empty);  // value tile read
             }
-            // scores of S_j: masked row max, then probabilities
-            if (!(good = ptx::mbar_wait(&hd->s_full[b], (j >> 1) & 1, err))) break;
+            // scores of S_j (this thread's 64 columns): masked max, exchanged
+            // with the other half of the row, then probabilities
+            good = good && ptx::mbar_wait(&hd->s_full[b], (j >> 1) & 1, err);
             tc_fence_after();
-            const uint32_t sb = tmem + lane_base + b * kFa;
-            float mx = m;
+            const uint32_t sb = tmem + lane_base + b * kFa + c0;
+            const bool full = j * kFa + kFa - 1 <= p0;  // no position of the tile is masked
+            float v[64];
+            tmem_ld32(sb, *reinterpret_cast<float(*)[32]>(&v[0]));
+            tmem_ld32(sb + 32, *reinterpret_cast<float(*)[32]>(&v[32]));
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&hd->s_free[b]);  // scores read
+            float hm = -INFINITY;
+            if (full) {
 #pragma unroll
-            for (int c = 0; c < 128; c += 32) {
-                float v[32];
-                tmem_ld32(sb + c, v);
-                tmem_ld_wait();
+                for (int i = 0; i < 64; ++i) hm = fmaxf(hm, v[i]);
+            } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (j * kFa + c + i <= qpos) mx = fmaxf(mx, v[i] * sl2);
+                for (int i = 0; i < 64; ++i)
+                    if (j * kFa + c0 + i <= qpos) hm = fmaxf(hm, v[i]);
             }
-            // mx is finite: position 128j <= qpos for every row of the tile
+            red[(b * 2 + hf) * kFa + r] = hm;
+            ptx::named_bar_sync(1, kFaSoftmaxWarps * 32);
+            const float other = red[(b * 2 + (hf ^ 1)) * kFa + r];
+            // finite: position 128j <= qpos for every row of the tile
+            const float mx = fmaxf(m, fmaxf(hm, other) * sl2);
             float sum = 0.f;
             unsigned char *ps = smem + kOffP;
 #pragma unroll
-            for (int c = 0; c < 128; c += 32) {
-                float v[32];
-                tmem_ld32(sb + c, v);
-                tmem_ld_wait();
+            for (int i = 0; i < 64; i += 8) {
+                uint32_t w[4];
 #pragma unroll
-                for (int i = 0; i < 32; i += 8) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int ca = c + i + 2 * e;
-                        const float pa = j * kFa + ca <= qpos ? exp2f(v[i + 2 * e] * sl2 - mx) : 0.f;
-                        const float pb =
-                            j * kFa + ca + 1 <= qpos ? exp2f(v[i + 2 * e + 1] * sl2 - mx) : 0.f;
-                        const __nv_bfloat162 p2 = __floats2bfloat162_rn(pa, pb);
-                        // the row sum takes the probabilities as stored
-                        sum += __low2float(p2) + __high2float(p2);
-                        w[e] = *reinterpret_cast<const uint32_t *>(&p2);
+                for (int e = 0; e < 4; ++e) {
+                    const int ca = c0 + i + 2 * e;
+                    float pa = fast_exp2(fmaf(v[i + 2 * e], sl2, -mx));
+                    float pb = fast_exp2(fmaf(v[i + 2 * e + 1], sl2, -mx));
+                    if (!full) {
+                        if (j * kFa + ca > qpos) pa = 0.f;
+                        if (j * kFa + ca + 1 > qpos) pb = 0.f;
                     }
-                    *reinterpret_cast<uint4 *>(ps + tile_offset(r, c + i)) = make_uint4(w[0], w[1], w[2], w[3]);
+                    const __nv_bfloat162 p2 = __floats2bfloat162_rn(pa, pb);
+                    // the row sum takes the probabilities as stored, so the
+                    // weights P V is normalised by sum to exactly one
+                    sum += __low2float(p2) + __high2float(p2);
+                    w[e] = *reinterpret_cast<const uint32_t *>(&p2);
                 }
+                *reinterpret_cast<uint4 *>(ps + tile_offset(r, c0 + i)) = make_uint4(w[0], w[1], w[2], w[3]);
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&hd->s_free[b]);
             fence_proxy_async_smem();  // P_j and V_j^T visible to the MMA
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&hd->p_ready);
@@ -285,22 +342,26 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             l = l * corr + sum;
             m = mx;
         }
+        // the row sum: both halves' shares
+        red[hf * kFa + r] = l;
+        ptx::named_bar_sync(1, kFaSoftmaxWarps * 32);
+        const float lt = l + red[(hf ^ 1) * kFa + r];
         if (good && n_kv > 0 && ptx::mbar_wait(&hd->o_full, (n_kv - 1) & 1, err)) {
             tc_fence_after();
-            const float inv = l > 0.f ? 1.f / l : 0.f;
-            bf16 *dst = ctx + ((size_t)(t0 + r) * Hq + h) * 128;
+            const float inv = lt > 0.f ? 1.f / lt : 0.f;
+            bf16 *dst = ctx + ((size_t)(t0 + r) * Hq + h) * 128 + c0;
 #pragma unroll
-            for (int c = 0; c < 128; c += 32) {
-                float v[32];
-                tmem_ld32(tmem + lane_base + 2 * kFa + c, v);
+            for (int c = 0; c < 64; c += 32) {
+                float vv[32];
+                tmem_ld32(tmem + lane_base + 2 * kFa + c0 + c, vv);
                 tmem_ld_wait();
 #pragma unroll
                 for (int i = 0; i < 32; i += 8) {
                     uint32_t w[4];
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float a = fmaf(o[c + i + 2 * e], corr, v[i + 2 * e]) * inv;
-                        const float bq = fmaf(o[c + i + 2 * e + 1], corr, v[i + 2 * e + 1]) * inv;
+                        const float a = fmaf(o[c + i + 2 * e], corr, vv[i + 2 * e]) * inv;
+                        const float bq = fmaf(o[c + i + 2 * e + 1], corr, vv[i + 2 * e + 1]) * inv;
                         const __nv_bfloat162 p2 = __floats2bfloat162_rn(a, bq);
                         w[e] = *reinterpret_cast<const uint32_t *>(&p2);
                     }
