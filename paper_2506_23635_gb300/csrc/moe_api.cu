@@ -587,35 +587,72 @@ k_dispatch(int S, int E, const int32_t *__restrict__ idx, int32_t *__restrict__ 
 // Step 4 (unfused): out[t,:] = residual + sum_k gate[t,k] * y_sorted[inv[t*K+k],:]
 // One thread per 4 consecutive outputs; k in ascending order.
 // ===========================================================================
+// Four consecutive values of a row in the output / residual type.
+__device__ __forceinline__ float4 load4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ float4 load4(const bf16 *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    float4 v;
+    unpack_bf16x2(u.x, v.x, v.y);
+    unpack_bf16x2(u.y, v.z, v.w);
+    return v;
+}
+__device__ __forceinline__ void store4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
+__device__ __forceinline__ void store4(bf16 *p, float4 v) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+    *reinterpret_cast<uint2 *>(p) = make_uint2(*reinterpret_cast<const uint32_t *>(&a),
+                                               *reinterpret_cast<const uint32_t *>(&b));
+}
+
+constexpr int kCombineMaxK = 256;  // = the largest top_k
+
+// out[t, :] = residual + sum_k gate[t,k] y[inv[t,k], :], k ascending.  Block
+// b takes token b / n_part and the b % n_part-th slice of its row; the
+// token's K sorted positions and gates are read once into shared memory, then
+// every thread's K row loads are independent (streamed past L1).
 template <typename TO, typename TR>
 __global__ void __launch_bounds__(256)
-k_combine(int T, int D, int K, const float *__restrict__ y, const int32_t *__restrict__ inv,
-          const float *__restrict__ gate, const TR *__restrict__ residual, TO *__restrict__ out,
-          unsigned *err) {
+k_combine(int T, int D, int K, int n_part, const float *__restrict__ y,
+          const int32_t *__restrict__ inv, const float *__restrict__ gate,
+          const TR *__restrict__ residual, TO *__restrict__ out, unsigned *err) {
+    __shared__ int s_j[kCombineMaxK];
+    __shared__ float s_g[kCombineMaxK];
+    ptx::grid_dependency_wait();
     const int S = T * K;
     const int nq = D >> 2;
-    const long long total = (long long)T * nq;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int t = (int)(i / nq);
-        const int d = (int)(i - (long long)t * nq) * 4;
-        float a[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int k = 0; k < K; ++k) {
+    const int per = (nq + n_part - 1) / n_part;
+    for (long long b = blockIdx.x; b < (long long)T * n_part; b += gridDim.x) {
+        const int t = (int)(b / n_part), part = (int)(b - (long long)t * n_part);
+        __syncthreads();  // the previous token's indices are no longer read
+        for (int k = threadIdx.x; k < K; k += blockDim.x) {
             const int j = inv[(size_t)t * K + k];
-            if (j < 0 || j >= S) {  // a slot left out by dispatch, or a corrupt index
-                if (j >= S) set_error(err, kErrIndex);
-                continue;
-            }
-            const float g = gate[(size_t)t * K + k];
-            const float4 v = *reinterpret_cast<const float4 *>(y + (size_t)j * D + d);
-            a[0] = fmaf(g, v.x, a[0]); a[1] = fmaf(g, v.y, a[1]);
-            a[2] = fmaf(g, v.z, a[2]); a[3] = fmaf(g, v.w, a[3]);
+            if (j >= S) set_error(err, kErrIndex);  // a corrupt index
+            s_j[k] = (j < 0 || j >= S) ? -1 : j;    // or a slot left out by dispatch
+            s_g[k] = gate[(size_t)t * K + k];
         }
-        if (residual)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) a[q] += to_f(residual[(size_t)t * D + d + q]);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) out[(size_t)t * D + d + q] = from_f<TO>(a[q]);
+        __syncthreads();
+        const int q1 = min(nq, (part + 1) * per);
+        for (int q = part * per + threadIdx.x; q < q1; q += blockDim.x) {
+            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+            for (int k = 0; k < K; ++k) {
+                const int j = s_j[k];
+                if (j < 0) continue;
+                const float g = s_g[k];
+                const uint4 u = ld_stream16(y + (size_t)j * D + 4 * q);
+                a.x = fmaf(g, __uint_as_float(u.x), a.x);
+                a.y = fmaf(g, __uint_as_float(u.y), a.y);
+                a.z = fmaf(g, __uint_as_float(u.z), a.z);
+                a.w = fmaf(g, __uint_as_float(u.w), a.w);
+            }
+            if (residual) {
+                const float4 r = load4(residual + (size_t)t * D + 4 * q);
+                a.x += r.x;
+                a.y += r.y;
+                a.z += r.z;
+                a.w += r.w;
+            }
+            store4(out + (size_t)t * D + 4 * q, a);
+        }
     }
 }
 
@@ -959,15 +996,19 @@ cudaError_t dispatch_any(const moe_dims &d, int T, const int32_t *idx, int32_t *
 template <typename TO, typename TR>
 cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const int32_t *inv,
                            const float *gate, const void *res, void *out, cudaStream_t st) {
-    const long long total = (long long)T * (d.d_model / 4);
+    // enough blocks for 8 per SM: a token's row is split into n_part slices
+    // of at least 256 float4 when there are few tokens
+    const int nq = d.d_model / 4;
     const long long cap = (long long)device_info().sm_count * 8;
-    const long long want = (total + 255) / 256;
-    const int grid = (int)std::max(1LL, std::min(want, cap));
+    int n_part = (int)std::max(1LL, std::min<long long>((cap + T - 1) / T, (nq + 255) / 256));
+    const int grid = (int)std::max(1LL, std::min((long long)T * n_part, cap));
+    int Tv = T, D = d.d_model, K = d.top_k;
+    const TR *rp = static_cast<const TR *>(res);
+    TO *op = static_cast<TO *>(out);
+    unsigned *err = device_info().err;
+    void *args[] = {&Tv, &D, &K, &n_part, &y, &inv, &gate, &rp, &op, &err};
     LaunchScope ls("combine", st);
-    k_combine<TO, TR><<<grid, 256, 0, st>>>(T, d.d_model, d.top_k, y, inv, gate,
-                                            static_cast<const TR *>(res), static_cast<TO *>(out),
-                                            device_info().err);
-    return cudaGetLastError();
+    return launch_pdl((const void *)k_combine<TO, TR>, dim3(grid), dim3(256), 0, st, args);
 }
 
 cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t *inv,
