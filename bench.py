@@ -56,6 +56,10 @@ WORKLOADS = {
     # (F=1024, 0.6 GB resident): the small case for captures of the cluster
     # route+dispatch kernel, whose work does not depend on F
     "dbrx-router-t8": (gen.LayerShape(6144, 1024, 16, 4, "bf16"), 8),
+    # the same narrow-expert layer on a 2048-token prefill (0.9 GB resident):
+    # the small case for captures of the prefill routing, dispatch, gather
+    # and combine kernels, whose work does not depend on F
+    "dbrx-router-t2048": (gen.LayerShape(6144, 1024, 16, 4, "bf16"), 2048),
     # the tiny fp32 layer (D=256, F=512, E=4, K=2), 8 tokens: the reference
     # arm's smallest case (runs anywhere, no GPU needed)
     "tiny-decode-t8": (gen.TINY, 8),

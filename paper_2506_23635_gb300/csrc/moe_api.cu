@@ -583,6 +583,113 @@ k_dispatch(int S, int E, const int32_t *__restrict__ idx, int32_t *__restrict__ 
     }
 }
 
+// Single-pass variant for up to kFastMaxChunks chunks (8192 slots) whose
+// per-(chunk, warp) expert counts fit in shared memory (the 2048-token
+// prefill: 8 x 32 x 16).
+// All chunks' warp counts are taken in one pass (each thread keeps its slots'
+// experts and in-warp ranks in registers), each expert's counts are scanned
+// in (chunk, warp) order by one warp, then every slot's position is written:
+// the same stable order as k_dispatch with three block barriers instead of
+// four per chunk.
+constexpr int kFastMaxChunks = 8;
+constexpr size_t kFastDispatchSmem = 40 * 1024;
+
+__global__ void __launch_bounds__(kDispatchThreads)
+k_dispatch_fast(int S, int E, const int32_t *__restrict__ idx, int32_t *__restrict__ counts,
+                int32_t *__restrict__ offsets, int32_t *__restrict__ perm,
+                int32_t *__restrict__ inv_perm, unsigned *err) {
+    constexpr int NW = kDispatchThreads / 32;
+    extern __shared__ int wh[];  // [C * NW][E]: counts, then exclusive in-expert starts
+    __shared__ int tot[256], off[256];
+    ptx::grid_dependency_wait();
+    const int C = (S + kDispatchThreads - 1) / kDispatchThreads;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const unsigned lt_mask = (1u << lane) - 1u;
+    for (int i = tid; i < C * NW * E; i += kDispatchThreads) wh[i] = 0;
+    __syncthreads();
+    int ec[kFastMaxChunks], rc[kFastMaxChunks];
+#pragma unroll
+    for (int c = 0; c < kFastMaxChunks; ++c) {  // every load in flight at once
+        const int s = c * kDispatchThreads + tid;
+        ec[c] = c < C && s < S ? idx[s] : -1;
+    }
+#pragma unroll
+    for (int c = 0; c < kFastMaxChunks; ++c) {
+        rc[c] = 0;
+        if (c < C) {  // uniform across the block
+            const int s = c * kDispatchThreads + tid;
+            int e = ec[c];
+            const bool valid = e >= 0 && e < E;
+            if (s < S && !valid) set_error(err, kErrIndex);
+            if (!valid) e = -1;
+            const unsigned same = __match_any_sync(0xffffffffu, e);
+            rc[c] = __popc(same & lt_mask);
+            if (valid && rc[c] == 0) wh[(c * NW + warp) * E + e] = __popc(same);
+            ec[c] = e;
+        }
+    }
+    __syncthreads();
+    // expert e: exclusive scan of its counts over (chunk, warp) = C*NW
+    // entries, lane l taking entries [l*C, (l+1)*C)
+    for (int e = warp; e < E; e += NW) {
+        int loc[kFastMaxChunks], sum = 0;
+#pragma unroll
+        for (int i = 0; i < kFastMaxChunks; ++i) {
+            loc[i] = i < C ? wh[(lane * C + i) * E + e] : 0;
+            sum += loc[i];
+        }
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        int run = incl - sum;
+#pragma unroll
+        for (int i = 0; i < kFastMaxChunks; ++i)
+            if (i < C) {
+                wh[(lane * C + i) * E + e] = run;
+                run += loc[i];
+            }
+        if (lane == 31) tot[e] = incl;
+    }
+    __syncthreads();
+    if (warp == 0) {  // exclusive scan of the expert totals
+        int carry = 0;
+        for (int base = 0; base < E; base += 32) {
+            const int e = base + lane;
+            const int c = e < E ? tot[e] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (e < E) {
+                off[e] = carry + incl - c;
+                counts[e] = c;
+                offsets[e] = carry + incl - c;
+            }
+            carry += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) offsets[E] = carry;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int c = 0; c < kFastMaxChunks; ++c) {
+        if (c >= C) break;
+        const int s = c * kDispatchThreads + tid;
+        const int e = ec[c];
+        if (e >= 0) {
+            const int pos = off[e] + wh[(c * NW + warp) * E + e] + rc[c];
+            perm[pos] = s;
+            inv_perm[s] = pos;
+        } else if (s < S) {
+            inv_perm[s] = -1;
+        }
+    }
+}
+
 // ===========================================================================
 // Step 4 (unfused): out[t,:] = residual + sum_k gate[t,k] * y_sorted[inv[t*K+k],:]
 // One thread per 4 consecutive outputs; k in ascending order.
@@ -987,6 +1094,21 @@ cudaError_t route_any(const moe_dims &d, int T, const void *x, const void *wr, f
 
 cudaError_t dispatch_any(const moe_dims &d, int T, const int32_t *idx, int32_t *counts,
                          int32_t *offsets, int32_t *perm, int32_t *inv, cudaStream_t st) {
+    const long long S = (long long)T * d.top_k;
+    const long long C = (S + kDispatchThreads - 1) / kDispatchThreads;
+    const size_t wh_bytes = (size_t)C * (kDispatchThreads / 32) * d.n_experts * sizeof(int);
+    if (C >= 1 && C <= kFastMaxChunks && wh_bytes <= kFastDispatchSmem) {
+        cudaError_t e = cudaFuncSetAttribute((const void *)k_dispatch_fast,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kFastDispatchSmem);
+        if (e != cudaSuccess) return e;
+        int Sv = (int)S, E = d.n_experts;
+        unsigned *err = device_info().err;
+        void *args[] = {&Sv, &E, &idx, &counts, &offsets, &perm, &inv, &err};
+        LaunchScope ls("dispatch", st);
+        return launch_pdl((const void *)k_dispatch_fast, dim3(1), dim3(kDispatchThreads), wh_bytes,
+                          st, args);
+    }
     LaunchScope ls("dispatch", st);
     k_dispatch<<<1, kDispatchThreads, 0, st>>>(T * d.top_k, d.n_experts, idx, counts, offsets,
                                                perm, inv, device_info().err);
