@@ -295,7 +295,10 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
         }
         __syncthreads();
         ptx::grid_dependency_wait();  // x may come from the previous kernel
-        if (!stage_router<TW>(wsm, wr, (uint32_t)((size_t)D * E * sizeof(TW)), &bar, err)) return;
+        const bool ok =
+            stage_router<TW>(wsm, wr, (uint32_t)((size_t)D * E * sizeof(TW)), &bar, err);
+        // a wait that gave up (recorded in err) ends the whole block, never part of it
+        if (!__syncthreads_and(ok)) return;
         staged_batch<TX, TW>(0, T, D, E, K, x, reinterpret_cast<const TW *>(wsm), part, lg, pk,
                              logits_opt, topk_idx, topk_gate, sidx);
     } else {
