@@ -620,7 +620,8 @@ def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5, prefill=F
         step(i)
     ms, launches, kstats = layer.time_steps(step, steps)
     sa_names = ("sa_prenorm", "qkv_rows_tc", "qkv_gemm_tc", "rope_cache", "attention_tc",
-                "attention", "attn_merge", "o_rows_tc", "o_gemm_tc", "residual_add")
+                "attention", "attn_merge", "o_rows_tc", "o_gemm_tc", "residual_add",
+                "residual_prenorm")
     sa_ms = sum(v[1] for k, v in kstats.items() if k in sa_names) / steps
     b = sa_bytes(a, T, ctx_len)
     peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))

@@ -463,6 +463,65 @@ k_residual_add(long long n4, int n_part, float *__restrict__ resid, const float 
     }
 }
 
+// Decoder layers: resid[t] += sum of the partial projections, then the MoE
+// block's input xn[t] = bf16(RMSNorm0(resid[t])) -- the residual add of the
+// attention block and the pre-norm of the MoE block in one pass, one
+// 1024-thread block per token (D/4 <= 4 * 1024 keeps the row in registers).
+constexpr int kResNormVec = 4;  // float4 per thread held in registers
+
+__global__ void __launch_bounds__(kNormThreads)
+k_residual_prenorm(int T, int D, int n_part, float *__restrict__ resid, const float *__restrict__ y,
+                   bf16 *__restrict__ xn, float eps) {
+    ptx::grid_dependency_wait();
+    __shared__ float red[kNormThreads / 32];
+    const int t = blockIdx.x;
+    const int nv = D >> 2;
+    const long long stride4 = (long long)T * nv;  // between partial projections, in float4
+    float4 *r = reinterpret_cast<float4 *>(resid + (size_t)t * D);
+    const float4 *a = reinterpret_cast<const float4 *>(y + (size_t)t * D);
+    float4 keep[kResNormVec];
+    float ss = 0.f;
+#pragma unroll
+    for (int u = 0; u < kResNormVec; ++u) {
+        const int i = threadIdx.x + u * kNormThreads;
+        keep[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < nv) {
+            float4 w = a[i];
+            for (int k = 1; k < n_part; ++k) {
+                const float4 v = a[k * stride4 + i];
+                w.x += v.x;
+                w.y += v.y;
+                w.z += v.z;
+                w.w += v.w;
+            }
+            float4 v = r[i];
+            v.x += w.x;
+            v.y += w.y;
+            v.z += w.z;
+            v.w += w.w;
+            r[i] = v;
+            keep[u] = v;
+            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+    }
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < kNormThreads / 32; ++w) tot += red[w];
+    const float sc = 1.0f / sqrtf(tot / (float)D + eps);
+    __nv_bfloat162 *o = reinterpret_cast<__nv_bfloat162 *>(xn + (size_t)t * D);
+#pragma unroll
+    for (int u = 0; u < kResNormVec; ++u) {
+        const int i = threadIdx.x + u * kNormThreads;
+        if (i < nv) {
+            o[2 * i] = __floats2bfloat162_rn(keep[u].x * sc, keep[u].y * sc);
+            o[2 * i + 1] = __floats2bfloat162_rn(keep[u].z * sc, keep[u].w * sc);
+        }
+    }
+}
+
 // ---- host ------------------------------------------------------------------------
 
 struct SaWs {
@@ -629,7 +688,10 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
 }
 
 // resid += W_o . ctx
-cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *resid) {
+// resid += W_o . ctx; with xn_next (decoder layers, D <= 4 * 4 * 1024) the
+// MoE block's normalised input is written in the same pass.
+cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *resid,
+                     bf16 *xn_next = nullptr, float eps = 0.f) {
     const moe_dims pd = proj_dims(c.d.d_model, c.nq());
     const int32_t *offsets = at<int32_t>(c.ws, c.L.offsets);
     float *y = at<float>(c.ws, c.L.qkv);
@@ -642,6 +704,14 @@ cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *r
         e = launch_gemm_down_tc(pd, c.T, ctx, offsets, w_o, y, c.st, "o_gemm_tc");
     }
     if (e != cudaSuccess) return e;
+    if (xn_next) {
+        int Tv = c.T, D = c.d.d_model;
+        const float *yc = y;
+        void *args[] = {&Tv, &D, &n_part, &resid, &yc, &xn_next, &eps};
+        LaunchScope ls("residual_prenorm", c.st);
+        return launch_pdl((const void *)k_residual_prenorm, dim3(c.T), dim3(kNormThreads), 0, c.st,
+                          args);
+    }
     long long n4 = (long long)c.T * c.d.d_model / 4;
     const long long cap = (long long)device_info().sm_count * 8;
     const int grid = (int)std::max(1LL, std::min((n4 + 255) / 256, cap));
@@ -669,6 +739,46 @@ moe_status setup_dispatch(const SaCall &c) {
 }  // namespace moe
 
 using namespace moe;
+
+namespace {
+
+moe_status sa_forward_impl(const moe_sa_dims *dims, int32_t T, const int32_t *seq,
+                           const int32_t *pos, int32_t n_seq, int32_t max_len, float *resid,
+                           const void *w_qkv, const void *w_o, void *k_cache, void *v_cache,
+                           float eps, void *ws, size_t ws_bytes, moe_stream_t stream,
+                           bf16 *xn_next) {
+    moe_status s = check_sa_call(dims, T, seq, pos, n_seq, max_len);
+    if (s != MOE_OK) return s;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(resid) || !ok_ptr(w_qkv) || !ok_ptr(w_o) || !ok_ptr(k_cache) ||
+        !ok_ptr(v_cache) || !(eps > 0.f))
+        return MOE_ERR_INVALID_ARG;
+    if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
+    SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
+    if (!tc_path_ok(proj_dims(c.nr(), dims->d_model)) ||
+        !tc_path_ok(proj_dims(dims->d_model, c.nq())))
+        return MOE_ERR_UNSUPPORTED;
+    bf16 *xn = at<bf16>(ws, c.L.xn);
+    float *q = at<float>(ws, c.L.q);
+    bf16 *ctx = at<bf16>(ws, c.L.ctx);
+    {
+        int Tv = T, D = dims->d_model;
+        const float *rc = resid;
+        int32_t *off = at<int32_t>(ws, c.L.offsets);
+        void *args[] = {&Tv, &D, &rc, &xn, &eps, &off};
+        LaunchScope ls("sa_prenorm", c.st);
+        if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(kNormThreads), 0, c.st, args) !=
+            cudaSuccess)
+            return MOE_ERR_CUDA;
+    }
+    bf16 *q16 = tc_attention(T) ? at<bf16>(ws, c.L.q16) : nullptr;
+    cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache, q16);
+    if (e == cudaSuccess) e = attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx, q16);
+    if (e == cudaSuccess) e = out_proj(c, ctx, w_o, resid, xn_next, eps);
+    return cuda_status(e);
+}
+
+}  // namespace
 
 extern "C" {
 
@@ -717,45 +827,23 @@ moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq
                           const void *w_qkv, const void *w_o, void *k_cache, void *v_cache,
                           float eps, void *ws, size_t ws_bytes, moe_stream_t stream) {
     MOE_INJECT("moe_sa_forward");
-    moe_status s = check_sa_call(dims, T, seq, pos, n_seq, max_len);
-    if (s != MOE_OK) return s;
-    if (T == 0) return MOE_OK;
-    if (!ok_ptr(resid) || !ok_ptr(w_qkv) || !ok_ptr(w_o) || !ok_ptr(k_cache) ||
-        !ok_ptr(v_cache) || !(eps > 0.f))
-        return MOE_ERR_INVALID_ARG;
-    if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
-    SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
-    if (!tc_path_ok(proj_dims(c.nr(), dims->d_model)) ||
-        !tc_path_ok(proj_dims(dims->d_model, c.nq())))
-        return MOE_ERR_UNSUPPORTED;
-    bf16 *xn = at<bf16>(ws, c.L.xn);
-    float *q = at<float>(ws, c.L.q);
-    bf16 *ctx = at<bf16>(ws, c.L.ctx);
-    {
-        int Tv = T, D = dims->d_model;
-        const float *rc = resid;
-        int32_t *off = at<int32_t>(ws, c.L.offsets);
-        void *args[] = {&Tv, &D, &rc, &xn, &eps, &off};
-        LaunchScope ls("sa_prenorm", c.st);
-        if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(kNormThreads), 0, c.st, args) !=
-            cudaSuccess)
-            return MOE_ERR_CUDA;
-    }
-    bf16 *q16 = tc_attention(T) ? at<bf16>(ws, c.L.q16) : nullptr;
-    cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache, q16);
-    if (e == cudaSuccess) e = attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx, q16);
-    if (e == cudaSuccess) e = out_proj(c, ctx, w_o, resid);
-    return cuda_status(e);
+    return sa_forward_impl(dims, T, seq, pos, n_seq, max_len, resid, w_qkv, w_o, k_cache, v_cache,
+                           eps, ws, ws_bytes, stream, nullptr);
 }
+
 
 moe_status moe_decoder_workspace_size(const moe_sa_dims *attn, const moe_dims *moe_d,
                                       int32_t max_tokens, size_t *bytes) {
     if (!bytes) return MOE_ERR_INVALID_ARG;
-    size_t a = 0, b = 0;
+    size_t a = 0, b = 0, c = 0;
     moe_status s = moe_sa_workspace_size(attn, max_tokens, &a);
     if (s != MOE_OK) return s;
-    if ((s = moe_stack_workspace_size(moe_d, max_tokens, &b)) != MOE_OK) return s;
-    *bytes = std::max(a, b);
+    if ((s = moe_workspace_size(moe_d, max_tokens, &b)) != MOE_OK) return s;
+    if ((s = moe_stack_workspace_size(moe_d, max_tokens, &c)) != MOE_OK) return s;
+    // the MoE block's normalised input, then the attention block's or the
+    // MoE layer's scratch (never live together)
+    const size_t xn = ((size_t)max_tokens * attn->d_model * 2 + 255) & ~size_t(255);
+    *bytes = std::max(xn + std::max(a, b), std::max(a, c));
     return MOE_OK;
 }
 
@@ -779,12 +867,29 @@ moe_status moe_decoder_forward(const moe_sa_dims *attn, const moe_dims *moe_d, i
     size_t need = 0;
     if ((s = moe_decoder_workspace_size(attn, moe_d, T, &need)) != MOE_OK) return s;
     if (!ws || !aligned16(ws) || ws_bytes < need) return MOE_ERR_WORKSPACE;
+    // the attention block's residual add and the MoE block's pre-norm run as
+    // one kernel when a row fits its registers; otherwise as the stack does
+    const bool fused = attn->d_model <= 4 * kResNormVec * kNormThreads;
+    const size_t xn_bytes = ((size_t)T * attn->d_model * 2 + 255) & ~size_t(255);
+    bf16 *xn = static_cast<bf16 *>(ws);
+    void *inner = static_cast<char *>(ws) + xn_bytes;
     for (int l = 0; l < n_layers; ++l) {
-        s = moe_sa_forward(attn, T, seq, pos, n_seq, max_len, resid, w_qkv[l], w_o[l],
-                           k_cache[l], v_cache[l], eps, ws, ws_bytes, stream);
-        if (s != MOE_OK) return s;
-        s = moe_stack_forward(moe_d, 1, T, &w_router[l], &w1[l], &v1[l], &w2[l], resid, eps, ws,
-                              ws_bytes, stream);
+        if (fused) {
+            s = sa_forward_impl(attn, T, seq, pos, n_seq, max_len, resid, w_qkv[l], w_o[l],
+                                k_cache[l], v_cache[l], eps, inner, ws_bytes - xn_bytes, stream,
+                                xn);
+            if (s != MOE_OK) return s;
+            // resid <- resid + MoE_l(xn): the combine reads each residual
+            // element before it writes the same element
+            s = moe_layer_forward(moe_d, T, xn, w_router[l], w1[l], v1[l], w2[l], resid, resid,
+                                  inner, ws_bytes - xn_bytes, stream);
+        } else {
+            s = moe_sa_forward(attn, T, seq, pos, n_seq, max_len, resid, w_qkv[l], w_o[l],
+                               k_cache[l], v_cache[l], eps, ws, ws_bytes, stream);
+            if (s != MOE_OK) return s;
+            s = moe_stack_forward(moe_d, 1, T, &w_router[l], &w1[l], &v1[l], &w2[l], resid, eps,
+                                  ws, ws_bytes, stream);
+        }
         if (s != MOE_OK) return s;
     }
     return MOE_OK;
