@@ -130,6 +130,50 @@ __device__ __forceinline__ Tile tile_of(const int *tprefix, const int32_t *offse
     return t;
 }
 
+// The CTA's work as segments (unit u, k-blocks [kb0, kb1)).  Standard: units
+// b, b+G, ... whole.  Stream-K (down projection with a tail buffer, at least
+// as many units as CTAs): CTA b takes the contiguous share [W b/G, W (b+1)/G)
+// of the W = units x nk (unit, k-block) pairs, so every CTA does the same
+// amount of work; a share is at least nk long, so a unit is split at most
+// once -- into a head (k-block 0 on) and a tail (ending at nk).
+struct SegIter {
+    bool sk;
+    int nk, G;
+    long long pos, end;
+    __device__ __forceinline__ bool next(int n_units, int &u, int &kb0, int &kb1) {
+        if (sk) {
+            if (pos >= end) return false;
+            u = (int)(pos / nk);
+            kb0 = (int)(pos - (long long)u * nk);
+            kb1 = (int)min((long long)nk, kb0 + (end - pos));
+            pos += kb1 - kb0;
+            return true;
+        }
+        if (pos >= n_units) return false;
+        u = (int)pos;
+        kb0 = 0;
+        kb1 = nk;
+        pos += G;
+        return true;
+    }
+};
+
+__device__ __forceinline__ SegIter make_segs(bool sk, int n_units, int nk) {
+    SegIter it;
+    it.sk = sk;
+    it.nk = nk;
+    it.G = gridDim.x;
+    if (sk) {
+        const long long W = (long long)n_units * nk;
+        it.pos = W * blockIdx.x / gridDim.x;
+        it.end = W * (blockIdx.x + 1) / gridDim.x;
+    } else {
+        it.pos = blockIdx.x;
+        it.end = 0;
+    }
+    return it;
+}
+
 // ---- the kernel ------------------------------------------------------------------
 
 template <int MODE, class C>
@@ -137,10 +181,13 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
           const __grid_constant__ CUtensorMap tmB1, const int32_t *__restrict__ offsets, int E,
           int S, int Kdim, int Nw, uint32_t a_bytes, bf16 *__restrict__ h_out,
-          float *__restrict__ y_out, unsigned *err) {
+          float *__restrict__ y_out, float *__restrict__ y_tail, unsigned *err) {
     // Kdim: reduction length (D for UP, F for DOWN); Nw: weight rows per
     // expert (F for UP, D for DOWN) = the output width.  a_bytes: bytes of
-    // the A box (rows x 128 B).  In a decode batch an expert holds at most T
+    // the A box (rows x 128 B).  y_tail (DOWN, optional): the second output
+    // buffer of the stream-K schedule (SegIter): heads go to y_out, tails to
+    // y_tail, and a unit done whole zeroes its part of y_tail, so the caller
+    // adds y_out + y_tail.  In a decode batch an expert holds at most T
     // slots, so only ceil(T/16)*16 rows are loaded; the MMA still reads 128
     // rows and the rows past the box give accumulator rows nobody stores.
     extern __shared__ unsigned char smem_raw[];
@@ -176,6 +223,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     tc_fence_after();
     const uint32_t tmem = hd->tmem_base;
     const int n_tiles = hd->tprefix[E];
+    const bool sk = MODE == kDown && y_tail != nullptr && n_tiles >= (int)gridDim.x;
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -184,10 +232,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             const uint64_t pol_b = ptx::policy_evict_first();
             uint32_t it = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < n_tiles && ok; u += gridDim.x) {
+            SegIter segs = make_segs(sk, n_tiles, nk);
+            int u, kb0, kb1;
+            while (ok && segs.next(n_tiles, u, kb0, kb1)) {
                 const Tile t = tile_of(hd->tprefix, offsets, E, ntn, u);
                 const int brow = t.e * Nw + t.nt * kCols;
-                for (int kb = 0; kb < nk; ++kb, ++it) {
+                for (int kb = kb0; kb < kb1; ++kb, ++it) {
                     const uint32_t s = it % kStages, ph = (it / kStages) & 1;
                     if (!(ok = ptx::mbar_wait(&hd->empty[s], ph ^ 1, err))) break;
                     unsigned char *sa = smem + s * kStageBytes;
@@ -212,12 +262,14 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         if (lane == 0) {
             uint32_t it = 0, tl = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < n_tiles && ok; u += gridDim.x, ++tl) {
+            SegIter segs = make_segs(sk, n_tiles, nk);
+            int u, kb0, kb1;
+            for (; ok && segs.next(n_tiles, u, kb0, kb1); ++tl) {
                 const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
                 if (!(ok = ptx::mbar_wait(&hd->tempty[acc], aph ^ 1, err))) break;
                 tc_fence_after();
                 const uint32_t d_tmem = tmem + acc * BN;
-                for (int kb = 0; kb < nk; ++kb, ++it) {
+                for (int kb = kb0; kb < kb1; ++kb, ++it) {
                     const uint32_t s = it % kStages, ph = (it / kStages) & 1;
                     if (!(ok = ptx::mbar_wait(&hd->full[s], ph, err))) break;
                     tc_fence_after();
@@ -226,7 +278,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk)
                         mma_bf16(d_tmem, adesc + 2 * kk, bdesc + 2 * kk, C::kIdesc,
-                                 (kb | kk) != 0 ? 1u : 0u);
+                                 (kb != kb0 || kk != 0) ? 1u : 0u);
                     mma_commit(&hd->empty[s]);  // stage free once these MMAs finish
                 }
                 if (ok) mma_commit(&hd->tfull[acc]);
@@ -241,9 +293,13 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         const int q = warp & 3;          // tensor-memory lane quarter of this warp
         const int m = q * 32 + lane;     // row of the tile = slot offset
         uint32_t tl = 0;
-        for (int u = blockIdx.x; u < n_tiles; u += gridDim.x, ++tl) {
+        SegIter segs = make_segs(sk, n_tiles, nk);
+        int u, kb0, kb1;
+        for (; segs.next(n_tiles, u, kb0, kb1); ++tl) {
             const Tile t = tile_of(hd->tprefix, offsets, E, ntn, u);
             const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
+            float *ydst = kb0 == 0 ? y_out : y_tail;          // head / tail of the unit
+            float *yzero = (y_tail && kb0 == 0 && kb1 == nk) ? y_tail : nullptr;
             if (!ptx::mbar_wait(&hd->tfull[acc], aph, err)) break;
             tc_fence_after();
             const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + acc * BN;
@@ -282,12 +338,20 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     tmem_ld32(base + c, v);
                     tmem_ld_wait();
                     if (row_ok) {
-                        float *dst = y_out + j * Nw + d0 + c;
+                        float *dst = ydst + j * Nw + d0 + c;
 #pragma unroll
                         for (int g = 0; g < 8; ++g)  // 4 columns per 16-byte store
                             if (d0 + c + g * 4 < Nw)
                                 *reinterpret_cast<float4 *>(dst + g * 4) =
                                     make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
+                        if (yzero) {
+                            float *z = yzero + j * Nw + d0 + c;
+#pragma unroll
+                            for (int g = 0; g < 8; ++g)
+                                if (d0 + c + g * 4 < Nw)
+                                    *reinterpret_cast<float4 *>(z + g * 4) =
+                                        make_float4(0.f, 0.f, 0.f, 0.f);
+                        }
                     }
                 }
             }
@@ -484,7 +548,8 @@ k_gather_rows(int S, int D, int K, const bf16 *__restrict__ x, const int32_t *__
 template <int MODE, class C>
 cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUtensorMap &b1,
                         const int32_t *offsets, int E, int S, int Kdim, int Nw, uint32_t a_bytes,
-                        bf16 *h_out, float *y_out, cudaStream_t st, const char *name = nullptr) {
+                        bf16 *h_out, float *y_out, cudaStream_t st, const char *name = nullptr,
+                        float *y_tail = nullptr) {
     const void *kern = (const void *)k_gemm_tc<MODE, C>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
@@ -492,7 +557,7 @@ cudaError_t launch_gemm(const CUtensorMap &a, const CUtensorMap &b0, const CUten
     unsigned *err = device_info().err;
     CUtensorMap ma = a, mb0 = b0, mb1 = b1;
     void *args[] = {&ma, &mb0, &mb1, &offsets, &E, &S, &Kdim, &Nw, &a_bytes, &h_out, &y_out,
-                    &err};
+                    &y_tail, &err};
     LaunchScope ls(name ? name : MODE == kUp ? "gemm_up_glu_tc" : "gemm_down_tc", st);
     return launch_pdl(kern, dim3(device_info().sm_count), dim3(kThreadsTc), C::kSmem, st, args);
 }
@@ -564,7 +629,7 @@ cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, co
 
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
-                                const char *name) {
+                                const char *name, float *y_tail) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
     const uint32_t arows = a_box_rows(T);
     CUtensorMap a, b0;
@@ -572,7 +637,7 @@ cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const i
         !make_map(&b0, w2, (uint64_t)E * D, (uint64_t)F, DownWide::BN))
         return cudaErrorInvalidValue;
     return launch_gemm<kDown, DownWide>(a, b0, b0, offsets, E, S, F, D, arows * BK * 2, nullptr,
-                                        y_sorted, st, name);
+                                        y_sorted, st, name, y_tail);
 }
 
 int gemm_rows_parts(int Kdim, int Nw) {

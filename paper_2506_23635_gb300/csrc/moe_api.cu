@@ -722,8 +722,9 @@ constexpr int kCombineMaxK = 256;  // = the largest top_k
 template <typename TO, typename TR>
 __global__ void __launch_bounds__(256)
 k_combine(int T, int D, int K, int n_part, const float *__restrict__ y,
-          const int32_t *__restrict__ inv, const float *__restrict__ gate,
-          const TR *__restrict__ residual, TO *__restrict__ out, unsigned *err) {
+          const float *__restrict__ y_tail, const int32_t *__restrict__ inv,
+          const float *__restrict__ gate, const TR *__restrict__ residual, TO *__restrict__ out,
+          unsigned *err) {
     __shared__ int s_j[kCombineMaxK];
     __shared__ float s_g[kCombineMaxK];
     ptx::grid_dependency_wait();
@@ -749,10 +750,19 @@ k_combine(int T, int D, int K, int n_part, const float *__restrict__ y,
                 if (j < 0) continue;
                 const float g = s_g[k];
                 const uint4 u = ld_stream16(y + (size_t)j * D + 4 * q);
-                a.x = fmaf(g, __uint_as_float(u.x), a.x);
-                a.y = fmaf(g, __uint_as_float(u.y), a.y);
-                a.z = fmaf(g, __uint_as_float(u.z), a.z);
-                a.w = fmaf(g, __uint_as_float(u.w), a.w);
+                float4 v = make_float4(__uint_as_float(u.x), __uint_as_float(u.y),
+                                       __uint_as_float(u.z), __uint_as_float(u.w));
+                if (y_tail) {  // head + tail of a split down projection, in that order
+                    const uint4 w = ld_stream16(y_tail + (size_t)j * D + 4 * q);
+                    v.x += __uint_as_float(w.x);
+                    v.y += __uint_as_float(w.y);
+                    v.z += __uint_as_float(w.z);
+                    v.w += __uint_as_float(w.w);
+                }
+                a.x = fmaf(g, v.x, a.x);
+                a.y = fmaf(g, v.y, a.y);
+                a.z = fmaf(g, v.z, a.z);
+                a.w = fmaf(g, v.w, a.w);
             }
             if (residual) {
                 const float4 r = load4(residual + (size_t)t * D + 4 * q);
@@ -944,6 +954,8 @@ WsLayout ws_layout(const moe_dims &d, int64_t T) {
     // ungated expert outputs: the tensor-core path, and the fp32 path above
     // the fused-combine limit
     L.y = o; o += (bf || T > kFusedCombineMaxTokens) ? up(S * d.d_model * 4) : 0;
+    // the stream-K down projection's tails (bf16 decode batches)
+    L.y_tail = o; o += (bf && T <= kStreamKMaxTokens) ? up(S * d.d_model * 4) : 0;
     L.total = o;
     return L;
 }
@@ -1119,8 +1131,9 @@ cudaError_t dispatch_any(const moe_dims &d, int T, const int32_t *idx, int32_t *
 }
 
 template <typename TO, typename TR>
-cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const int32_t *inv,
-                           const float *gate, const void *res, void *out, cudaStream_t st) {
+cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const float *y_tail,
+                           const int32_t *inv, const float *gate, const void *res, void *out,
+                           cudaStream_t st) {
     // enough blocks for 8 per SM: a token's row is split into n_part slices
     // of at least 256 float4 when there are few tokens
     const int nq = d.d_model / 4;
@@ -1131,16 +1144,18 @@ cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const int32
     const TR *rp = static_cast<const TR *>(res);
     TO *op = static_cast<TO *>(out);
     unsigned *err = device_info().err;
-    void *args[] = {&Tv, &D, &K, &n_part, &y, &inv, &gate, &rp, &op, &err};
+    void *args[] = {&Tv, &D, &K, &n_part, &y, &y_tail, &inv, &gate, &rp, &op, &err};
     LaunchScope ls("combine", st);
     return launch_pdl((const void *)k_combine<TO, TR>, dim3(grid), dim3(256), 0, st, args);
 }
 
 cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t *inv,
-                        const float *gate, const void *res, void *out, cudaStream_t st) {
+                        const float *gate, const void *res, void *out, cudaStream_t st,
+                        const float *y_tail = nullptr) {
     // the residual has the output's dtype
-    if (d.out_dtype == MOE_BF16) return launch_combine<bf16, bf16>(d, T, y, inv, gate, res, out, st);
-    return launch_combine<float, float>(d, T, y, inv, gate, res, out, st);
+    if (d.out_dtype == MOE_BF16)
+        return launch_combine<bf16, bf16>(d, T, y, y_tail, inv, gate, res, out, st);
+    return launch_combine<float, float>(d, T, y, y_tail, inv, gate, res, out, st);
 }
 
 bool use_stream_path(const moe_dims &d, int T) {
@@ -1314,8 +1329,11 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
         float *y = at<float>(ws, L.y);
         e = launch_gather_rows(d, T, x, perm, xs, st);
         if (e == cudaSuccess) e = launch_gemm_up_tc(d, T, xs, offsets, w1, v1, h, st);
-        if (e == cudaSuccess) e = launch_gemm_down_tc(d, T, h, offsets, w2, y, st);
-        if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st);
+        // decode batches: the stream-K down projection keeps every SM busy
+        // when the selected experts give few weight tiles
+        float *y_tail = T <= kStreamKMaxTokens ? at<float>(ws, L.y_tail) : nullptr;
+        if (e == cudaSuccess) e = launch_gemm_down_tc(d, T, h, offsets, w2, y, st, nullptr, y_tail);
+        if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st, y_tail);
         return cuda_status(e);
     }
     e = launch_up_glu_gemv(d, T, x, perm, offsets, w1, v1, h, st);

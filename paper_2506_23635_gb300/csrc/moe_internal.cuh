@@ -158,8 +158,11 @@ struct LaunchScope {
 
 // Workspace layout of moe_layer_forward / moe_expert_ffn for T tokens.
 struct WsLayout {
-    size_t idx, gate, counts, offsets, perm, inv_perm, h, xs, y, total;
+    size_t idx, gate, counts, offsets, perm, inv_perm, h, xs, y, y_tail, total;
 };
+// Decode batches of up to this many tokens take the stream-K down projection
+// (a second [T*K, D] fp32 output, added by the combine).
+constexpr int kStreamKMaxTokens = 64;
 WsLayout ws_layout(const moe_dims &d, int64_t T);
 
 // Decode-path launchers (ffn_gemv.cu).
@@ -221,10 +224,12 @@ cudaError_t launch_attn_prefill_tc(int T, int Hq, int Hkv, int n_seq, int L, con
                                    const int32_t *pos, const void *q16, const void *k_cache,
                                    const void *v_cache, void *ctx, int *tile_ok, cudaStream_t st);
 
-// name: the profiling name of the launch (default "gemm_down_tc").
+// name: the profiling name of the launch (default "gemm_down_tc").  y_tail
+// (optional, [T*K, D]): the stream-K schedule's second output; the result is
+// then y_sorted + y_tail.
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
-                                const char *name = nullptr);
+                                const char *name = nullptr, float *y_tail = nullptr);
 
 // Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
 // kStreamMaxSlots slots; the GLU hidden vectors h are bf16.  Batches of at
