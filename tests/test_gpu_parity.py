@@ -22,9 +22,9 @@ def moe():
 
 # (D, F, E, K, T, dtype): tiny layer, ragged widths, K = E, E = 1,
 # E = 256, minimum widths, token counts on both sides of the fused combine
-# limit (64), and a prefill-like batch whose experts hold 2-3 slot tiles
-# (two slot tiles per tensor-core work unit, with a one-tile remainder and
-# ragged reduction and output widths).
+# limit (64), a prefill-like batch whose experts hold 2-3 slot tiles (ragged
+# reduction and output widths), and a decode batch with more down-projection
+# tiles than SMs (the stream-K schedule splits tiles into heads and tails).
 SMALL = [
     (256, 512, 4, 2, 8, "f32"),
     (64, 96, 8, 2, 1, "bf16"),
@@ -36,6 +36,7 @@ SMALL = [
     (8, 8, 3, 2, 300, "f32"),
     (264, 520, 16, 4, 64, "bf16"),
     (200, 264, 3, 2, 400, "bf16"),
+    (4096, 256, 16, 4, 16, "bf16"),  # ~250 down-projection tiles: stream-K heads and tails
 ]
 
 
