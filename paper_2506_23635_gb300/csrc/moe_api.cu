@@ -345,17 +345,36 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
 // ---------------------------------------------------------------------------
 // Route and dispatch of a decode batch (T <= 64, T*K <= 256) in one launch of
 // a cluster of kClusterCtas CTAs.  CTA r bulk-copies rows [d0_r, d1_r) of W_r
-// into its shared memory and computes the partial logits of every token over
-// that slice of d; after a cluster barrier CTA 0 adds the kClusterCtas
-// partials in rank order (reading them through distributed shared memory),
-// selects the top-k of every token and ranks all T*K slots with a stable
-// counting sort, as k_dispatch does.  A second cluster barrier keeps the
-// other CTAs (and their shared memory) alive until CTA 0 has read it.
+// (before waiting for the previous kernel: the router is a weight) and the
+// same columns of every token row of x into its shared memory, and computes
+// the partial logits of every token over that slice of d.  After a cluster
+// barrier, token t is finished by one warp of CTA t mod kClusterCtas: it adds
+// the kClusterCtas partials in rank order (through distributed shared
+// memory), selects the top-k and writes the slot experts into CTA 0's shared
+// memory.  After a second cluster barrier (every partial read, every slot
+// written) CTA 0 ranks all T*K slots with a stable counting sort, as
+// k_dispatch does, and the other CTAs leave.
 // ---------------------------------------------------------------------------
 constexpr int kClusterCtas = 8;
 constexpr int kClusterThreads = 256;
 constexpr int kClusterMaxTokens = 64;
 constexpr int kClusterMaxSlots = 256;
+constexpr size_t kClusterMaxSmem = 192 * 1024;  // + ~28 KB static, within 227 KB
+
+// Rows of d per CTA (the largest slice) and the byte stride of a staged token
+// row: the slice plus 16 bytes, so that the rows of neighbouring tokens start
+// in different shared-memory banks.
+__host__ __device__ inline int cluster_rows(int D) {
+    return (D / 8 + kClusterCtas - 1) / kClusterCtas * 8;
+}
+__host__ __device__ inline size_t cluster_x_stride(int D, int x_bytes) {
+    return (size_t)cluster_rows(D) * x_bytes + 16;
+}
+// dynamic shared memory: partial logits [T][E] fp32 (128-byte rounded), the
+// router slice [rows][E], the token slices [T][stride]
+__host__ __device__ inline size_t cluster_part_bytes(int T, int E) {
+    return (((size_t)T * E * 4) + 127) & ~size_t(127);
+}
 
 template <typename TX, typename TW>
 __global__ void __launch_bounds__(kClusterThreads)
@@ -367,15 +386,19 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ __align__(128) unsigned char dsm[];
-    // dynamic: partial logits [T][E] fp32, then the staged router slice
+    constexpr int NW = kClusterThreads / 32;
     float *part = reinterpret_cast<float *>(dsm);
-    const size_t part_bytes = (((size_t)T * E * 4) + 127) & ~size_t(127);
+    const size_t part_bytes = cluster_part_bytes(T, E);
+    const int rows = cluster_rows(D);
     TW *wr_s = reinterpret_cast<TW *>(dsm + part_bytes);
-    __shared__ float pk[kStagedWarps][256];
+    unsigned char *x_s = dsm + part_bytes + (size_t)rows * E * sizeof(TW);
+    const size_t xs_stride = cluster_x_stride(D, (int)sizeof(TX));
+    __shared__ float lg[NW][256];
+    __shared__ float pk[NW][256];
     __shared__ int sidx[kClusterMaxSlots];
     __shared__ int cnt[256], run[256];
-    __shared__ int wh[kClusterThreads / 32][256];
-    __shared__ uint64_t bar;
+    __shared__ int wh[NW][256];
+    __shared__ uint64_t bar[2];
     const int rank = (int)cluster.block_rank();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     // this CTA's rows of d, a multiple of 8 rows (16-byte aligned slices)
@@ -385,19 +408,41 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
     const int dn = d1 - d0;
 
     if (tid == 0) {
-        ptx::mbar_init(&bar, 1);
+        ptx::mbar_init(&bar[0], 1);
+        ptx::mbar_init(&bar[1], 1);
         ptx::fence_barrier_init();
     }
     __syncthreads();
+    if (tid == 0 && dn > 0) {
+        const uint32_t bytes = (uint32_t)((size_t)dn * E * sizeof(TW));
+        const uint64_t pol = ptx::policy_evict_last();
+        ptx::mbar_arrive_expect_tx(&bar[0], bytes);
+        constexpr uint32_t kChunk = 32768;
+        for (uint32_t o = 0; o < bytes; o += kChunk)
+            ptx::bulk_g2s(reinterpret_cast<unsigned char *>(wr_s) + o,
+                          reinterpret_cast<const unsigned char *>(wr + (size_t)d0 * E) + o,
+                          min(kChunk, bytes - o), &bar[0], pol);
+    }
     ptx::grid_dependency_wait();  // x may come from the previous kernel
+    if (warp == 0 && dn > 0) {
+        // one bulk copy per token row: dn elements from column d0 (16-byte
+        // aligned because D and d0 are multiples of 8)
+        const uint32_t row_bytes = (uint32_t)((size_t)dn * sizeof(TX));
+        const uint64_t pol = ptx::policy_evict_first();
+        if (lane == 0) ptx::mbar_arrive_expect_tx(&bar[1], row_bytes * (uint32_t)T);
+        __syncwarp();
+        for (int t = lane; t < T; t += 32)
+            ptx::bulk_g2s(x_s + (size_t)t * xs_stride, x + (size_t)t * D + d0, row_bytes,
+                          &bar[1], pol);
+    }
     bool ok = true;
-    if (dn > 0)
-        ok = stage_router<TW>(reinterpret_cast<unsigned char *>(wr_s), wr + (size_t)d0 * E,
-                              (uint32_t)((size_t)dn * E * sizeof(TW)), &bar, err);
+    if (dn > 0) {
+        ok = ptx::mbar_wait(&bar[0], 0, err);
+        ok = ptx::mbar_wait(&bar[1], 0, err) && ok;
+    }
     // partial logits: token t is taken by a group of P threads (P = 256/T,
     // at most 32), thread p of the group accumulating 16 experts over rows
     // p, p+P, ... of the slice; the group then adds its P sums with shuffles
-    const int O = T * E;
     int P = 32;
     while (P > 1 && P * T > kClusterThreads) P >>= 1;
     const int groups = kClusterThreads / P;
@@ -405,7 +450,7 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
     const bool vec = (E % 8) == 0 && sizeof(TW) == 2;
     for (int t0 = 0; t0 < T; t0 += groups) {
         const int t = t0 + tid / P;
-        const TX *xr = x + (size_t)(t < T ? t : 0) * D + d0;
+        const TX *xr = reinterpret_cast<const TX *>(x_s + (size_t)(t < T ? t : 0) * xs_stride);
         for (int e0 = 0; e0 < E; e0 += 16) {
             const int ne = min(16, E - e0);
             float acc[16];
@@ -448,20 +493,21 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
         }
     }
     cluster.sync();  // every CTA's partials are written
-    if (rank == 0) {
-        for (int o = tid; o < O; o += kClusterThreads) {
+    // token t: warp (t / kClusterCtas) mod NW of CTA t mod kClusterCtas
+    int *sidx0 = cluster.map_shared_rank(sidx, 0);
+    for (int t = rank + kClusterCtas * warp; t < T; t += kClusterCtas * NW) {
+        for (int e = lane; e < E; e += 32) {
             float v = 0.f;
-            for (int r = 0; r < kClusterCtas; ++r) v += cluster.map_shared_rank(part, r)[o];
-            part[o] = v;  // own partial was read first (r = 0)
+            for (int r = 0; r < kClusterCtas; ++r)
+                v += cluster.map_shared_rank(part, r)[(size_t)t * E + e];
+            lg[warp][e] = v;
         }
+        __syncwarp();
+        select_topk(E, K, t, lg[warp], pk[warp], nullptr, topk_idx, topk_gate, sidx0 + t * K);
+        __syncwarp();
     }
-    cluster.sync();  // CTA 0 has read every partial; the others may leave
+    cluster.sync();  // every partial is read and every slot is in CTA 0
     if (rank != 0) return;
-    __syncthreads();
-    // top-k of every token, one warp per token
-    for (int t = warp; t < T; t += kClusterThreads / 32)
-        select_topk(E, K, t, part + (size_t)t * E, pk[warp], nullptr, topk_idx, topk_gate,
-                    sidx + t * K);
     // stable dispatch of the S <= 256 slots (one chunk of k_dispatch)
     const int S = T * K;
     for (int e = tid; e < E; e += kClusterThreads) cnt[e] = 0;
@@ -488,7 +534,6 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
         }
         if (lane == 0) offsets[E] = carry;
     }
-    constexpr int NW = kClusterThreads / 32;
     for (int i = tid; i < NW * E; i += kClusterThreads) wh[i / E][i % E] = 0;
     __syncthreads();
     const int sl = tid;
@@ -1031,6 +1076,15 @@ cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x,
     return launch_pdl(kern, dim3(1), dim3(kStagedThreads), staged ? wrb : 0, st, args);
 }
 
+// Dynamic shared memory of the cluster kernel: the partial logits, one CTA's
+// slice of the router and the same slice of every token row.
+size_t cluster_smem_bytes(const moe_dims &d, int T) {
+    const int wb = d.w_dtype == MOE_BF16 ? 2 : 4, xb = d.x_dtype == MOE_BF16 ? 2 : 4;
+    return cluster_part_bytes(T, d.n_experts) +
+           (size_t)cluster_rows(d.d_model) * d.n_experts * wb +
+           (size_t)T * cluster_x_stride(d.d_model, xb);
+}
+
 template <typename TX, typename TW>
 cudaError_t launch_route_dispatch_cluster(const moe_dims &d, int T, const void *x,
                                           const void *wr, int32_t *idx, float *gate,
@@ -1040,9 +1094,7 @@ cudaError_t launch_route_dispatch_cluster(const moe_dims &d, int T, const void *
     const TX *xp = static_cast<const TX *>(x);
     const TW *wp = static_cast<const TW *>(wr);
     unsigned *err = device_info().err;
-    const int rows = (D / 8 + kClusterCtas - 1) / kClusterCtas * 8;
-    const size_t part_bytes = (((size_t)T * E * 4) + 127) & ~size_t(127);
-    const size_t smem = part_bytes + (size_t)rows * E * sizeof(TW);
+    const size_t smem = cluster_smem_bytes(d, T);
     const void *kern = (const void *)k_route_dispatch_cluster<TX, TW>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
@@ -1066,14 +1118,9 @@ cudaError_t launch_route_dispatch_cluster(const moe_dims &d, int T, const void *
     return cudaLaunchKernelExC(&cfg, kern, args);
 }
 
-// Shared memory of the cluster kernel: the partial logits and one CTA's
-// eighth of the router.
 bool cluster_route_ok(const moe_dims &d, int T) {
     if (T < 1 || T > kClusterMaxTokens || T * d.top_k > kClusterMaxSlots) return false;
-    const int rows = (d.d_model / 8 + kClusterCtas - 1) / kClusterCtas * 8;
-    const size_t smem = (((size_t)T * d.n_experts * 4) + 127) +
-                        (size_t)rows * d.n_experts * (d.w_dtype == MOE_BF16 ? 2 : 4);
-    return smem <= 160 * 1024;
+    return cluster_smem_bytes(d, T) <= kClusterMaxSmem;
 }
 
 cudaError_t route_dispatch_cluster_any(const moe_dims &d, int T, const void *x, const void *wr,
