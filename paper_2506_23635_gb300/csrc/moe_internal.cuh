@@ -231,6 +231,17 @@ cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const i
                                 const void *w2, float *y_sorted, cudaStream_t st,
                                 const char *name = nullptr, float *y_tail = nullptr);
 
+// Prefill forms of the two grouped GEMMs (ffn_tc_wm.cu): the expert weights
+// as the MMA's M operand, the slots as a per-tile N; chosen by
+// launch_gemm_up_tc / launch_gemm_down_tc above kWmMinTokens tokens.
+constexpr int kWmMinTokens = 65;
+cudaError_t launch_gemm_up_wm(const moe_dims &d, int T, const void *x_sorted,
+                              const int32_t *offsets, const void *w1, const void *v1, void *h,
+                              cudaStream_t st);
+cudaError_t launch_gemm_down_wm(const moe_dims &d, int T, const void *h, const int32_t *offsets,
+                                const void *w2, float *y_sorted, cudaStream_t st,
+                                const char *name);
+
 // Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
 // kStreamMaxSlots slots; the GLU hidden vectors h are bf16.  Batches of at
 // most kStreamMaxTokens tokens take them; larger ones take the tcgen05 GEMMs.

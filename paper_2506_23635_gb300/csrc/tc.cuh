@@ -53,6 +53,48 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
         : "memory");
 }
 
+// ---- CTA pairs (cta_group::2): one MMA over the tensor cores of two SMs ----
+//
+// A pair is CTAs 2i and 2i+1 of a cluster.  One warp of EACH CTA allocates
+// and frees tensor memory collectively (the same columns in both SMs); the
+// even CTA issues the MMAs: M = 256 rows of A (rows 0-127 from its own
+// shared memory, rows 128-255 from the odd CTA's, at the same offsets), N
+// columns of B (the first N/2 from its own shared memory, the rest from the
+// odd CTA's), accumulator rows 0-127 in its tensor memory and 128-255 in the
+// odd CTA's, at the same column address.
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *holder, uint32_t cols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     ptx::smem_u32(holder)),
+                 "r"(cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t cols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                              uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on the mbarrier at this offset in every CTA of cta_mask once all
+// earlier pair MMAs of this thread finish.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar, uint16_t cta_mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(ptx::smem_u32(bar)),
+        "h"(cta_mask)
+        : "memory");
+}
+
 // 32 consecutive fp32 columns of this warp's 32 tensor-memory lanes.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];

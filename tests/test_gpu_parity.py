@@ -156,6 +156,39 @@ def test_all_tokens_one_expert():
     assert_parity(to_numpy(out), want, "bf16", "one expert")
 
 
+@pytest.mark.parametrize("T", [256, 257, 513])
+def test_one_expert_slot_runs(T):
+    """Every token to the same top-1 expert with exactly T slots: the prefill
+    GEMMs cut an expert into runs of at most 256 slots (256 -> one full run,
+    257 -> 128 + 129, 513 -> 171 + 171 + 171); ragged F and D."""
+    m = moe()
+    D, F, E, K = 136, 200, 8, 1
+    shape = gen.LayerShape(D, F, E, K, "bf16")
+    x = gen.host_normal((4 * T, D), 1.0, "bf16", 29, "x")
+    x64 = gen.to_f64(x, "bf16")
+    col = np.zeros(D)
+    col[: D // 2] = 0.25
+    w_r = np.zeros((D, E), np.float64)
+    w_r[:, 5] = col
+    w_r = gen.store(w_r, "bf16")
+    proj = x64 @ gen.to_f64(w_r, "bf16")[:, 5]
+    xs = np.where((proj < 0)[:, None], -x64, x64)  # sign flips are exact in bf16
+    keep = np.abs(proj) > 0.1
+    xs = xs[keep][:T]
+    assert xs.shape[0] == T
+    xb = gen.store(xs, "bf16")
+    w1, v1, w2 = gen.host_expert_weights(shape, 29)
+    d = _dims(m, shape)
+    want, idx, _ = oracle.layer_tokens(xb, w_r, w1, v1, w2, "bf16", K)
+    assert np.all(idx == 5)
+    X, WR, W1, V1, W2 = (dev(a, "bf16") for a in (xb, w_r, w1, v1, w2))
+    counts, _, _, _ = m.dispatch(d, m.route(d, X, WR)[0])
+    assert counts.cpu().numpy()[5] == T
+    out = m.layer_forward(d, X, WR, W1, V1, W2)
+    assert m.get_last_error() == 0
+    assert_parity(to_numpy(out), want, "bf16", f"one expert, {T} slots")
+
+
 def test_empty_batch_is_a_no_op():
     m = moe()
     d = m.dims(64, 64, 4, 2)
