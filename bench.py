@@ -212,21 +212,36 @@ def measured_peaks():
         return {"hbm_gbs": HBM_FALLBACK_GBS}, "fallback"
 
 
-def source_digest() -> str:
-    """sha256 over the CUDA sources: ties a committed ncu counter to the code
-    it was taken on."""
+# The CUDA sources each measured kernel is built from (its translation unit
+# and the headers it includes); other kernels use every source.
+_STREAM_SRC = ("ffn_stream.cu", "ptx.cuh", "moe_internal.cuh")
+_GEMM_SRC = ("ffn_tc.cu", "ffn_tc_wm.cu", "tc.cuh", "ptx.cuh", "moe_internal.cuh")
+KERNEL_SOURCES = {
+    "up_glu_stream": _STREAM_SRC,
+    "down_combine_stream": _STREAM_SRC,
+    "gemm_up_glu_tc": _GEMM_SRC,
+    "gemm_down_tc": _GEMM_SRC,
+}
+
+
+def source_digest(kernel: str = None) -> str:
+    """sha256 over the CUDA sources of a kernel (all sources when it has no
+    entry in KERNEL_SOURCES): ties a committed ncu counter to the code it was
+    taken on."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2506_23635_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+    names = KERNEL_SOURCES.get(kernel) or [
+        n for n in os.listdir(csrc) if n.endswith((".cu", ".cuh"))]
+    for name in sorted(names):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()[:16]
 
 
 def committed_traffic(kernel: str, workload: str):
     """DRAM bytes per launch from the committed ncu summary for this kernel
-    and workload, or None if there is none or the sources changed since."""
+    and workload, or None if there is none or the kernel's sources changed
+    since."""
     path = os.path.join(ROOT, "profiles", f"ncu_{kernel}_{workload}.md")
     try:
         text = open(path).read()
@@ -234,7 +249,7 @@ def committed_traffic(kernel: str, workload: str):
         return None
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
     s = re.search(r"source_digest:\s*([0-9a-f]+)", text)
-    if not m or not s or s.group(1) != source_digest():
+    if not m or not s or s.group(1) != source_digest(kernel):
         return None
     return float(m.group(1))
 

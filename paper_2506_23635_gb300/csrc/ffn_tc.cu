@@ -616,7 +616,7 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
 
 cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, const int32_t *offsets,
                               const void *w1, const void *v1, void *h, cudaStream_t st) {
-    if (T >= kWmMinTokens) return launch_gemm_up_wm(d, T, x_sorted, offsets, w1, v1, h, st);
+    if (use_wm(d, T)) return launch_gemm_up_wm(d, T, x_sorted, offsets, w1, v1, h, st);
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
     const uint32_t arows = a_box_rows(T);
     CUtensorMap a, b0, b1;
@@ -631,7 +631,7 @@ cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted, co
 cudaError_t launch_gemm_down_tc(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
                                 const char *name, float *y_tail) {
-    if (T >= kWmMinTokens && y_tail == nullptr)
+    if (use_wm(d, T) && y_tail == nullptr)
         return launch_gemm_down_wm(d, T, h, offsets, w2, y_sorted, st, name);
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
     const uint32_t arows = a_box_rows(T);

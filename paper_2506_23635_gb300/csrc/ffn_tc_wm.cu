@@ -28,11 +28,11 @@
 // G takes units b, b+G, ...
 //
 // Per CTA, 6 warps:
-//   warp 0     TMA producer (one lane): the A tile and a fixed box of slot
-//              rows (256 per tile, 128 per CTA of a pair; rows past the run
-//              are loaded and not used) into a ring of stages -- each copy
-//              instruction costs more than its bytes, and two per stage ran
-//              1.2-1.3x faster than one per 16-128-row piece;
+//   warp 0     TMA producer (one lane): the A tile and the run's slot rows
+//              (N, or N/2 per CTA of a pair, as one box: a tensor map per box
+//              height) into a ring of stages -- a copy instruction costs more
+//              than its bytes: two per stage ran 1.2-1.3x faster than one per
+//              16-128-row piece;
 //              in a pair both CTAs' copies complete on the even CTA's
 //              barrier of the stage (cta_group::2 copies), which expects the
 //              bytes of both;
@@ -88,6 +88,12 @@ struct WmCfg {
     static_assert(kStages <= kWmMaxStages, "stages");
     static_assert(kStageBytes % 1024 == 0, "stages stay 1024-byte aligned");
     static_assert(kSmem <= 227 * 1024, "shared memory");
+};
+
+// The slot rows [S, Kdim] with box heights 16, 32, ..., 256 rows: map i
+// loads 16 (i + 1) rows.  A pair uses the first 8.
+struct SlotMaps {
+    CUtensorMap m[16];
 };
 
 struct WmHeader {
@@ -190,14 +196,14 @@ __device__ __forceinline__ void wm_tma3(void *dst_smem, const CUtensorMap *tmap,
 template <int MODE, int CG>
 __global__ void __launch_bounds__(kWmThreads, 1)
 k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
-          const __grid_constant__ CUtensorMap tmB, int a_mode, const int32_t *__restrict__ offsets,
+          const __grid_constant__ SlotMaps tmB, int a_mode, const int32_t *__restrict__ offsets,
           int E, int S, int Kdim, int Nw, bf16 *__restrict__ h_out, float *__restrict__ y_out,
           unsigned *err) {
     // DOWN: tmA0 = W2 [E*D, F] (128-row box).  UP, a_mode 0: tmA0 = W1 and
     // tmA1 = V1, [E*F, D] each (64-row boxes); a_mode 1 / 2: tmA0 = both as
     // one 3-D tensor [2][E*F][D] (box 64 rows x 2), W1 first (1) or V1
     // first (2).  tmB: the sorted slot rows [S, Kdim] (x_sorted for UP, h
-    // for DOWN), box kRowsB rows.  Kdim: reduction length; Nw: output width
+    // for DOWN).  Kdim: reduction length; Nw: output width
     // (F for UP, D for DOWN).
     using C = WmCfg<MODE, CG>;
     extern __shared__ unsigned char smem_raw[];
@@ -227,7 +233,7 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
         ptx::fence_barrier_init();
         ptx::prefetch_tmap(&tmA0);
         if (MODE == kWmUp && a_mode == 0) ptx::prefetch_tmap(&tmA1);
-        ptx::prefetch_tmap(&tmB);
+        ptx::prefetch_tmap(&tmB.m[C::kRowsB / 16 - 1]);
     }
     if (warp == 1) {
         if (CG == 2) tmem_alloc_pair(&hd->tmem_base, kWmTmemCols);
@@ -251,7 +257,8 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
             bool ok = true;
             for (int u = unit0; ok && u < n_units; u += ustride) {
                 const WmTile t = wm_tile(hd->tprefix, offsets, E, u, C::kGran);
-                const int brow = t.s0 + (int)rank * (t.n / CG);
+                const uint32_t rows_b = (uint32_t)(t.n / CG);  // a multiple of 16, <= kRowsB
+                const int brow = t.s0 + (int)(rank * rows_b);
                 const int arow = t.e * Nw + (t.wt * CG + (int)rank) * C::kOutPerCta;
 
                 for (int kb = 0; kb < nk; ++kb, ++it) {
@@ -263,7 +270,7 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
                     uint64_t *fb = &hd->full[s];
                     const uint32_t fbc = CG == 2 ? ptx::map_rank(ptx::smem_u32(fb), 0) : 0u;
                     // the even CTA expects the bytes of both CTAs of the pair
-                    if (issuer) ptx::mbar_arrive_expect_tx(fb, kStageBytes * CG);
+                    if (issuer) ptx::mbar_arrive_expect_tx(fb, (kStageA + rows_b * (kWmBK * 2)) * CG);
                     if (MODE == kWmUp && a_mode != 0) {
                         wm_tma3<CG>(sa, &tmA0, kx, arow, fb, fbc, pol_w);
                     } else {
@@ -271,7 +278,7 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
                         if (MODE == kWmUp)
                             wm_tma<CG>(sa + kStageA / 2, &tmA1, kx, arow, fb, fbc, pol_w);
                     }
-                    wm_tma<CG>(sb, &tmB, kx, brow, fb, fbc, pol_x);
+                    wm_tma<CG>(sb, &tmB.m[rows_b / 16 - 1], kx, brow, fb, fbc, pol_x);
                 }
             }
             // let copies still in flight land before the block can exit: the
@@ -417,13 +424,14 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
 }
 
 template <int MODE, int CG>
-cudaError_t launch_wm_cg(const CUtensorMap &a0, const CUtensorMap &a1, const CUtensorMap &b,
+cudaError_t launch_wm_cg(const CUtensorMap &a0, const CUtensorMap &a1, const SlotMaps &b,
                          int a_mode, const int32_t *offsets, int E, int S, int Kdim, int Nw,
                          bf16 *h, float *y, int grid, cudaStream_t st, const char *name) {
     using C = WmCfg<MODE, CG>;
     const void *kern = (const void *)k_gemm_wm<MODE, CG>;
     unsigned *err = device_info().err;
-    CUtensorMap m0 = a0, m1 = a1, mb = b;
+    CUtensorMap m0 = a0, m1 = a1;
+    SlotMaps mb = b;
     void *args[] = {&m0, &m1, &mb, &a_mode, &offsets, &E, &S, &Kdim, &Nw, &h, &y, &err};
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -441,6 +449,14 @@ cudaError_t launch_wm_cg(const CUtensorMap &a0, const CUtensorMap &a1, const CUt
     cfg.numAttrs = CG == 2 ? 2 : 1;
     LaunchScope ls(name, st);
     return cudaLaunchKernelExC(&cfg, kern, args);
+}
+
+// The first n maps of the slot rows [S, Kdim] (box heights 16, ..., 16 n).
+bool slot_maps(SlotMaps &b, const void *base, int S, int Kdim, int n) {
+    for (int i = 0; i < n; ++i)
+        if (!make_map(&b.m[i], base, (uint64_t)S, (uint64_t)Kdim, 16u * (i + 1))) return false;
+    for (int i = n; i < 16; ++i) b.m[i] = b.m[n - 1];
+    return true;
 }
 
 // CTA pairs when the device can keep pairs resident (one per two SMs), else
@@ -479,27 +495,23 @@ int wm_pairs() {
 }
 
 template <int MODE>
-cudaError_t launch_wm(const CUtensorMap (&a)[2], const CUtensorMap (&b)[2], int a_mode,
+cudaError_t launch_wm(const CUtensorMap (&a)[2], const void *slots, int a_mode,
                       const int32_t *offsets, int E, int S, int Kdim, int Nw, bf16 *h, float *y,
                       cudaStream_t st, const char *name) {
     const int pairs = wm_pairs<MODE>();
+    SlotMaps b;
+    if (!slot_maps(b, slots, S, Kdim, pairs > 0 ? 8 : 16)) return cudaErrorInvalidValue;
     if (pairs > 0)
-        return launch_wm_cg<MODE, 2>(a[0], a[1], b[1], a_mode, offsets, E, S, Kdim, Nw, h, y,
+        return launch_wm_cg<MODE, 2>(a[0], a[1], b, a_mode, offsets, E, S, Kdim, Nw, h, y,
                                      2 * pairs, st, name);
     const void *kern = (const void *)k_gemm_wm<MODE, 1>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)WmCfg<MODE, 1>::kSmem);
     if (e != cudaSuccess) return e;
-    return launch_wm_cg<MODE, 1>(a[0], a[1], b[0], a_mode, offsets, E, S, Kdim, Nw, h, y,
+    return launch_wm_cg<MODE, 1>(a[0], a[1], b, a_mode, offsets, E, S, Kdim, Nw, h, y,
                                  device_info().sm_count, st, name);
 }
 
-// The slot rows [S, Kdim] in the box of each form: 256 rows (one CTA per
-// tile), 128 rows (a pair).
-bool slot_maps(CUtensorMap (&b)[2], const void *base, int S, int Kdim) {
-    return make_map(&b[0], base, (uint64_t)S, (uint64_t)Kdim, WmCfg<kWmDown, 1>::kRowsB) &&
-           make_map(&b[1], base, (uint64_t)S, (uint64_t)Kdim, WmCfg<kWmDown, 2>::kRowsB);
-}
 
 // W1 and V1 [rows, cols] as one 3-D tensor [2][rows][cols] based at the
 // lower address, the higher one a stride away (box 64 columns x 64 rows x
@@ -528,7 +540,7 @@ cudaError_t launch_gemm_up_wm(const moe_dims &d, int T, const void *x_sorted,
                               const int32_t *offsets, const void *w1, const void *v1, void *h,
                               cudaStream_t st) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
-    CUtensorMap a[2], b[2];
+    CUtensorMap a[2];
     bool v1_first = false;
     int a_mode;
     if (weight_pair_map(&a[0], w1, v1, (uint64_t)E * F, (uint64_t)D, &v1_first)) {
@@ -540,8 +552,7 @@ cudaError_t launch_gemm_up_wm(const moe_dims &d, int T, const void *x_sorted,
             return cudaErrorInvalidValue;
         a_mode = 0;
     }
-    if (!slot_maps(b, x_sorted, S, D)) return cudaErrorInvalidValue;
-    return launch_wm<kWmUp>(a, b, a_mode, offsets, E, S, D, F, static_cast<bf16 *>(h), nullptr, st,
+    return launch_wm<kWmUp>(a, x_sorted, a_mode, offsets, E, S, D, F, static_cast<bf16 *>(h), nullptr, st,
                             "gemm_up_glu_tc");
 }
 
@@ -549,11 +560,10 @@ cudaError_t launch_gemm_down_wm(const moe_dims &d, int T, const void *h, const i
                                 const void *w2, float *y_sorted, cudaStream_t st,
                                 const char *name) {
     const int S = T * d.top_k, D = d.d_model, F = d.ffn_hidden, E = d.n_experts;
-    CUtensorMap a[2], b[2];
-    if (!make_map(&a[0], w2, (uint64_t)E * D, (uint64_t)F, 128) || !slot_maps(b, h, S, F))
-        return cudaErrorInvalidValue;
+    CUtensorMap a[2];
+    if (!make_map(&a[0], w2, (uint64_t)E * D, (uint64_t)F, 128)) return cudaErrorInvalidValue;
     a[1] = a[0];
-    return launch_wm<kWmDown>(a, b, 0, offsets, E, S, F, D, nullptr, y_sorted, st,
+    return launch_wm<kWmDown>(a, h, 0, offsets, E, S, F, D, nullptr, y_sorted, st,
                               name ? name : "gemm_down_tc");
 }
 

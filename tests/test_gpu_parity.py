@@ -160,18 +160,19 @@ def test_all_tokens_one_expert():
 def test_one_expert_slot_runs(T):
     """Every token to the same top-1 expert with exactly T slots: the prefill
     GEMMs cut an expert into runs of at most 256 slots (256 -> one full run,
-    257 -> 128 + 129, 513 -> 171 + 171 + 171); ragged F and D."""
+    257 -> 128 + 129, 513 -> 171 + 171 + 171); ragged F and D; the other
+    expert holds none."""
     m = moe()
-    D, F, E, K = 136, 200, 8, 1
+    D, F, E, K = 136, 200, 2, 1
     shape = gen.LayerShape(D, F, E, K, "bf16")
     x = gen.host_normal((4 * T, D), 1.0, "bf16", 29, "x")
     x64 = gen.to_f64(x, "bf16")
     col = np.zeros(D)
     col[: D // 2] = 0.25
     w_r = np.zeros((D, E), np.float64)
-    w_r[:, 5] = col
+    w_r[:, 1] = col
     w_r = gen.store(w_r, "bf16")
-    proj = x64 @ gen.to_f64(w_r, "bf16")[:, 5]
+    proj = x64 @ gen.to_f64(w_r, "bf16")[:, 1]
     xs = np.where((proj < 0)[:, None], -x64, x64)  # sign flips are exact in bf16
     keep = np.abs(proj) > 0.1
     xs = xs[keep][:T]
@@ -180,13 +181,41 @@ def test_one_expert_slot_runs(T):
     w1, v1, w2 = gen.host_expert_weights(shape, 29)
     d = _dims(m, shape)
     want, idx, _ = oracle.layer_tokens(xb, w_r, w1, v1, w2, "bf16", K)
-    assert np.all(idx == 5)
+    assert np.all(idx == 1)
     X, WR, W1, V1, W2 = (dev(a, "bf16") for a in (xb, w_r, w1, v1, w2))
     counts, _, _, _ = m.dispatch(d, m.route(d, X, WR)[0])
-    assert counts.cpu().numpy()[5] == T
+    assert counts.cpu().numpy()[1] == T
     out = m.layer_forward(d, X, WR, W1, V1, W2)
     assert m.get_last_error() == 0
     assert_parity(to_numpy(out), want, "bf16", f"one expert, {T} slots")
+
+
+@pytest.mark.parametrize("layout", ["w1_first", "v1_first", "same_tensor"])
+def test_prefill_weight_layouts(layout):
+    """The prefill up projection reads a tile of W1 and V1 rows as one copy
+    over both tensors when V1 lies a whole tensor or more after W1 or before
+    it, else as two copies (here: W1 and V1 the same tensor)."""
+    m = moe()
+    D, F, E, K, T = 136, 200, 2, 2, 160
+    L = _host((D, F, E, K, T, "bf16"), seed=31)
+    sh = L.shape
+    d = _dims(m, sh)
+    v1_host = L.w1 if layout == "same_tensor" else L.v1
+    want, idx, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, v1_host, L.w2, "bf16", K)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    if layout == "v1_first":
+        both = torch.empty((2,) + tuple(w1.shape), dtype=w1.dtype, device=w1.device)
+        both[0].copy_(v1)
+        both[1].copy_(w1)
+        v1, w1 = both[0], both[1]
+    elif layout == "w1_first":
+        both = torch.stack([w1, v1])
+        w1, v1 = both[0], both[1]
+    else:
+        v1 = w1
+    out = m.layer_forward(d, x, w_r, w1, v1, w2)
+    assert m.get_last_error() == 0
+    assert_parity(to_numpy(out), want, "bf16", f"prefill, {layout}")
 
 
 def test_empty_batch_is_a_no_op():
