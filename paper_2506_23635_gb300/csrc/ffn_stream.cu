@@ -93,6 +93,9 @@ k_up_glu_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ x,
     const int W = n_stages;  // consumer warps; warp W is the producer
 
     if (threadIdx.x == 0) init_header(hd, n_stages);
+    // one CTA per SM, all resident: the next kernel's CTAs can only take an
+    // SM this grid has left, so let them launch (and wait on the device) now
+    ptx::launch_dependents();
     ptx::grid_dependency_wait();  // perm/offsets come from the previous kernel
     if (warp == 0) chunk_prefix<NS>(offsets, E, S, hd->prefix, err);
     __syncthreads();
@@ -219,6 +222,7 @@ k_down_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ h,
     const int W = n_stages;  // consumer warps; warp W is the producer
 
     if (threadIdx.x == 0) init_header(hd, n_stages);
+    ptx::launch_dependents();  // as in k_up_glu_stream
     ptx::grid_dependency_wait();
     if (warp == 0) chunk_prefix<NS>(offsets, E, S, hd->prefix, err);
     __syncthreads();

@@ -216,8 +216,8 @@ __device__ __forceinline__ void warp_logits16(const TX *xrow, const TW *wr_s, in
 
 // Stage W_r into dynamic shared memory (bulk copies on one mbarrier).
 template <typename TW>
-__device__ __forceinline__ bool stage_router(unsigned char *dst, const TW *wr, uint32_t bytes,
-                                             uint64_t *bar, unsigned *err) {
+__device__ __forceinline__ void stage_router_issue(unsigned char *dst, const TW *wr, uint32_t bytes,
+                                                   uint64_t *bar) {
     if (threadIdx.x == 0) {
         const uint64_t pol = ptx::policy_evict_last();
         ptx::mbar_arrive_expect_tx(bar, bytes);
@@ -226,7 +226,6 @@ __device__ __forceinline__ bool stage_router(unsigned char *dst, const TW *wr, u
             ptx::bulk_g2s(dst + o, reinterpret_cast<const unsigned char *>(wr) + o,
                           min(kChunk, bytes - o), bar, pol);
     }
-    return ptx::mbar_wait(bar, 0, err);
 }
 
 // Logits + top-k of tokens [t0, t0+n) (n <= 8) by the 8 warps of the block.
@@ -294,9 +293,13 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
             ptx::fence_barrier_init();
         }
         __syncthreads();
+        // W_r does not come from the previous kernel: its copy starts before
+        // the dependency wait, and the next kernel may launch at once (its
+        // CTAs take the other SMs and wait for this one on the device)
+        stage_router_issue<TW>(wsm, wr, (uint32_t)((size_t)D * E * sizeof(TW)), &bar);
+        ptx::launch_dependents();
         ptx::grid_dependency_wait();  // x may come from the previous kernel
-        const bool ok =
-            stage_router<TW>(wsm, wr, (uint32_t)((size_t)D * E * sizeof(TW)), &bar, err);
+        const bool ok = ptx::mbar_wait(&bar, 0, err);
         // a wait that gave up (recorded in err) ends the whole block, never part of it
         if (!__syncthreads_and(ok)) return;
         staged_batch<TX, TW>(0, T, D, E, K, x, reinterpret_cast<const TW *>(wsm), part, lg, pk,

@@ -218,6 +218,27 @@ def test_prefill_weight_layouts(layout):
     assert_parity(to_numpy(out), want, "bf16", f"prefill, {layout}")
 
 
+@pytest.mark.parametrize("E,K", [(2, 1), (4, 4), (5, 3), (8, 2), (16, 4), (16, 16), (17, 4)])
+def test_one_token_layer(E, K):
+    """One token: the fused routing kernel and the two streaming kernels,
+    over expert counts and top-k widths (K = 1, K = E, E not a multiple of
+    8)."""
+    m = moe()
+    L = _host((136, 200, E, K, 1, "bf16"), seed=37)
+    sh = L.shape
+    d = _dims(m, sh)
+    want, _, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, "bf16", K)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    m.layer_forward(d, x, w_r, w1, v1, w2)
+    torch.cuda.synchronize()
+    n0 = m.launch_count()
+    out = m.layer_forward(d, x, w_r, w1, v1, w2)
+    torch.cuda.synchronize()
+    assert m.launch_count() - n0 == 3
+    assert m.get_last_error() == 0
+    assert_parity(to_numpy(out), want, "bf16", f"one token, E={E}, K={K}")
+
+
 def test_empty_batch_is_a_no_op():
     m = moe()
     d = m.dims(64, 64, 4, 2)
