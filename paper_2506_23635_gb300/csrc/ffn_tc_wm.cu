@@ -251,7 +251,10 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
-            const uint64_t pol_w = ptx::policy_evict_first();
+            // a weight tile serves the 2-3 slot runs of its expert on
+            // neighbouring pairs: normal priority keeps it in L2 between them
+            // (evict-first: 2-3% slower, DRAM reads 14% above the weights)
+            const uint64_t pol_w = ptx::policy_evict_normal();
             const uint64_t pol_x = ptx::policy_evict_last();
             uint32_t it = 0;
             bool ok = true;
