@@ -103,7 +103,11 @@ __device__ void block_logits(int D, int E, const TX *__restrict__ x, const TW *_
 }
 
 // Warp-level softmax + top-k of one token's logits l[0..E); writes
-// topk_idx/topk_gate[t*K + k] (and sidx[k] if non-null).
+// topk_idx/topk_gate[t*K + k] (and sidx[k] if non-null).  A NaN logit (a
+// token with a NaN or infinite component) ranks as -inf, so the K picks are
+// always distinct experts in [0, E) (K <= E): the indices that address the
+// dispatch arrays stay in range whatever the data; such a token's gates
+// are NaN.
 __device__ void select_topk(int E, int K, int t, const float *l, float *pk,
                             float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
                             float *__restrict__ topk_gate, int *sidx) {
@@ -125,7 +129,7 @@ __device__ void select_topk(int E, int K, int t, const float *l, float *pk,
         int bi = 0x7fffffff;
         for (int i = 0, e = lane; e < E; ++i, e += 32) {
             if ((taken >> i) & 1u) continue;
-            const float v = l[e];
+            const float v = isnan(l[e]) ? -INFINITY : l[e];
             if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
         }
 #pragma unroll
@@ -315,7 +319,11 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
     }
     if (warp != 0) return;
     const int S = T * K;
-    const int e = lane < S ? sidx[lane] : -1;
+    int e = lane < S ? sidx[lane] : -1;
+    if (e >= E) {  // cannot come from select_topk; never index with it
+        set_error(err, kErrIndex);
+        e = -1;
+    }
     if (e >= 0) atomicAdd(&cnt[e], 1);
     __syncwarp();
     int carry = 0;
@@ -515,7 +523,11 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
     const int S = T * K;
     for (int e = tid; e < E; e += kClusterThreads) cnt[e] = 0;
     __syncthreads();
-    for (int sl = tid; sl < S; sl += kClusterThreads) atomicAdd(&cnt[sidx[sl]], 1);
+    for (int sl = tid; sl < S; sl += kClusterThreads) {
+        const int e = sidx[sl];
+        if (e >= 0 && e < E) atomicAdd(&cnt[e], 1);
+        else set_error(err, kErrIndex);  // cannot come from select_topk
+    }
     __syncthreads();
     if (warp == 0) {
         int carry = 0;
@@ -540,7 +552,7 @@ k_route_dispatch_cluster(int T, int D, int E, int K, const TX *__restrict__ x,
     for (int i = tid; i < NW * E; i += kClusterThreads) wh[i / E][i % E] = 0;
     __syncthreads();
     const int sl = tid;
-    const int e = sl < S ? sidx[sl] : -1;
+    const int e = (sl < S && sidx[sl] >= 0 && sidx[sl] < E) ? sidx[sl] : -1;
     const unsigned same = __match_any_sync(0xffffffffu, e);
     const int rk = __popc(same & ((1u << lane) - 1u));
     if (e >= 0 && rk == 0) wh[warp][e] = __popc(same);

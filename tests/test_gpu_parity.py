@@ -239,6 +239,35 @@ def test_one_token_layer(E, K):
     assert_parity(to_numpy(out), want, "bf16", f"one token, E={E}, K={K}")
 
 
+@pytest.mark.parametrize("T", [1, 3, 70, 600])
+def test_nan_token_stays_contained(T):
+    """A token whose row is NaN (its logits are NaN) is routed to valid
+    experts, raises no device error and spoils only its own output row: the
+    other tokens match the oracle (one-token, cluster, large-batch and
+    prefill paths)."""
+    m = moe()
+    D, F, E, K = 136, 200, 8, 2
+    L = _host((D, F, E, K, T, "bf16"), seed=41)
+    sh = L.shape
+    d = _dims(m, sh)
+    x = gen.to_f64(L.x, "bf16").copy()
+    bad = T // 2
+    x[bad, :] = np.nan
+    xb = gen.store(x, "bf16")
+    X, WR, W1, V1, W2 = (dev(a, "bf16") for a in (xb, L.w_r, L.w1, L.v1, L.w2))
+    idx, _, _ = m.route(d, X, WR)
+    ii = idx.cpu().numpy()
+    assert ii.min() >= 0 and ii.max() < E
+    assert all(len(set(r)) == K for r in ii.tolist())
+    out = to_numpy(m.layer_forward(d, X, WR, W1, V1, W2))
+    assert m.get_last_error() == 0
+    assert not np.isfinite(out[bad]).any()
+    others = np.array([t for t in range(T) if t != bad], dtype=np.int32)
+    if others.size:
+        want, _, _ = oracle.layer_tokens(xb, L.w_r, L.w1, L.v1, L.w2, "bf16", K, tokens=others)
+        assert_parity(out[others], want, "bf16", f"tokens beside a NaN token, T={T}")
+
+
 def test_empty_batch_is_a_no_op():
     m = moe()
     d = m.dims(64, 64, 4, 2)
