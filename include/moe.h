@@ -95,7 +95,9 @@ moe_status moe_workspace_size(const moe_dims *dims, int32_t max_tokens,
  *   logits_opt [T, E]  float32, written if non-NULL
  *   topk_idx   [T, K]  int32 expert ids, descending logit, ties -> lower id
  *   topk_gate  [T, K]  float32 renormalised gates (sum over k is 1)
- * fp32 accumulation.  Errors: MOE_ERR_INVALID_ARG (nulls, sizes). */
+ * fp32 accumulation.  A NaN logit ranks below every number, so a token with
+ * a NaN (or infinite) component still gets K distinct experts in [0, E);
+ * its gates are NaN.  Errors: MOE_ERR_INVALID_ARG (nulls, sizes). */
 moe_status moe_route(const moe_dims *dims, int32_t T, const void *x,
                      const void *w_router, float *logits_opt,
                      int32_t *topk_idx, float *topk_gate, moe_stream_t stream);
@@ -247,7 +249,10 @@ moe_status moe_get_last_error(moe_stream_t stream);
  * the environment, the named entry point (moe_route, moe_dispatch,
  * moe_expert_ffn, moe_combine, moe_layer_forward, moe_layer_forward_dense,
  * moe_prenorm, moe_stack_forward, moe_sa_qkv, moe_sa_attend, moe_sa_forward,
- * moe_decoder_forward) returns that status at once without launching. */
+ * moe_decoder_forward) returns that status at once without launching.
+ * With MOE_WM_SINGLE_CTA=1 the prefill expert GEMMs (batches whose experts
+ * hold 128 or more slots on average) run one CTA per tile, the form used on
+ * devices that cannot keep CTA pairs resident, instead of CTA pairs. */
 moe_status moe_selftest_wait_timeout(uint64_t limit_ns, int32_t *gave_up,
                                      moe_stream_t stream);
 

@@ -51,6 +51,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <stdlib.h>
+
 #include <mutex>
 
 #include "tc.cuh"
@@ -497,11 +499,19 @@ int wm_pairs() {
     return cached[dev];
 }
 
+// The single-CTA form serves devices that cannot keep CTA pairs resident;
+// MOE_WM_SINGLE_CTA=1 in the environment (read on every call) selects it
+// anyway, so that it can be tested where pairs are available.
+bool single_cta_forced() {
+    const char *v = getenv("MOE_WM_SINGLE_CTA");
+    return v && v[0] == '1' && v[1] == 0;
+}
+
 template <int MODE>
 cudaError_t launch_wm(const CUtensorMap (&a)[2], const void *slots, int a_mode,
                       const int32_t *offsets, int E, int S, int Kdim, int Nw, bf16 *h, float *y,
                       cudaStream_t st, const char *name) {
-    const int pairs = wm_pairs<MODE>();
+    const int pairs = single_cta_forced() ? 0 : wm_pairs<MODE>();
     SlotMaps b;
     if (!slot_maps(b, slots, S, Kdim, pairs > 0 ? 8 : 16)) return cudaErrorInvalidValue;
     if (pairs > 0)

@@ -268,6 +268,26 @@ def test_nan_token_stays_contained(T):
         assert_parity(out[others], want, "bf16", f"tokens beside a NaN token, T={T}")
 
 
+@pytest.mark.parametrize("case", [(200, 264, 3, 2, 400), (136, 200, 2, 1, 513)],
+                         ids=lambda c: "D{}F{}E{}K{}T{}".format(*c))
+def test_prefill_single_cta_form(case, monkeypatch):
+    """The prefill GEMMs' one-CTA-per-tile form (MOE_WM_SINGLE_CTA=1) against
+    the oracle and against the CTA-pair form."""
+    m = moe()
+    D, F, E, K, T = case
+    L = _host((D, F, E, K, T, "bf16"), seed=43)
+    d = _dims(m, L.shape)
+    x, w_r, w1, v1, w2 = _devlayer(L)
+    pair = to_numpy(m.layer_forward(d, x, w_r, w1, v1, w2))
+    monkeypatch.setenv("MOE_WM_SINGLE_CTA", "1")
+    single = to_numpy(m.layer_forward(d, x, w_r, w1, v1, w2))
+    monkeypatch.delenv("MOE_WM_SINGLE_CTA")
+    assert m.get_last_error() == 0
+    want, _, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, "bf16", K)
+    assert_parity(single, want, "bf16", "single-CTA prefill GEMMs")
+    assert_parity(single, pair, "bf16", "single-CTA vs CTA-pair prefill GEMMs")
+
+
 def test_empty_batch_is_a_no_op():
     m = moe()
     d = m.dims(64, 64, 4, 2)
