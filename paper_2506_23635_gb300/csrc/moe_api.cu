@@ -102,55 +102,6 @@ __device__ void block_logits(int D, int E, const TX *__restrict__ x, const TW *_
     }
 }
 
-// Warp-level softmax + top-k of one token's logits l[0..E); writes
-// topk_idx/topk_gate[t*K + k] (and sidx[k] if non-null).  A NaN logit (a
-// token with a NaN or infinite component) ranks as -inf, so the K picks are
-// always distinct experts in [0, E) (K <= E): the indices that address the
-// dispatch arrays stay in range whatever the data; such a token's gates
-// are NaN.
-__device__ void select_topk(int E, int K, int t, const float *l, float *pk,
-                            float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
-                            float *__restrict__ topk_gate, int *sidx) {
-    const int lane = threadIdx.x & 31;
-    if (logits_opt)
-        for (int e = lane; e < E; e += 32) logits_opt[(size_t)t * E + e] = l[e];
-    float m = -INFINITY;
-    for (int e = lane; e < E; e += 32) m = fmaxf(m, l[e]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    float z = 0.f;
-    for (int e = lane; e < E; e += 32) z += expf(l[e] - m);
-    z = warp_sum(z);
-
-    uint32_t taken = 0;  // bit i: expert lane + 32*i already selected
-    float psel = 0.f;
-    for (int k = 0; k < K; ++k) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
-        for (int i = 0, e = lane; e < E; ++i, e += 32) {
-            if ((taken >> i) & 1u) continue;
-            const float v = isnan(l[e]) ? -INFINITY : l[e];
-            if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-        }
-        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
-        const float p = expf(bv - m) / z;
-        psel += p;
-        if (lane == 0) {
-            topk_idx[(size_t)t * K + k] = bi;
-            pk[k] = p;
-            if (sidx) sidx[k] = bi;
-        }
-    }
-    __syncwarp();
-    for (int k = lane; k < K; k += 32) topk_gate[(size_t)t * K + k] = pk[k] / psel;
-}
-
 template <typename TX, typename TW>
 __global__ void __launch_bounds__(kRouteThreads)
 k_route(int T, int D, int E, int K, const TX *__restrict__ x, const TW *__restrict__ wr,
@@ -1163,8 +1114,14 @@ cudaError_t route_dispatch_small_any(const moe_dims &d, int T, const void *x, co
                                                      inv, st);
 }
 
+// scratch (optional, scratch_bytes): room for the tensor-core router's
+// partial logits; without it (moe_route) the CUDA-core kernel routes.
 cudaError_t route_any(const moe_dims &d, int T, const void *x, const void *wr, float *logits,
-                      int32_t *idx, float *gate, cudaStream_t st) {
+                      int32_t *idx, float *gate, cudaStream_t st, void *scratch = nullptr,
+                      size_t scratch_bytes = 0) {
+    if (scratch && route_tc_ok(d, T) && aligned16(scratch) &&
+        scratch_bytes >= route_tc_scratch_bytes(d, T))
+        return launch_route_tc(d, T, x, wr, logits, idx, gate, static_cast<float *>(scratch), st);
     if (d.w_dtype == MOE_BF16) return launch_route<bf16, bf16>(d, T, x, wr, logits, idx, gate, st);
     return launch_route<float, float>(d, T, x, wr, logits, idx, gate, st);
 }
@@ -1371,7 +1328,10 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
     } else if (small_route_ok(d, T)) {
         e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
     } else {
-        e = route_any(d, T, x, w_router, nullptr, idx, gate, st);
+        // the GLU hidden vectors' region is free until the up projection:
+        // scratch for the tensor-core router
+        e = route_any(d, T, x, w_router, nullptr, idx, gate, st, h,
+                      L.xs > L.h ? L.xs - L.h : 0);
         if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
     }
     if (e != cudaSuccess) return MOE_ERR_CUDA;

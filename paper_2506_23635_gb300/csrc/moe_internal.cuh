@@ -124,6 +124,55 @@ __device__ __forceinline__ int chunk_expert(const int *prefix, int E, int q) {
     return lo;
 }
 
+// Warp-level softmax + top-k of one token's logits l[0..E); writes
+// topk_idx/topk_gate[t*K + k] (and sidx[k] if non-null).  A NaN logit (a
+// token with a NaN or infinite component) ranks as -inf, so the K picks are
+// always distinct experts in [0, E) (K <= E): the indices that address the
+// dispatch arrays stay in range whatever the data; such a token's gates
+// are NaN.
+__device__ inline void select_topk(int E, int K, int t, const float *l, float *pk,
+                            float *__restrict__ logits_opt, int32_t *__restrict__ topk_idx,
+                            float *__restrict__ topk_gate, int *sidx) {
+    const int lane = threadIdx.x & 31;
+    if (logits_opt)
+        for (int e = lane; e < E; e += 32) logits_opt[(size_t)t * E + e] = l[e];
+    float m = -INFINITY;
+    for (int e = lane; e < E; e += 32) m = fmaxf(m, l[e]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float z = 0.f;
+    for (int e = lane; e < E; e += 32) z += expf(l[e] - m);
+    z = warp_sum(z);
+
+    uint32_t taken = 0;  // bit i: expert lane + 32*i already selected
+    float psel = 0.f;
+    for (int k = 0; k < K; ++k) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int i = 0, e = lane; e < E; ++i, e += 32) {
+            if ((taken >> i) & 1u) continue;
+            const float v = isnan(l[e]) ? -INFINITY : l[e];
+            if (v > bv || (v == bv && e < bi)) { bv = v; bi = e; }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+        }
+        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+        const float p = expf(bv - m) / z;
+        psel += p;
+        if (lane == 0) {
+            topk_idx[(size_t)t * K + k] = bi;
+            pk[k] = p;
+            if (sidx) sidx[k] = bi;
+        }
+    }
+    __syncwarp();
+    for (int k = lane; k < K; k += 32) topk_gate[(size_t)t * K + k] = pk[k] / psel;
+}
+
 // ---- host side -----------------------------------------------------------
 
 struct DeviceInfo {
@@ -247,6 +296,15 @@ cudaError_t launch_gemm_up_wm(const moe_dims &d, int T, const void *x_sorted,
 cudaError_t launch_gemm_down_wm(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                 const void *w2, float *y_sorted, cudaStream_t st,
                                 const char *name);
+
+// Router logits of batches of 128 or more tokens on the tensor cores
+// (route_tc.cu), E <= 16, bf16: partial logits of ksplit shares of d in
+// `scratch` (route_tc_scratch_bytes), then top-k and gates as moe_route.
+bool route_tc_ok(const moe_dims &d, int T);
+size_t route_tc_scratch_bytes(const moe_dims &d, int T);
+cudaError_t launch_route_tc(const moe_dims &d, int T, const void *x, const void *wr,
+                            float *logits, int32_t *idx, float *gate, float *scratch,
+                            cudaStream_t st);
 
 // Bulk-copy pipelined decode kernels (ffn_stream.cu), bf16 only, up to
 // kStreamMaxSlots slots; the GLU hidden vectors h are bf16.  Batches of at
