@@ -80,25 +80,39 @@ __device__ __forceinline__ void write_trivial_dispatch(int T, int32_t *offsets) 
     }
 }
 
-// One 1024-thread block per token: every thread's loads of the row are in
-// flight together.
+// One block per token: 1024 threads for decode batches (every thread's
+// loads of the row in flight together), 256 threads with 16 float4 of the
+// row each for larger batches (the 1024-thread form ran at 1.9 TB/s over
+// 2048 tokens: too little work per thread between block barriers).  The row
+// stays in registers between the sum of squares and the scaling.
 constexpr int kNormThreads = 1024;
+constexpr int kNormThreadsWide = 256;
+constexpr int kNormWideMinTokens = 64;
+constexpr int kNormMaxVec = 16;  // float4 per thread: D <= 4 * 16 * 256
 
-__global__ void __launch_bounds__(kNormThreads)
+template <int NT, int VEC>
+__global__ void __launch_bounds__(NT)
 k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ xn, float eps,
              int32_t *offsets) {
     // the projection after this kernel may start now: its weight loads do
     // not depend on anything here
     ptx::launch_dependents();
     ptx::grid_dependency_wait();
-    __shared__ float red[kNormThreads / 32];
+    __shared__ float red[NT / 32];
     const int t = blockIdx.x;
     if (t == 0) write_trivial_dispatch(T, offsets);
     const float4 *r = reinterpret_cast<const float4 *>(resid + (size_t)t * D);
     const int nv = D >> 2;
+    float4 keep[VEC];
     float ss = 0.f;
-#pragma unroll 4
-    for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+#pragma unroll
+    for (int u = 0; u < VEC; ++u) {
+        const int i = threadIdx.x + u * NT;
+        keep[u] = i < nv ? r[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+        ss += keep[u].x * keep[u].x + keep[u].y * keep[u].y + keep[u].z * keep[u].z +
+              keep[u].w * keep[u].w;
+    }
+    for (int i = threadIdx.x + VEC * NT; i < nv; i += NT) {  // rows wider than the registers
         const float4 v = r[i];
         ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
     }
@@ -107,11 +121,18 @@ k_sa_prenorm(int T, int D, const float *__restrict__ resid, bf16 *__restrict__ x
     __syncthreads();
     float tot = 0.f;
 #pragma unroll
-    for (int w = 0; w < kNormThreads / 32; ++w) tot += red[w];
+    for (int w = 0; w < NT / 32; ++w) tot += red[w];
     const float s = 1.0f / sqrtf(tot / (float)D + eps);
     __nv_bfloat162 *o = reinterpret_cast<__nv_bfloat162 *>(xn + (size_t)t * D);
-#pragma unroll 4
-    for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+#pragma unroll
+    for (int u = 0; u < VEC; ++u) {
+        const int i = threadIdx.x + u * NT;
+        if (i < nv) {
+            o[2 * i] = __floats2bfloat162_rn(keep[u].x * s, keep[u].y * s);
+            o[2 * i + 1] = __floats2bfloat162_rn(keep[u].z * s, keep[u].w * s);
+        }
+    }
+    for (int i = threadIdx.x + VEC * NT; i < nv; i += NT) {
         const float4 v = r[i];
         o[2 * i] = __floats2bfloat162_rn(v.x * s, v.y * s);
         o[2 * i + 1] = __floats2bfloat162_rn(v.z * s, v.w * s);
@@ -148,6 +169,23 @@ k_rope_cache(int T, int Hq, int Hkv, int n_seq, int L, RopeRates rates,
     const int nq = Hq * kHeadDim, nkv = Hkv * kHeadDim;
     const int tb = blockIdx.y * kRopeTokens;
     const int nt = min(kRopeTokens, T - tb);
+    // every token's pair first (independent loads in flight together, and
+    // in flight while the angles are formed), the projection's partial sums
+    // added in order
+    const bool row_ok = hr < Hq + 2 * Hkv;
+    float av[kRopeTokens], bv[kRopeTokens];
+#pragma unroll
+    for (int u = 0; u < kRopeTokens; ++u) {
+        av[u] = 0.f;
+        bv[u] = 0.f;
+        if (row_ok && u < nt) {
+            const float *row = qkv + (size_t)(tb + u) * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
+            for (int k = 0; k < n_part; ++k) {
+                av[u] += row[k * part_stride + i];
+                bv[u] += row[k * part_stride + i + H2];
+            }
+        }
+    }
     // the angles of every token of the block: pair i of token tb+u turns by
     // pos * rate_i, formed and reduced to [-pi, pi] in fp64 (exact to far
     // below fp32 resolution at any cache position), evaluated in fp32
@@ -166,22 +204,7 @@ k_rope_cache(int T, int Hq, int Hkv, int n_seq, int L, RopeRates rates,
         sincosf((float)red, &sn_s[u][k], &cs_s[u][k]);
     }
     __syncthreads();
-    if (hr >= Hq + 2 * Hkv) return;
-    // every token's pair first (independent loads in flight together), the
-    // projection's partial sums added in order
-    float av[kRopeTokens], bv[kRopeTokens];
-#pragma unroll
-    for (int u = 0; u < kRopeTokens; ++u) {
-        av[u] = 0.f;
-        bv[u] = 0.f;
-        if (u < nt) {
-            const float *row = qkv + (size_t)(tb + u) * (nq + 2 * nkv) + (size_t)hr * kHeadDim;
-            for (int k = 0; k < n_part; ++k) {
-                av[u] += row[k * part_stride + i];
-                bv[u] += row[k * part_stride + i + H2];
-            }
-        }
-    }
+    if (!row_ok) return;
 #pragma unroll
     for (int u = 0; u < kRopeTokens; ++u) {
         if (u >= nt) break;
@@ -465,25 +488,28 @@ k_residual_add(long long n4, int n_part, float *__restrict__ resid, const float 
 
 // Decoder layers: resid[t] += sum of the partial projections, then the MoE
 // block's input xn[t] = bf16(RMSNorm0(resid[t])) -- the residual add of the
-// attention block and the pre-norm of the MoE block in one pass, one
-// 1024-thread block per token (D/4 <= 4 * 1024 keeps the row in registers).
-constexpr int kResNormVec = 4;  // float4 per thread held in registers
+// attention block and the pre-norm of the MoE block in one pass, one block
+// per token with the row in registers (NT threads x VEC float4: 1024 x 4 for
+// decode batches, 256 x 16 for larger ones, as k_sa_prenorm; D <= 16384).
+constexpr int kResNormCap = 4 * 4 * kNormThreads;  // row length the fused form holds
 
-__global__ void __launch_bounds__(kNormThreads)
+template <int NT, int VEC>
+__global__ void __launch_bounds__(NT)
 k_residual_prenorm(int T, int D, int n_part, float *__restrict__ resid, const float *__restrict__ y,
                    bf16 *__restrict__ xn, float eps) {
+    static_assert(4 * NT * VEC == kResNormCap, "both forms hold a row of kResNormCap");
     ptx::grid_dependency_wait();
-    __shared__ float red[kNormThreads / 32];
+    __shared__ float red[NT / 32];
     const int t = blockIdx.x;
     const int nv = D >> 2;
     const long long stride4 = (long long)T * nv;  // between partial projections, in float4
     float4 *r = reinterpret_cast<float4 *>(resid + (size_t)t * D);
     const float4 *a = reinterpret_cast<const float4 *>(y + (size_t)t * D);
-    float4 keep[kResNormVec];
+    float4 keep[VEC];
     float ss = 0.f;
 #pragma unroll
-    for (int u = 0; u < kResNormVec; ++u) {
-        const int i = threadIdx.x + u * kNormThreads;
+    for (int u = 0; u < VEC; ++u) {
+        const int i = threadIdx.x + u * NT;
         keep[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (i < nv) {
             float4 w = a[i];
@@ -509,12 +535,12 @@ k_residual_prenorm(int T, int D, int n_part, float *__restrict__ resid, const fl
     __syncthreads();
     float tot = 0.f;
 #pragma unroll
-    for (int w = 0; w < kNormThreads / 32; ++w) tot += red[w];
+    for (int w = 0; w < NT / 32; ++w) tot += red[w];
     const float sc = 1.0f / sqrtf(tot / (float)D + eps);
     __nv_bfloat162 *o = reinterpret_cast<__nv_bfloat162 *>(xn + (size_t)t * D);
 #pragma unroll
-    for (int u = 0; u < kResNormVec; ++u) {
-        const int i = threadIdx.x + u * kNormThreads;
+    for (int u = 0; u < VEC; ++u) {
+        const int i = threadIdx.x + u * NT;
         if (i < nv) {
             o[2 * i] = __floats2bfloat162_rn(keep[u].x * sc, keep[u].y * sc);
             o[2 * i + 1] = __floats2bfloat162_rn(keep[u].z * sc, keep[u].w * sc);
@@ -709,8 +735,11 @@ cudaError_t out_proj(const SaCall &c, const void *ctx, const void *w_o, float *r
         const float *yc = y;
         void *args[] = {&Tv, &D, &n_part, &resid, &yc, &xn_next, &eps};
         LaunchScope ls("residual_prenorm", c.st);
-        return launch_pdl((const void *)k_residual_prenorm, dim3(c.T), dim3(kNormThreads), 0, c.st,
-                          args);
+        if (c.T >= kNormWideMinTokens)
+            return launch_pdl((const void *)k_residual_prenorm<kNormThreadsWide, kNormMaxVec>,
+                              dim3(c.T), dim3(kNormThreadsWide), 0, c.st, args);
+        return launch_pdl((const void *)k_residual_prenorm<kNormThreads, 4>, dim3(c.T),
+                          dim3(kNormThreads), 0, c.st, args);
     }
     long long n4 = (long long)c.T * c.d.d_model / 4;
     const long long cap = (long long)device_info().sm_count * 8;
@@ -767,9 +796,13 @@ moe_status sa_forward_impl(const moe_sa_dims *dims, int32_t T, const int32_t *se
         int32_t *off = at<int32_t>(ws, c.L.offsets);
         void *args[] = {&Tv, &D, &rc, &xn, &eps, &off};
         LaunchScope ls("sa_prenorm", c.st);
-        if (launch_pdl((const void *)k_sa_prenorm, dim3(T), dim3(kNormThreads), 0, c.st, args) !=
-            cudaSuccess)
-            return MOE_ERR_CUDA;
+        const cudaError_t e =
+            T >= kNormWideMinTokens
+                ? launch_pdl((const void *)k_sa_prenorm<kNormThreadsWide, kNormMaxVec>, dim3(T),
+                             dim3(kNormThreadsWide), 0, c.st, args)
+                : launch_pdl((const void *)k_sa_prenorm<kNormThreads, 4>, dim3(T),
+                             dim3(kNormThreads), 0, c.st, args);
+        if (e != cudaSuccess) return MOE_ERR_CUDA;
     }
     bf16 *q16 = tc_attention(T) ? at<bf16>(ws, c.L.q16) : nullptr;
     cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache, q16);
@@ -869,7 +902,7 @@ moe_status moe_decoder_forward(const moe_sa_dims *attn, const moe_dims *moe_d, i
     if (!ws || !aligned16(ws) || ws_bytes < need) return MOE_ERR_WORKSPACE;
     // the attention block's residual add and the MoE block's pre-norm run as
     // one kernel when a row fits its registers; otherwise as the stack does
-    const bool fused = attn->d_model <= 4 * kResNormVec * kNormThreads;
+    const bool fused = attn->d_model <= kResNormCap;
     const size_t xn_bytes = ((size_t)T * attn->d_model * 2 + 255) & ~size_t(255);
     bf16 *xn = static_cast<bf16 *>(ws);
     void *inner = static_cast<char *>(ws) + xn_bytes;
