@@ -150,8 +150,8 @@ k_sa_setup(int T, int32_t *offsets) {
 // and the values to the caches [n_seq, Hkv, L, 128] in bf16.  A block holds
 // kRopeRows head rows of one token, 64 threads each: thread i turns the pair
 // (i, i + 64) of a query or key head, or copies two value elements.
-constexpr int kRopeRows = 16;  // head rows per block
-constexpr int kRopeTokens = 8;  // tokens per block, one after the other
+constexpr int kRopeRows = 8;  // head rows per block
+constexpr int kRopeTokens = 4;  // tokens per block, one after the other
 
 __global__ void __launch_bounds__(kRopeRows * kHeadDim / 2)
 k_rope_cache(int T, int Hq, int Hkv, int n_seq, int L, RopeRates rates,
