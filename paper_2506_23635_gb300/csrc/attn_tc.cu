@@ -5,21 +5,22 @@
 // head h), key/value head g = h / (Hq/Hkv), over cache positions 0 .. p0+127
 // in key/value tiles of 128 positions:
 //
-//   warp 0      TMA: the tile's bf16 queries once, then the key tiles of
-//               positions [128j, 128j+128) into a two-stage ring and the value
-//               tiles into one stage (free again once transposed);
+//   warp 0      TMA: the tile's bf16 queries once, then the key and the value
+//               tiles of positions [128j, 128j+128) into two-stage rings;
 //   warp 1      tensor memory (512 columns: two score buffers and one output
 //               tile) and the MMAs: S_j = Q K_j^T (M = 128 queries, N = 128
 //               positions, K = 128 dims) into score buffer j % 2, and once
-//               the softmax warps have written P_j and V_j^T,
+//               the softmax warps have written P_j,
 //               O_j = P_j V_j (M = 128 queries, N = 128 dims, K = 128
-//               positions) into the output tile;
+//               positions) into the output tile, V_j read as it lies in the
+//               cache: an MN-major operand (dims contiguous, 128-byte
+//               swizzle), so no transpose;
 //   warps 2-9   two threads per query row, each owning 64 of the 128 score
 //               columns and of the 128 output dims: fold O_{j-1} into the
-//               row's fp32 accumulator (registers), transpose V_j into the
-//               K-major V^T tile with ldmatrix.trans / stmatrix (positions
-//               past the tile's last query are written as zero), then the
-//               online softmax of S_j (causal mask, base-2 exponent of the
+//               row's fp32 accumulator (registers), zero the rows of V_j past
+//               the tile's last query (a key/value tile that runs past it:
+//               those cache rows may hold anything, and 0 * NaN is NaN), then
+//               the online softmax of S_j (causal mask, base-2 exponent of the
 //               1/sqrt(128)-scaled scores; the two halves of a row exchange
 //               their maxima through shared memory) and the bf16
 //               probabilities P_j, written in the 128-byte-swizzled K-major
@@ -42,11 +43,10 @@ constexpr int kFaSoftmaxWarps = 8;       // two threads per query row
 constexpr int kFaThreads = (2 + kFaSoftmaxWarps) * 32;
 constexpr uint32_t kHalfBytes = kFa * 128;     // one 64-column half of a 128-row tile
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;  // 32 KB
-// shared memory: Q, K[2], V, V^T, P (each a 32 KB tile), then the header
+// shared memory: Q, K[2], V[2], P (each a 32 KB tile), then the header
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kTileBytes;
 constexpr uint32_t kOffV = 3 * kTileBytes;
-constexpr uint32_t kOffVt = 4 * kTileBytes;
 constexpr uint32_t kOffP = 5 * kTileBytes;
 constexpr uint32_t kOffHdr = 6 * kTileBytes;
 constexpr uint32_t kOffRed = kOffHdr + 256;  // row max / sum exchange: [2][2][128] floats
@@ -55,14 +55,16 @@ static_assert(kFaSmem <= 227 * 1024, "shared memory");
 // kind::f16 instruction descriptor: bf16 A and B, fp32 D, K-major, N = M = 128
 constexpr uint32_t kFaIdesc =
     (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kFa >> 3) << 17) | ((uint32_t)(kFa >> 4) << 24);
+// the same with B MN-major (bit 16): O = P V with V as stored
+constexpr uint32_t kFaIdescVmn = kFaIdesc | (1u << 16);
 constexpr uint32_t kFaTmemCols = 512;  // S[0] 0..127, S[1] 128..255, O 256..383
 
 struct FaHeader {
     uint64_t q_full;
     uint64_t kv_full[2];   // key tile j in stage j % 2
     uint64_t kv_empty[2];
-    uint64_t v_full;       // value tile j (one stage)
-    uint64_t v_empty;      // the softmax warps have transposed it (one arrival each)
+    uint64_t v_full[2];    // value tile j in stage j % 2
+    uint64_t v_empty[2];   // the MMA of O_j has read it
     uint64_t s_full[2];
     uint64_t s_free[2];  // the softmax warps have read score buffer b (one arrival each)
     uint64_t p_ready;    // P_j and V_j^T written (one arrival per softmax warp)
@@ -78,25 +80,33 @@ __device__ __forceinline__ uint32_t tile_offset(uint32_t r, uint32_t k) {
     return (k >> 6) * kHalfBytes + swizzle_offset(r, k & 63u);
 }
 
-// Four 8x8 bf16 blocks, transposed on the way into registers / stored as is.
-__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(addr)
-                 : "memory");
-}
-__device__ __forceinline__ void stsm_x4(uint32_t addr, const uint32_t (&r)[4]) {
-    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(addr),
-                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
-                 : "memory");
-}
-
 // 2^x on the special-function unit (the probabilities are rounded to bf16
 // right after, far coarser than its error).
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+
+// Shared-memory descriptor of an MN-major operand written by TMA with the
+// 128-byte swizzle: a row of 128 B holds 64 consecutive MN elements of one k,
+// 8 rows (k) make a 1024-byte atom; the next 8 k follow 1024 B on (stride
+// offset), the next 64 MN elements 16 KB on (leading offset: the second
+// 64-column box of the tile).
+__device__ __forceinline__ uint64_t smem_desc_mn(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(kHalfBytes >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// O (+)= P V: P [128 queries, 128 positions] K-major, V [128 positions,
+// 128 dims] as stored (MN-major); K = 16 positions per instruction.
+__device__ __forceinline__ void issue_pv(uint32_t d_tmem, uint32_t p_smem, uint32_t v_smem) {
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+        const uint64_t ad = smem_desc(p_smem + (ks >> 2) * kHalfBytes) + 2 * (ks & 3);
+        const uint64_t bd = smem_desc_mn(v_smem + ks * 16 * 128);
+        mma_bf16(d_tmem, ad, bd, kFaIdescVmn, ks != 0 ? 1u : 0u);
+    }
 }
 
 __device__ __forceinline__ void issue_128x128x128(uint32_t d_tmem, uint32_t a_smem, uint32_t b_smem) {
@@ -134,8 +144,10 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             ptx::mbar_init(&hd->s_free[b], kFaSoftmaxWarps);
         }
         ptx::mbar_init(&hd->p_ready, kFaSoftmaxWarps);
-        ptx::mbar_init(&hd->v_full, 1);
-        ptx::mbar_init(&hd->v_empty, kFaSoftmaxWarps);
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(&hd->v_full[b], 1);
+            ptx::mbar_init(&hd->v_empty[b], 1);
+        }
         ptx::mbar_init(&hd->o_full, 1);
         ptx::mbar_init(&hd->done, 1);
         ptx::fence_barrier_init();
@@ -184,18 +196,19 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                     ptx::tma_load_2d(smem + kOffK + b * kTileBytes + half * kHalfBytes, &tmK,
                                      half * 64, row0 + j * kFa, &hd->kv_full[b], pol);
                 issued = j + 1;
-                if (!ptx::mbar_wait(&hd->v_empty, (j & 1) ^ 1, err)) break;
-                ptx::mbar_arrive_expect_tx(&hd->v_full, kTileBytes);
+                if (!ptx::mbar_wait(&hd->v_empty[b], ((j >> 1) & 1) ^ 1, err)) break;
+                ptx::mbar_arrive_expect_tx(&hd->v_full[b], kTileBytes);
                 for (int half = 0; half < 2; ++half)
-                    ptx::tma_load_2d(smem + kOffV + half * kHalfBytes, &tmV, half * 64,
-                                     row0 + j * kFa, &hd->v_full, pol);
+                    ptx::tma_load_2d(smem + kOffV + b * kTileBytes + half * kHalfBytes, &tmV,
+                                     half * 64, row0 + j * kFa, &hd->v_full[b], pol);
                 v_issued = j + 1;
             }
             // let loads still in flight land before the block can exit
             ptx::mbar_wait(&hd->q_full, 0, err);
             for (int j = (issued > 2 ? issued - 2 : 0); j < issued; ++j)
                 ptx::mbar_wait(&hd->kv_full[j & 1], (j >> 1) & 1, err);
-            if (v_issued > 0) ptx::mbar_wait(&hd->v_full, (v_issued - 1) & 1, err);
+            for (int j = (v_issued > 2 ? v_issued - 2 : 0); j < v_issued; ++j)
+                ptx::mbar_wait(&hd->v_full[j & 1], (j >> 1) & 1, err);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -213,10 +226,12 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                 }
                 if (j >= 1) {  // O_{j-1} = P_{j-1} V_{j-1}
                     const int jp = j - 1;
+                    if (!(good = ptx::mbar_wait(&hd->v_full[jp & 1], (jp >> 1) & 1, err))) break;
                     if (!(good = ptx::mbar_wait(&hd->p_ready, jp & 1, err))) break;
                     tc_fence_after();
-                    issue_128x128x128(tmem + 2 * kFa, sbase + kOffP, sbase + kOffVt);
+                    issue_pv(tmem + 2 * kFa, sbase + kOffP, sbase + kOffV + (jp & 1) * kTileBytes);
                     mma_commit(&hd->o_full);
+                    mma_commit(&hd->v_empty[jp & 1]);  // value tile jp read once these finish
                 }
             }
             mma_commit(&hd->done);
@@ -257,34 +272,19 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                     for (int i = 0; i < 32; ++i) o[c + i] = fmaf(o[c + i], corr, v[i]);
                 }
             }
-            // V_j -> V^T (row = dim, column = position), zero past `last`: warp
-            // w8 transposes position blocks 2w8, 2w8+1, four 8x8 blocks (dims
-            // 32k..32k+31) per ldmatrix.trans / stmatrix pair
-            good = good && ptx::mbar_wait(&hd->v_full, j & 1, err);
-            {
-                const uint32_t vs = sbase + kOffV, vt = sbase + kOffVt;
-                const bool clip = j * kFa + kFa - 1 > last;
+            // a value tile that runs past the tile's last query: its rows past
+            // `last` are zeroed before P_j V_j reads them (P is zero there, but
+            // those cache rows may hold anything); thread (r, hf) clears half
+            // hf of row r
+            if (j * kFa + kFa - 1 > last) {
+                good = good && ptx::mbar_wait(&hd->v_full[b], (j >> 1) & 1, err);
+                if (j * kFa + r > last) {
+                    unsigned char *vrow = smem + kOffV + b * kTileBytes + hf * kHalfBytes;
 #pragma unroll
-                for (int pbi = 0; pbi < 2; ++pbi) {
-                    const int pb = w8 * 2 + pbi;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const int db = 4 * k + (lane >> 3);  // this lane's block for the addresses
-                        uint32_t rr[4];
-                        ldsm_x4_trans(vs + tile_offset(8 * pb + (lane & 7), 8 * db), rr);
-                        if (clip) {  // register i holds positions 8pb + 2(lane%4) and +1
-                            const int pa = j * kFa + 8 * pb + 2 * (lane & 3);
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                if (pa > last) rr[i] &= 0xffff0000u;
-                                if (pa + 1 > last) rr[i] &= 0x0000ffffu;
-                            }
-                        }
-                        stsm_x4(vt + tile_offset(8 * db + (lane & 7), 8 * pb), rr);
-                    }
+                    for (int c = 0; c < 64; c += 8)
+                        *reinterpret_cast<uint4 *>(vrow + swizzle_offset((uint32_t)r, (uint32_t)c)) =
+                            make_uint4(0u, 0u, 0u, 0u);
                 }
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&hd->v_empty);  // value tile read
             }
             // scores of S_j (this thread's 64 columns): masked max, exchanged
             // with the other half of the row, then probabilities
@@ -335,7 +335,7 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                 }
                 *reinterpret_cast<uint4 *>(ps + tile_offset(r, c0 + i)) = make_uint4(w[0], w[1], w[2], w[3]);
             }
-            fence_proxy_async_smem();  // P_j and V_j^T visible to the MMA
+            fence_proxy_async_smem();  // P_j (and a clipped V_j) visible to the MMA
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&hd->p_ready);
             corr = exp2f(m - mx);  // 0 on the first tile (m = -inf)

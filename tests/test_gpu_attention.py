@@ -224,6 +224,33 @@ def test_decoder_layers(kind):
     assert rel <= 5e-3 * np.sqrt(n_layers), f"decoder layers: rel L2 of the update {rel:.3e}"
 
 
+def test_prefill_ignores_cache_rows_past_the_chunk():
+    """Positions 37..336 of sequence 1 (two tensor-core tiles whose last
+    key/value tile runs past their last query, and a CUDA-core tail) with NaN
+    in every cache row the chunk does not reach: the result equals the
+    oracle's, which reads only positions up to each token's own."""
+    m = moe()
+    shape, w_qkv, w_o, kc, vc, seq, pos = _case((256, 4, 2, 2, 400, "chunk300"), seed=13)
+    nan = gen.store(np.full(1, np.nan), "bf16")[0]
+    kc = kc.copy()
+    vc = vc.copy()
+    kc[1, :, 337:, :] = nan
+    vc[1, :, 337:, :] = nan
+    T = seq.size
+    x = np.random.default_rng(17).normal(size=(T, shape.d_model)).astype(np.float32)
+    want, _, _ = oracle.sa_forward(x.astype(np.float64), w_qkv, w_o, "bf16", shape.n_heads,
+                                   shape.n_kv_heads, shape.rope_base, EPS, seq, pos,
+                                   gen.to_f64(kc, "bf16"), gen.to_f64(vc, "bf16"))
+    resid = torch.from_numpy(x).cuda()
+    m.sa_forward(_sa(m, shape), resid, dev(w_qkv, "bf16"), dev(w_o, "bf16"),
+                 torch.from_numpy(seq).cuda(), torch.from_numpy(pos).cuda(), dev(kc, "bf16"),
+                 dev(vc, "bf16"), eps=EPS)
+    assert m.get_last_error() == 0
+    got = to_numpy(resid)
+    assert np.isfinite(got).all()
+    assert_parity(got - x, want - x, "bf16", "prefill chunk beside NaN cache rows")
+
+
 @pytest.mark.parametrize("T,ctx_len", [(1, 2048), (8, 2048), (256, 256)])
 def test_dbrx_attention_block(T, ctx_len):
     """DBRX's attention dims (D = 6144, 48 query and 8 key/value heads of
