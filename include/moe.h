@@ -331,7 +331,10 @@ moe_status moe_sa_qkv(const moe_sa_dims *dims, int32_t T, const void *x_norm,
                       void *v_cache, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /* moe_sa_attend: ctx[t, h dh .. (h+1) dh) = softmax over positions
- * 0..pos[t] of q[t,h] . K / sqrt(dh), applied to V (bf16 out). */
+ * 0..pos[t] of q[t,h] . K / sqrt(dh), applied to V (bf16 out).  As in
+ * moe_sa_forward, every 128 consecutive tokens that are positions
+ * p0..p0+127 of one sequence (a prefill chunk) are attended on the tensor
+ * cores from q rounded to bf16; the other tokens use q as given. */
 moe_status moe_sa_attend(const moe_sa_dims *dims, int32_t T, const float *q,
                          const int32_t *seq, const int32_t *pos, int32_t n_seq,
                          int32_t max_len, const void *k_cache, const void *v_cache,

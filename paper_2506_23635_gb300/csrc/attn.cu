@@ -460,6 +460,22 @@ k_attn_merge(int n_split, const float *__restrict__ part_ml, const float *__rest
     ctx[(size_t)th * kHeadDim + d] = __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
 }
 
+// The tensor-core attention's bf16 copy of fp32 queries, for a call that
+// brings its own queries (moe_sa_attend); in the whole block the rotary
+// kernel writes it.  n4 groups of four elements.
+__global__ void __launch_bounds__(256)
+k_q_bf16(long long n4, const float *__restrict__ q, bf16 *__restrict__ q16) {
+    ptx::grid_dependency_wait();
+    const float4 *a = reinterpret_cast<const float4 *>(q);
+    __nv_bfloat162 *o = reinterpret_cast<__nv_bfloat162 *>(q16);
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+         i += (long long)gridDim.x * blockDim.x) {
+        const float4 v = a[i];
+        o[2 * i] = __floats2bfloat162_rn(v.x, v.y);
+        o[2 * i + 1] = __floats2bfloat162_rn(v.z, v.w);
+    }
+}
+
 // resid += y_0 + ... + y_{n_part-1} (partial projections n4 float4 apart,
 // added in order before the residual).
 __global__ void __launch_bounds__(256)
@@ -852,7 +868,21 @@ moe_status moe_sa_attend(const moe_sa_dims *dims, int32_t T, const float *q, con
         return MOE_ERR_INVALID_ARG;
     if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
     SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
-    return cuda_status(attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx));
+    // the same kernels as the whole block: full prefill tiles on the tensor
+    // cores, from a bf16 copy of the queries
+    bf16 *q16 = nullptr;
+    if (tc_attention(T)) {
+        q16 = at<bf16>(ws, c.L.q16);
+        long long n4 = (long long)T * dims->n_heads * dims->head_dim / 4;
+        const float *qc = q;
+        void *args[] = {&n4, &qc, &q16};
+        const int blocks = (int)std::min<long long>((n4 + 255) / 256, 4LL * device_info().sm_count);
+        LaunchScope ls("q_bf16", c.st);
+        cudaError_t e = launch_pdl((const void *)k_q_bf16, dim3(std::max(blocks, 1)), dim3(256), 0,
+                                   c.st, args);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return cuda_status(attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx, q16));
 }
 
 moe_status moe_sa_forward(const moe_sa_dims *dims, int32_t T, const int32_t *seq,

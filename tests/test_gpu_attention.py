@@ -278,3 +278,61 @@ def test_dbrx_attention_block(T, ctx_len):
                  torch.from_numpy(pos).cuda(), dev(kc, "bf16"), dev(vc, "bf16"), eps=EPS)
     assert m.get_last_error() == 0
     assert_parity(to_numpy(resid) - x, want - x, "bf16", f"DBRX attention block T={T}")
+
+
+def _plateau_case(levels, T, L=600, seed=41):
+    """Queries u (one bf16-exact unit vector for every token and head) and
+    keys c(pos) * u * sqrt(128) / log2(e) plus N(0,1) noise, so the scaled
+    score of position pos is c(pos) in base-2 units (+ ~0.13 noise): the
+    running row maximum steps as `levels` says.  Sequence 1, positions
+    0..T-1; values N(0,1)."""
+    rng = np.random.default_rng(seed)
+    Hq, Hkv, dh = 4, 2, 128
+    u = rng.normal(size=dh)
+    u = gen.to_f64(gen.store(u / np.linalg.norm(u), "bf16"), "bf16")
+    q = np.tile(u, (T, Hq)).astype(np.float32)
+    c = np.zeros(L)
+    for lo, hi, lv in levels:
+        c[lo:hi] = lv
+    k = np.empty((2, Hkv, L, dh))
+    k[:] = rng.normal(size=(2, Hkv, L, dh))
+    k[1] += (c[:, None] * u[None, :] * np.sqrt(dh) / np.log2(np.e))[None]
+    kc = gen.store(k, "bf16")
+    vc = gen.store(rng.normal(size=(2, Hkv, L, dh)), "bf16")
+    seq = np.ones(T, np.int32)
+    pos = np.arange(T, dtype=np.int32)
+    return gen.AttnShape(512, Hq, Hkv, dh, 10000.0, "bf16"), q, kc, vc, seq, pos
+
+
+# (levels as (first, end, base-2 score), tokens): the exponent base moves in
+# the first tile, stays while the maximum rises by 4.5 (probabilities up to
+# 2^4.5), moves by 9 in the third tile and again inside the diagonal tile of
+# the fourth, then the scores drop by 20; a ragged CUDA-core tail after four
+# tensor-core tiles.  Then a maximum of 40 in the first tile that nothing
+# later approaches (every later probability ~2^-40).
+PLATEAUS = [
+    ([(100, 230, 8.5), (230, 300, 13.0), (300, 420, 22.0), (420, 470, 31.0),
+      (470, 600, 11.0)], 571),
+    ([(0, 12, 40.0)], 512),
+]
+
+
+@pytest.mark.parametrize("levels,T", PLATEAUS, ids=["rising", "first-tile-max"])
+def test_prefill_running_max_rescales(levels, T):
+    """The prefill tensor-core attention keeps the exponent base of a row
+    until the row maximum passes it by more than 8 (base 2) and then
+    rescales the output accumulated in tensor memory: scores built to step
+    across that threshold (and below it) give the oracle's attention."""
+    m = moe()
+    shape, q, kc, vc, seq, pos = _plateau_case(levels, T)
+    a = _sa(m, shape)
+    m.profile_reset()
+    m.profile_enable(True)
+    ctx = m.sa_attend(a, torch.from_numpy(q).cuda(), torch.from_numpy(seq).cuda(),
+                      torch.from_numpy(pos).cuda(), dev(kc, "bf16"), dev(vc, "bf16"))
+    assert m.get_last_error() == 0
+    m.profile_enable(False)
+    assert m.profile_read().get("attention_tc", (0,))[0] == 1, "tensor-core attention did not run"
+    want = oracle.attention(q.reshape(T, shape.n_heads, 128).astype(np.float64),
+                            gen.to_f64(kc, "bf16"), gen.to_f64(vc, "bf16"), seq, pos)
+    assert_parity(to_numpy(ctx), want.reshape(T, -1), "bf16", "attention across rescales", True)
