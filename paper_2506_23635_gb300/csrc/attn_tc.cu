@@ -299,7 +299,9 @@ k_attn_prefill_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                         // S_{j+1} replaces P_j: only after P_j V_j has finished
                         const int b1 = (j + 1) & 1;
                         if (!(good = fa_wait(&hd->o_full[x], j & 1, err))) break;
-                        if (!(good = fa_wait(&hd->kv_full[b1], ((j + 1) >> 1) & 1, err))) break;
+                        // (head B follows head A, which has waited for key tile j+1)
+                        if (x == 0 && !(good = fa_wait(&hd->kv_full[b1], ((j + 1) >> 1) & 1, err)))
+                            break;
                         tc_fence_after();
                         issue_qk(tmem + kColS + x * kFa, sbase + kOffQ + x * kTileBytes,
                                  sbase + kOffK + b1 * kTileBytes);
