@@ -336,3 +336,33 @@ def test_prefill_running_max_rescales(levels, T):
     want = oracle.attention(q.reshape(T, shape.n_heads, 128).astype(np.float64),
                             gen.to_f64(kc, "bf16"), gen.to_f64(vc, "bf16"), seq, pos)
     assert_parity(to_numpy(ctx), want.reshape(T, -1), "bf16", "attention across rescales", True)
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(5, 5), (6, 2), (5, 1), (8, 1), (4, 2)],
+                         ids=["G1", "G3", "G5", "G8", "G2"])
+def test_prefill_head_groups(Hq, Hkv):
+    """The tensor-core prefill attention pairs the query heads of a
+    key/value head two to a CTA; with 1, 3 or 5 heads per group the last head
+    of each group is alone in its CTA.  Two full 128-token tiles at positions
+    7..262 of sequence 0 and a 3-token tail, random queries and caches,
+    against the oracle (and the kernel must have run)."""
+    m = moe()
+    rng = np.random.default_rng(50 + Hq * 8 + Hkv)
+    dh, L, T = 128, 300, 259
+    q = rng.normal(size=(T, Hq * dh)).astype(np.float32)
+    q = gen.to_f64(gen.store(q, "bf16"), "bf16").astype(np.float32)  # bf16-exact
+    kc = gen.store(rng.normal(size=(1, Hkv, L, dh)), "bf16")
+    vc = gen.store(rng.normal(size=(1, Hkv, L, dh)), "bf16")
+    seq = np.zeros(T, np.int32)
+    pos = np.arange(7, 7 + T, dtype=np.int32)
+    a = _sa(m, gen.AttnShape(512, Hq, Hkv, dh, 10000.0, "bf16"))
+    m.profile_reset()
+    m.profile_enable(True)
+    ctx = m.sa_attend(a, torch.from_numpy(q).cuda(), torch.from_numpy(seq).cuda(),
+                      torch.from_numpy(pos).cuda(), dev(kc, "bf16"), dev(vc, "bf16"))
+    assert m.get_last_error() == 0
+    m.profile_enable(False)
+    assert m.profile_read().get("attention_tc", (0,))[0] == 1, "tensor-core attention did not run"
+    want = oracle.attention(q.reshape(T, Hq, dh).astype(np.float64), gen.to_f64(kc, "bf16"),
+                            gen.to_f64(vc, "bf16"), seq, pos)
+    assert_parity(to_numpy(ctx), want.reshape(T, -1), "bf16", f"prefill Hq={Hq} Hkv={Hkv}", True)
