@@ -63,7 +63,8 @@ constexpr int kFaHeads = 2;              // query heads per CTA
 constexpr int kFaWarpsPerHead = 4;       // one thread per query row
 constexpr int kFaThreads = (2 + kFaHeads * kFaWarpsPerHead) * 32;
 // how far (base 2) the row maximum may pass the exponent base in use before
-// the base moves and O is rescaled: probabilities up to 2^8, exact in bf16
+// the base moves and O is rescaled: probabilities up to 2^8, well inside the
+// range of bf16 (which rounds them as it would any other value)
 constexpr float kFaRescale = 8.f;
 constexpr uint32_t kHalfBytes = kFa * 128;       // one 64-column half of a 128-row tile
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;  // 32 KB
