@@ -211,17 +211,22 @@ moe_status moe_stack_forward(const moe_dims *dims, int32_t n_layers, int32_t T,
  * memory owned by the library.  Every GPU that loads this part of the
  * library holds that array until the process exits.
  *   - Limit: a call is accepted when moe_workspace_size(dims, T) is at most
- *     MOE_NOALLOC_SCRATCH_BYTES (16 MiB: e.g. the DBRX-shaped layer up to
- *     64 tokens); larger T returns MOE_ERR_WORKSPACE and launches nothing.
+ *     MOE_NOALLOC_SCRATCH_BYTES (24 MiB: the DBRX-shaped layer, D = 6144,
+ *     F = 10752, E = 16, K = 4, fits at every T from 1 to 64, whose largest
+ *     workspace is 20.25 MiB at T = 64); a larger workspace returns
+ *     MOE_ERR_WORKSPACE and launches nothing.
  *   - The first call on a device looks up the array's device address (once
- *     per device, with that device current); make that first call before
- *     any stream capture on the device.
+ *     per device, with that device current) and keeps it until the process
+ *     exits; make that first call before any stream capture on the device.
+ *     The kept address belongs to the device's context of that moment: after
+ *     cudaDeviceReset (or a reset of the primary context) on a device, do not
+ *     call this entry point on that device again in the same process.
  *   - Allocates nothing (no cudaMalloc, cudaFree or allocating library call).
  *   - Every call uses the same array, which keeps the last call's contents;
  *     nothing in it has to start at zero.  Calls whose executions overlap on
  *     the GPU (different streams, or different host threads on one device)
  *     race on the array: serialise them. */
-#define MOE_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+#define MOE_NOALLOC_SCRATCH_BYTES (24u * 1024u * 1024u)
 
 moe_status moe_layer_forward_noalloc(const moe_dims *dims, int32_t T,
                                      const void *x, const void *w_router,

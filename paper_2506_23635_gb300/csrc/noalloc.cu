@@ -13,7 +13,8 @@
 // it until the process exits.  Host code cannot use the array's name as a
 // device address (on the host it names a stand-in object), so the device
 // address is looked up with cudaGetSymbolAddress once per device, with that
-// device current, on the first call made on that device.
+// device current, on the first call made on that device, and kept until the
+// process exits (it is not valid across a reset of the device's context).
 //
 // This file adds a path next to the existing ones; it calls the existing
 // public moe_layer_forward with the array as its workspace and changes
@@ -50,6 +51,7 @@ extern "C" moe_status moe_layer_forward_noalloc(const moe_dims *dims, int32_t T,
                                                 const void *v1, const void *w2,
                                                 const void *residual_opt, void *out,
                                                 moe_stream_t stream) {
+    MOE_INJECT("moe_layer_forward_noalloc");
     size_t need = 0;
     moe_status s = moe_workspace_size(dims, T < 0 ? 0 : T, &need);
     if (s != MOE_OK) return s;

@@ -278,13 +278,14 @@ def stack_forward(d: Dims, weights: StackWeights, resid, ws=None, eps: float = S
     return resid
 
 
-NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024  # MOE_NOALLOC_SCRATCH_BYTES
+NOALLOC_SCRATCH_BYTES = 24 * 1024 * 1024  # MOE_NOALLOC_SCRATCH_BYTES
 
 
 def layer_forward_noalloc(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, stream=None):
     """The whole layer with the library's fixed device scratch array instead
     of a workspace (for callers that cannot allocate; T limited so that the
-    workspace fits in 16 MiB).  Returns out [T, D] (out_dtype)."""
+    workspace fits in NOALLOC_SCRATCH_BYTES, 24 MiB).  Returns out [T, D]
+    (out_dtype)."""
     T = x.shape[0]
     if out is None:
         out = torch.empty((T, d.d_model), dtype=_tdt(d.out_dtype), device=x.device)

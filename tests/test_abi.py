@@ -137,6 +137,37 @@ def test_noalloc_validation(lib):
     assert call(1, x=None) == 1
 
 
+def test_noalloc_limit_holds_the_dbrx_decode_range(lib):
+    """The no-allocation entry point's scratch array holds the DBRX-shaped
+    layer's workspace at every decode batch the header promises (1..64
+    tokens); the binding's constant is the header's."""
+    hdr = open(os.path.join(ROOT, "include", "moe.h")).read()
+    m = re.search(r"#define MOE_NOALLOC_SCRATCH_BYTES \((\d+)u \* 1024u \* 1024u\)", hdr)
+    assert m is not None
+    assert int(m.group(1)) * 1024 * 1024 == lib.NOALLOC_SCRATCH_BYTES
+    d = lib.dims(**DBRX)
+    sizes = [lib.workspace_size(d, T) for T in range(1, 65)]
+    assert max(sizes) <= lib.NOALLOC_SCRATCH_BYTES, max(sizes)
+
+
+def test_noalloc_injected_failure(lib):
+    """MOE_INJECT_FAILURE reaches the no-allocation entry point by its own
+    name (a caller's error path can be tested without a GPU)."""
+    code = (
+        "import ctypes, sys; sys.path.insert(0, %r)\n"
+        "from paper_2506_23635_gb300 import moe\n"
+        "L = moe.lib(); d = moe.dims(64, 64, 4, 2)\n"
+        "print(L.moe_layer_forward_noalloc(ctypes.byref(d), 4, None, None, None, None, None,\n"
+        "                                  None, None, None))\n" % ROOT)
+    import subprocess
+    import sys
+    env = dict(os.environ, MOE_INJECT_FAILURE="moe_layer_forward_noalloc:5")
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env,
+                         timeout=120)
+    assert out.returncode == 0, out.stderr
+    assert int(out.stdout.split()[0]) == 5
+
+
 def test_launch_count_starts_at_zero_without_launches(lib):
     assert lib.launch_count() >= 0
 

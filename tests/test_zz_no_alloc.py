@@ -51,6 +51,24 @@ def test_noalloc_matches_workspace_path_twice():
         assert_parity(to_numpy(out), to_numpy(want), "bf16", "noalloc vs workspace path")
 
 
+def test_noalloc_one_token_twice():
+    """One token (the decode path that streams the selected experts' rows):
+    two calls in a row against the workspace path."""
+    need_gpu()
+    from paper_2506_23635_gb300 import moe
+
+    sh, (x, w_r, w1, v1, w2) = _layer(1, 45)
+    d = moe.dims(sh.d_model, sh.ffn_hidden, sh.n_experts, sh.top_k)
+    x2 = dev(gen.host_normal((1, sh.d_model), 1.0, "bf16", 46, "x2"), "bf16")
+    for xi in (x, x2):
+        want = moe.layer_forward(d, xi, w_r, w1, v1, w2)
+        out = torch.empty_like(want)
+        assert _call_noalloc(moe, d, xi, w_r, w1, v1, w2, out) == 0
+        torch.cuda.synchronize()
+        assert moe.get_last_error() == 0
+        assert_parity(to_numpy(out), to_numpy(want), "bf16", "noalloc vs workspace path, T=1")
+
+
 def test_noalloc_rejects_sizes_beyond_its_scratch():
     need_gpu()
     from paper_2506_23635_gb300 import moe
