@@ -52,6 +52,9 @@ def _bind(path: str) -> ctypes.CDLL:
     lib.orc_layer_tokens.argtypes = [I, I, I, I, I, I, P, P, I, P, P, P, P, I,
                                      P, P, P, P]
     lib.orc_layer_tokens.restype = I
+    lib.orc_layer_experts_tokens.argtypes = [I, I, I, I, I, I, I, I, P, P, I, P, P, P, P, I,
+                                             P, P]
+    lib.orc_layer_experts_tokens.restype = I
     lib.orc_layer_dense_masked.argtypes = [I, I, I, I, I, P, I, P, P, P, P, I, P]
     lib.orc_layer_dense_masked.restype = I
     lib.orc_num_threads.restype = I
@@ -162,6 +165,26 @@ class OracleLib:
         if rc != 0:
             raise ValueError("token index out of range")
         return out, idx, gate
+
+    def layer_experts_tokens(self, x, w_r, w1, v1, w2, dtype: str, top_k: int,
+                             e_begin: int, e_end: int, tokens=None, residual=None):
+        """One node's share of the expert-parallel layer (Sec. 4.3): the
+        gated outputs of the selected experts in [e_begin, e_end) only, for
+        the listed tokens (default: all), plus ``residual`` ([T,D] float64)
+        when given.  w1, v1, w2 hold every expert.  Returns out [n,D] f64."""
+        x = _storage(x, dtype)
+        w_r, w1, v1, w2 = (_storage(a, dtype) for a in (w_r, w1, v1, w2))
+        T, D = x.shape
+        E, F, _ = w1.shape
+        tok = _c(np.arange(T) if tokens is None else tokens, np.int32)
+        out = np.empty((tok.shape[0], D), np.float64)
+        res = None if residual is None else _c(residual, np.float64)
+        rc = self.lib.orc_layer_experts_tokens(T, D, F, E, top_k, e_begin, e_end, tok.shape[0],
+                                               _p(tok), _p(x), _DT[dtype], _p(w_r), _p(w1),
+                                               _p(v1), _p(w2), _DT[dtype], _p(res), _p(out))
+        if rc != 0:
+            raise ValueError("token or expert range out of range")
+        return out
 
     def rmsnorm0(self, x64: np.ndarray, eps: float) -> np.ndarray:
         """Parameter-free RMS pre-norm of each row (fp64)."""
@@ -369,6 +392,10 @@ def layer_tokens(*a, **k):
 
 def layer_dense_masked(*a, **k):
     return default().layer_dense_masked(*a, **k)
+
+
+def layer_experts_tokens(*a, **k):
+    return default().layer_experts_tokens(*a, **k)
 
 
 def layer_steps(*a, **k):

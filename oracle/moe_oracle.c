@@ -206,6 +206,49 @@ int orc_layer_tokens(int T, int D, int F, int E, int K, int n_tok,
     return rc;
 }
 
+/* One node's share of the decentralised expert-parallel layer (Sec. 4.3,
+ * Fig. 7): the node routes the token over all E experts like every other
+ * node, runs only the selected experts it holds, e_begin <= e < e_end, and
+ * contributes their gated outputs; the all-reduce of the nodes' [T,D]
+ * shares forms the weighted sum.  out[i,:] = residual (if given) + sum over
+ * k with e_begin <= idx[k] < e_end of g[k] * y^(k).  w1, v1, w2 hold all E
+ * experts.  Returns 0, or -1 on an out-of-range token or expert range. */
+int orc_layer_experts_tokens(int T, int D, int F, int E, int K, int e_begin,
+                             int e_end, int n_tok, const int32_t *tokens,
+                             const void *x, int xdt, const void *wr,
+                             const void *w1, const void *v1, const void *w2,
+                             int wdt, const double *residual, double *out)
+{
+    if (e_begin < 0 || e_end > E || e_begin >= e_end) return -1;
+    double *xt = (double *)malloc(sizeof(double) * (size_t)D);
+    double *lg = (double *)malloc(sizeof(double) * (size_t)E);
+    double *h = (double *)malloc(sizeof(double) * (size_t)F);
+    double *y = (double *)malloc(sizeof(double) * (size_t)D);
+    int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * (size_t)K);
+    double *g = (double *)malloc(sizeof(double) * (size_t)K);
+    int rc = 0;
+    for (int i = 0; i < n_tok; ++i) {
+        int t = tokens[i];
+        if (t < 0 || t >= T) { rc = -1; break; }
+        for (int d = 0; d < D; ++d) xt[d] = orc_load(x, xdt, (size_t)t * D + d);
+        orc_router_logits(1, D, E, xt, ORC_F64, wr, wdt, lg);
+        orc_topk_gates(1, E, K, lg, idx, g);
+        double *o = out + (size_t)i * D;
+        for (int d = 0; d < D; ++d)
+            o[d] = residual ? residual[(size_t)t * D + d] : 0.0;
+        for (int k = 0; k < K; ++k) {
+            int e = idx[k];
+            if (e < e_begin || e >= e_end) continue; /* another node's expert */
+            orc_expert_ffn(D, F, xt, orc_expert_ptr(w1, wdt, (size_t)F * D, e),
+                           orc_expert_ptr(v1, wdt, (size_t)F * D, e),
+                           orc_expert_ptr(w2, wdt, (size_t)D * F, e), wdt, h, y);
+            for (int d = 0; d < D; ++d) o[d] += g[k] * y[d];
+        }
+    }
+    free(xt); free(lg); free(h); free(y); free(idx); free(g);
+    return rc;
+}
+
 /* Busy full loading (Sec. 4.2): every expert computes every token and the
  * unselected experts' outputs are zeroed in the weighted sum.  The result is
  * the same layer; it is kept as an independent route to the output. */

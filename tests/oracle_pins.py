@@ -296,6 +296,46 @@ def pin_layer_steps_agree(orc):
     assert st["counts"].sum() == idx.size
 
 
+def pin_experts_partition_sums_to_layer(orc):
+    """Sec. 4.3: the all-reduce of the nodes' shares is the weighted sum.
+    The share of [0, E) is the layer (same arithmetic, bit for bit); the
+    shares of any partition of [0, E) into contiguous ranges add up to it;
+    a residual is carried by the share it is given to."""
+    L = _small_layer(E=7, K=3)
+    sh = L.shape
+    E = sh.n_experts
+    out, _, _ = orc.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k)
+    whole = orc.layer_experts_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k, 0, E)
+    assert np.array_equal(whole, out), "share of every expert"
+    for cuts in ((0, 3, 7), (0, 1, 4, 6, 7), tuple(range(E + 1))):
+        parts = [orc.layer_experts_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k,
+                                          b, e) for b, e in zip(cuts[:-1], cuts[1:])]
+        _close(np.sum(parts, axis=0), out, 1e-12, 1e-13, msg=f"partition {cuts}")
+    res = np.random.default_rng(9).normal(size=out.shape)
+    first = orc.layer_experts_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k, 0, 3,
+                                     residual=res)
+    rest = orc.layer_experts_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, sh.top_k, 3, E)
+    _close(first + rest, out + res, 1e-12, 1e-13, msg="residual on one share")
+
+
+def pin_experts_single_expert_k1(orc):
+    """K = 1 and a one-expert share [e, e+1): a token whose arg-max logit
+    (numpy) is e gets exactly that expert's output, every other token an
+    exact zero row."""
+    L = _small_layer(K=1)
+    sh = L.shape
+    x64 = gen.to_f64(L.x, sh.dtype)
+    best = np.argmax(x64 @ gen.to_f64(L.w_r, sh.dtype), axis=1)
+    for e in range(sh.n_experts):
+        part = orc.layer_experts_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, sh.dtype, 1, e, e + 1)
+        for t in range(x64.shape[0]):
+            if best[t] == e:
+                _, y = orc.expert_ffn(x64[t], L.w1[e], L.v1[e], L.w2[e], sh.dtype)
+                assert np.array_equal(part[t], y), "the selected expert's output"
+            else:
+                assert not np.any(part[t]), "another node's expert contributes nothing"
+
+
 # --------------------------------------------------------------------------
 # stack glue (reading C9): RMSNorm0 and the residual stream
 # --------------------------------------------------------------------------

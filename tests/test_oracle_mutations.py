@@ -31,9 +31,14 @@ MUTATIONS = [
      "for (int s = S - 1; s >= 0; --s)\n            if (idx[s] == e) {"),
     ("offsets_not_scanned", "offsets[e + 1] = offsets[e] + counts[e];",
      "offsets[e + 1] = counts[e];"),
-    ("combine_ungated", "for (int d = 0; d < D; ++d) o[d] += g[k] * y[d];",
-     "for (int d = 0; d < D; ++d) o[d] += y[d];"),
+    ("combine_ungated", "o[d] += g[k] * y[d];\n        }\n        if (idx_out)",
+     "o[d] += y[d];\n        }\n        if (idx_out)"),
     ("dense_mask_ungated", "mask[idx[k]] = g[k];", "mask[idx[k]] = 1.0;"),
+    ("experts_range_upper_inclusive", "if (e < e_begin || e >= e_end) continue;",
+     "if (e < e_begin || e > e_end) continue;"),
+    ("experts_range_ignored", "if (e < e_begin || e >= e_end) continue;", "(void)e_begin;"),
+    ("experts_share_ungated", "o[d] += g[k] * y[d];\n        }\n    }\n    free(",
+     "o[d] += y[d];\n        }\n    }\n    free("),
     ("bf16_round_to_9_bits", "const double ulp = ldexp(1.0, e - 8);",
      "const double ulp = ldexp(1.0, e - 9);"),
     ("bf16_round_truncates", "out[i] = nearbyint(v / ulp) * ulp;",
