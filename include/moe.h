@@ -175,6 +175,42 @@ moe_status moe_layer_forward_dense(const moe_dims *dims, int32_t T,
                                    void *out, void *ws, size_t ws_bytes,
                                    moe_stream_t stream);
 
+/* ---- one node's share of an expert-parallel layer ------------------------
+ * Sec. 4.3 (Fig. 7), the paper's decentralised design: every node holds the
+ * router and a disjoint range of the experts; it routes every token itself,
+ * runs its own experts on the tokens that selected them, and the nodes' gated
+ * outputs are summed by one all-reduce of a [T, D] partial per layer (the
+ * exchange of expert outputs of Sec. 3.1, whose cost is the communication
+ * term of Eq. 1).  moe_layer_forward_experts is one node's part:
+ *   partial_out[t,:] = residual_opt[t,:]
+ *       + sum over k with e_begin <= topk_idx[t,k] < e_end of
+ *         gate[t,k] * y[(t,k),:]
+ * where the routing (router over all E experts, softmax, top-k, gates,
+ * dispatch) is the whole layer's, as in moe_layer_forward.
+ *   0 <= e_begin < e_end <= E  (dims->n_experts is the whole layer's E);
+ *   w_router [D, E]: the whole router;
+ *   w1_local, v1_local [e_end - e_begin, F, D], w2_local [e_end - e_begin,
+ *     D, F]: the weights of experts e_begin..e_end-1 only (a node's resident
+ *     share; a caller holding every expert passes w1 + e_begin*F*D, ...);
+ *   residual_opt [T, D] float32 or NULL (give it to one node only, so that
+ *     the sum carries it once);
+ *   partial_out [T, D] float32 whatever dims->out_dtype says; a token none of
+ *     whose experts lies in the range gets its residual row (or zeros);
+ *   ws: moe_workspace_size(dims, T) bytes.
+ * The partials of disjoint ranges covering [0, E), summed, give
+ * moe_layer_forward's output in fp32 (the k sum in another order).  The
+ * sum itself (NCCL all-reduce between GPUs) is the caller's.  Errors: as
+ * moe_layer_forward, plus MOE_ERR_INVALID_ARG for an empty or out-of-range
+ * expert range. */
+moe_status moe_layer_forward_experts(const moe_dims *dims, int32_t T,
+                                     const void *x, const void *w_router,
+                                     int32_t e_begin, int32_t e_end,
+                                     const void *w1_local, const void *v1_local,
+                                     const void *w2_local,
+                                     const float *residual_opt,
+                                     float *partial_out, void *ws,
+                                     size_t ws_bytes, moe_stream_t stream);
+
 /* ---- stack of layers (decode through consecutive MoE blocks) -------------
  * The paper runs DBRX's 40 decoder layers (Table 1); a stack of MoE blocks
  * needs the glue between them, which the paper does not print.  Reading
@@ -253,8 +289,10 @@ moe_status moe_get_last_error(moe_stream_t stream);
  * Host-side fault injection: with MOE_INJECT_FAILURE="<entry>:<status>" in
  * the environment, the named entry point (moe_route, moe_dispatch,
  * moe_expert_ffn, moe_combine, moe_layer_forward, moe_layer_forward_dense,
- * moe_prenorm, moe_stack_forward, moe_sa_qkv, moe_sa_attend, moe_sa_forward,
- * moe_decoder_forward) returns that status at once without launching.
+ * moe_layer_forward_experts, moe_prenorm, moe_stack_forward,
+ * moe_layer_forward_noalloc, moe_sa_qkv,
+ * moe_sa_attend, moe_sa_forward, moe_decoder_forward) returns that status at
+ * once without launching.
  * With MOE_WM_SINGLE_CTA=1 the prefill expert GEMMs (batches whose experts
  * hold 128 or more slots on average) run one CTA per tile, the form used on
  * devices that cannot keep CTA pairs resident, instead of CTA pairs. */

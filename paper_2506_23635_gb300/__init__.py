@@ -7,4 +7,4 @@ kernel behind the C ABI declared in ``include/moe.h``; ``paper_2506_23635_gb300.
 is the Python binding.  Submodules are imported lazily so that the input
 generators can be used without loading the CUDA library.
 """
-__all__ = ["inputs", "moe", "configs"]
+__all__ = ["inputs", "moe", "perf_model", "expert_parallel"]

@@ -318,12 +318,16 @@ k_down_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ h,
     if (!ok) return;
     const int tid = threadIdx.x;
     if (FUSED) {
+        // only the slots of this launch's experts (sorted positions
+        // [offsets[0], offsets[E]): all of them for the whole layer, one
+        // node's share for an expert range) hold a row of ylocal
+        const int j_lo = offsets[0], j_hi = offsets[E];
         for (int idx = tid; idx < T * R; idx += W * 32) {
             const int t = idx / R, r = idx - t * R;
             float v = 0.f;
             for (int k = 0; k < K; ++k) {
                 const int j = inv_perm[(size_t)t * K + k];
-                if (j < 0 || j >= S) continue;
+                if (j < j_lo || j >= j_hi || j < 0 || j >= S) continue;
                 v = fmaf(gate[(size_t)t * K + k], ylocal[(size_t)j * rows_max + r], v);
             }
             if (residual) v += to_f(residual[(size_t)t * D + r0 + r]);

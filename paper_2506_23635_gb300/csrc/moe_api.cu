@@ -730,25 +730,29 @@ constexpr int kCombineMaxK = 256;  // = the largest top_k
 // b takes token b / n_part and the b % n_part-th slice of its row; the
 // token's K sorted positions and gates are read once into shared memory, then
 // every thread's K row loads are independent (streamed past L1).
+// range (optional, n_range experts): the dispatch offsets of a contiguous
+// range of experts; only the slots at sorted positions [range[0],
+// range[n_range]) are summed (one node's share of an expert-parallel layer).
 template <typename TO, typename TR>
 __global__ void __launch_bounds__(256)
 k_combine(int T, int D, int K, int n_part, const float *__restrict__ y,
           const float *__restrict__ y_tail, const int32_t *__restrict__ inv,
           const float *__restrict__ gate, const TR *__restrict__ residual, TO *__restrict__ out,
-          unsigned *err) {
+          const int32_t *__restrict__ range, int n_range, unsigned *err) {
     __shared__ int s_j[kCombineMaxK];
     __shared__ float s_g[kCombineMaxK];
     ptx::grid_dependency_wait();
     const int S = T * K;
     const int nq = D >> 2;
     const int per = (nq + n_part - 1) / n_part;
+    const int j_lo = range ? range[0] : 0, j_hi = range ? range[n_range] : S;
     for (long long b = blockIdx.x; b < (long long)T * n_part; b += gridDim.x) {
         const int t = (int)(b / n_part), part = (int)(b - (long long)t * n_part);
         __syncthreads();  // the previous token's indices are no longer read
         for (int k = threadIdx.x; k < K; k += blockDim.x) {
             const int j = inv[(size_t)t * K + k];
-            if (j >= S) set_error(err, kErrIndex);  // a corrupt index
-            s_j[k] = (j < 0 || j >= S) ? -1 : j;    // or a slot left out by dispatch
+            if (j >= S) set_error(err, kErrIndex);     // a corrupt index
+            s_j[k] = (j < j_lo || j >= j_hi) ? -1 : j;  // or a slot left out
             s_g[k] = gate[(size_t)t * K + k];
         }
         __syncthreads();
@@ -1152,7 +1156,7 @@ cudaError_t dispatch_any(const moe_dims &d, int T, const int32_t *idx, int32_t *
 template <typename TO, typename TR>
 cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const float *y_tail,
                            const int32_t *inv, const float *gate, const void *res, void *out,
-                           cudaStream_t st) {
+                           cudaStream_t st, const int32_t *range, int n_range) {
     // enough blocks for 8 per SM: a token's row is split into n_part slices
     // of at least 256 float4 when there are few tokens
     const int nq = d.d_model / 4;
@@ -1163,18 +1167,22 @@ cudaError_t launch_combine(const moe_dims &d, int T, const float *y, const float
     const TR *rp = static_cast<const TR *>(res);
     TO *op = static_cast<TO *>(out);
     unsigned *err = device_info().err;
-    void *args[] = {&Tv, &D, &K, &n_part, &y, &y_tail, &inv, &gate, &rp, &op, &err};
+    void *args[] = {&Tv, &D, &K, &n_part, &y, &y_tail, &inv, &gate, &rp, &op, &range, &n_range,
+                    &err};
     LaunchScope ls("combine", st);
     return launch_pdl((const void *)k_combine<TO, TR>, dim3(grid), dim3(256), 0, st, args);
 }
 
 cudaError_t combine_any(const moe_dims &d, int T, const float *y, const int32_t *inv,
                         const float *gate, const void *res, void *out, cudaStream_t st,
-                        const float *y_tail = nullptr) {
+                        const float *y_tail = nullptr, const int32_t *range = nullptr,
+                        int n_range = 0) {
     // the residual has the output's dtype
     if (d.out_dtype == MOE_BF16)
-        return launch_combine<bf16, bf16>(d, T, y, y_tail, inv, gate, res, out, st);
-    return launch_combine<float, float>(d, T, y, y_tail, inv, gate, res, out, st);
+        return launch_combine<bf16, bf16>(d, T, y, y_tail, inv, gate, res, out, st, range,
+                                          n_range);
+    return launch_combine<float, float>(d, T, y, y_tail, inv, gate, res, out, st, range,
+                                        n_range);
 }
 
 bool use_stream_path(const moe_dims &d, int T) {
@@ -1199,6 +1207,34 @@ cudaError_t prenorm_any(const moe_dims &d, int T, const void *r, void *xn, float
 
 template <typename P> P *at(void *ws, size_t off) {
     return reinterpret_cast<P *>(static_cast<char *>(ws) + off);
+}
+
+// Routing and dispatch of the whole layer into the workspace regions of L:
+// the fused one-CTA or one-cluster kernels for decode batches, else the
+// router (on the tensor cores for large batches, with the GLU hidden
+// vectors' region, free until the up projection, as its scratch) and the
+// dispatch kernel.
+cudaError_t route_dispatch_ws(const moe_dims &d, int T, const void *x, const void *w_router,
+                              const WsLayout &L, void *ws, cudaStream_t st) {
+    int32_t *idx = at<int32_t>(ws, L.idx);
+    float *gate = at<float>(ws, L.gate);
+    int32_t *counts = at<int32_t>(ws, L.counts);
+    int32_t *offsets = at<int32_t>(ws, L.offsets);
+    int32_t *perm = at<int32_t>(ws, L.perm);
+    int32_t *inv = at<int32_t>(ws, L.inv_perm);
+    if (T == 1 && small_route_ok(d, T))
+        return route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv,
+                                        st);
+    if (cluster_route_ok(d, T))
+        return route_dispatch_cluster_any(d, T, x, w_router, idx, gate, counts, offsets, perm,
+                                          inv, st);
+    if (small_route_ok(d, T))
+        return route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv,
+                                        st);
+    cudaError_t e = route_any(d, T, x, w_router, nullptr, idx, gate, st, at<float>(ws, L.h),
+                              L.xs > L.h ? L.xs - L.h : 0);
+    if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
+    return e;
 }
 
 }  // namespace
@@ -1311,29 +1347,13 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
     if (!ws || !aligned16(ws) || ws_bytes < L.total) return MOE_ERR_WORKSPACE;
     cudaStream_t st = (cudaStream_t)stream;
     const moe_dims &d = *dims;
-    int32_t *idx = at<int32_t>(ws, L.idx);
     float *gate = at<float>(ws, L.gate);
-    int32_t *counts = at<int32_t>(ws, L.counts);
     int32_t *offsets = at<int32_t>(ws, L.offsets);
     int32_t *perm = at<int32_t>(ws, L.perm);
     int32_t *inv = at<int32_t>(ws, L.inv_perm);
     float *h = at<float>(ws, L.h);
 
-    cudaError_t e;
-    if (T == 1 && small_route_ok(d, T)) {
-        e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
-    } else if (cluster_route_ok(d, T)) {
-        e = route_dispatch_cluster_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv,
-                                       st);
-    } else if (small_route_ok(d, T)) {
-        e = route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv, st);
-    } else {
-        // the GLU hidden vectors' region is free until the up projection:
-        // scratch for the tensor-core router
-        e = route_any(d, T, x, w_router, nullptr, idx, gate, st, h,
-                      L.xs > L.h ? L.xs - L.h : 0);
-        if (e == cudaSuccess) e = dispatch_any(d, T, idx, counts, offsets, perm, inv, st);
-    }
+    cudaError_t e = route_dispatch_ws(d, T, x, w_router, L, ws, st);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     if (use_stream_path(d, T)) {
         // decode, bf16: bulk-copy pipelined kernels, combine fused into the
@@ -1366,6 +1386,79 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
         float *y = at<float>(ws, L.y);
         e = launch_down_gemv(d, T, h, perm, offsets, w2, nullptr, y, nullptr, nullptr, false, st);
         if (e == cudaSuccess) e = combine_any(d, T, y, inv, gate, residual_opt, out, st);
+    }
+    return cuda_status(e);
+}
+
+moe_status moe_layer_forward_experts(const moe_dims *dims, int32_t T, const void *x,
+                                     const void *w_router, int32_t e_begin, int32_t e_end,
+                                     const void *w1_local, const void *v1_local,
+                                     const void *w2_local, const float *residual_opt,
+                                     float *partial_out, void *ws, size_t ws_bytes,
+                                     moe_stream_t stream) {
+    MOE_INJECT("moe_layer_forward_experts");
+    moe_status s = check_dims(dims);
+    if (s != MOE_OK) return s;
+    if ((s = check_T(dims, T)) != MOE_OK) return s;
+    if (e_begin < 0 || e_end > dims->n_experts || e_begin >= e_end) return MOE_ERR_INVALID_ARG;
+    if (T == 0) return MOE_OK;
+    if (!ok_ptr(x) || !ok_ptr(w_router) || !ok_ptr(w1_local) || !ok_ptr(v1_local) ||
+        !ok_ptr(w2_local) || !ok_opt(residual_opt) || !ok_ptr(partial_out))
+        return MOE_ERR_INVALID_ARG;
+    const WsLayout L = ws_layout(*dims, T);
+    if (!ws || !aligned16(ws) || ws_bytes < L.total) return MOE_ERR_WORKSPACE;
+    cudaStream_t st = (cudaStream_t)stream;
+    const moe_dims &d = *dims;
+    float *gate = at<float>(ws, L.gate);
+    int32_t *offsets = at<int32_t>(ws, L.offsets);
+    int32_t *perm = at<int32_t>(ws, L.perm);
+    int32_t *inv = at<int32_t>(ws, L.inv_perm);
+    float *h = at<float>(ws, L.h);
+
+    // every node routes and dispatches over all E experts (the replicated
+    // router of Sec. 4.3) ...
+    cudaError_t e = route_dispatch_ws(d, T, x, w_router, L, ws, st);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    // ... and runs the expert kernels over its own experts only: their
+    // dispatch offsets start at offsets[e_begin] and address the same sorted
+    // slot arrays, and the weights hold experts e_begin..e_end-1
+    moe_dims dl = d;
+    dl.n_experts = e_end - e_begin;
+    dl.out_dtype = MOE_F32;
+    const int32_t *loff = offsets + e_begin;
+    if (use_stream_path(d, T)) {
+        e = launch_up_glu_stream(dl, T, x, perm, loff, w1_local, v1_local, h, st);
+        if (e == cudaSuccess)
+            e = launch_down_stream(dl, T, h, loff, inv, w2_local, gate, residual_opt, partial_out,
+                                   nullptr, true, st);
+        return cuda_status(e);
+    }
+    if (tc_path_ok(d)) {
+        void *xs = at<void>(ws, L.xs);
+        float *y = at<float>(ws, L.y);
+        float *y_tail = T <= kStreamKMaxTokens ? at<float>(ws, L.y_tail) : nullptr;
+        e = launch_gather_rows(d, T, x, perm, xs, st);
+        if (e == cudaSuccess) e = launch_gemm_up_tc(dl, T, xs, loff, w1_local, v1_local, h, st);
+        if (e == cudaSuccess)
+            e = launch_gemm_down_tc(dl, T, h, loff, w2_local, y, st, nullptr, y_tail);
+        if (e == cudaSuccess)
+            e = combine_any(dl, T, y, inv, gate, residual_opt, partial_out, st, y_tail, loff,
+                            dl.n_experts);
+        return cuda_status(e);
+    }
+    e = launch_up_glu_gemv(dl, T, x, perm, loff, w1_local, v1_local, h, st);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    if (T <= kFusedCombineMaxTokens) {
+        // the fused down projection sums over the experts it is given
+        e = launch_down_gemv(dl, T, h, perm, loff, w2_local, gate, nullptr, residual_opt,
+                             partial_out, true, st);
+    } else {
+        float *y = at<float>(ws, L.y);
+        e = launch_down_gemv(dl, T, h, perm, loff, w2_local, nullptr, y, nullptr, nullptr, false,
+                             st);
+        if (e == cudaSuccess)
+            e = combine_any(dl, T, y, inv, gate, residual_opt, partial_out, st, nullptr, loff,
+                            dl.n_experts);
     }
     return cuda_status(e);
 }

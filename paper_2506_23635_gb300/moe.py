@@ -27,7 +27,8 @@ _STATUS = {
 # Every function the header declares (checked by the CPU tests).
 EXPORTS = (
     "moe_workspace_size", "moe_route", "moe_dispatch", "moe_expert_ffn",
-    "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc", "moe_status_string",
+    "moe_combine", "moe_layer_forward", "moe_layer_forward_noalloc",
+    "moe_layer_forward_experts", "moe_status_string",
     "moe_prenorm", "moe_stack_workspace_size", "moe_stack_forward",
     "moe_selftest_wait_timeout", "moe_dense_workspace_size", "moe_layer_forward_dense",
     "moe_get_last_error", "moe_launch_count", "moe_profile_enable",
@@ -97,6 +98,7 @@ def lib() -> ctypes.CDLL:
         "moe_combine": [DP, I32, P, P, P, P, P, P],
         "moe_layer_forward": [DP, I32, P, P, P, P, P, P, P, P, SZ, P],
         "moe_layer_forward_noalloc": [DP, I32, P, P, P, P, P, P, P, P],
+        "moe_layer_forward_experts": [DP, I32, P, P, I32, I32, P, P, P, P, P, P, SZ, P],
         "moe_prenorm": [DP, I32, P, P, ctypes.c_float, P],
         "moe_selftest_wait_timeout": [ctypes.c_uint64, P, P],
         "moe_dense_workspace_size": [DP, I32, ctypes.POINTER(SZ)],
@@ -230,6 +232,25 @@ def layer_forward(d: Dims, x, w_r, w1, v1, w2, residual=None, out=None, ws=None,
     _check(lib().moe_layer_forward(ctypes.byref(d), T, _ptr(x), _ptr(w_r), _ptr(w1), _ptr(v1),
                                    _ptr(w2), _ptr(residual), _ptr(out), _ptr(ws), ws.numel(),
                                    _stream(stream)), "moe_layer_forward")
+    return out
+
+
+def layer_forward_experts(d: Dims, x, w_r, e_begin: int, e_end: int, w1_local, v1_local,
+                          w2_local, residual=None, out=None, ws=None, stream=None):
+    """One node's share of an expert-parallel layer (Sec. 4.3): the whole
+    routing, then only experts e_begin..e_end-1, whose weights are
+    ``w1_local`` [n, F, D], ``v1_local`` [n, F, D], ``w2_local`` [n, D, F]
+    (n = e_end - e_begin).  Returns the fp32 partial [T, D] (plus
+    ``residual`` [T, D] fp32 when given)."""
+    T = x.shape[0]
+    if out is None:
+        out = torch.empty((T, d.d_model), dtype=torch.float32, device=x.device)
+    ws = alloc_workspace(d, T, x.device) if ws is None else ws
+    _check(lib().moe_layer_forward_experts(ctypes.byref(d), T, _ptr(x), _ptr(w_r), e_begin,
+                                           e_end, _ptr(w1_local), _ptr(v1_local),
+                                           _ptr(w2_local), _ptr(residual), _ptr(out), _ptr(ws),
+                                           ws.numel(), _stream(stream)),
+           "moe_layer_forward_experts")
     return out
 
 

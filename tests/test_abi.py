@@ -127,6 +127,23 @@ def test_layer_and_ffn_validation(lib):
 
 
 @no_gpu
+def test_expert_range_validation(lib):
+    L = lib.lib()
+    d = lib.dims(**DBRX)
+    need = lib.workspace_size(d, 8)
+    f = lambda b, e, T=8, ws=A, n=need, x=A, out=A: L.moe_layer_forward_experts(
+        ctypes.byref(d), T, x, A, b, e, A, A, A, None, out, ws, n, None)
+    for b, e in ((0, 0), (4, 3), (-1, 4), (0, 17), (16, 16)):
+        assert f(b, e) == 1, (b, e)
+    assert f(0, 0, T=0) == 1  # the range is checked even when there is no token
+    assert f(0, 16, T=0) == 0
+    assert f(0, 8, x=None) == 1
+    assert f(0, 8, out=MIS) == 1
+    assert f(0, 8, ws=None) == 3
+    assert f(8, 16, n=need - 1) == 3
+
+
+@no_gpu
 def test_noalloc_validation(lib):
     L = lib.lib()
     d = lib.dims(**DBRX)
