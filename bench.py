@@ -41,6 +41,8 @@ UNIT = "us/token-step"
 SEED = 1234
 POOL = 64  # distinct token inputs cycled through by the timed steps
 HBM_FALLBACK_GBS = 6800.0
+BF16_FALLBACK_TFLOPS = 1900.0
+BF16_SUSTAINED_FALLBACK_TFLOPS = 1700.0
 
 # name: (shape, tokens per step)
 WORKLOADS = {
@@ -288,6 +290,34 @@ def token_pool(shape, T, seed, pool=POOL):
     return np.stack(xs), w_r
 
 
+def workload_config(workload, shape, T, U, world):
+    """The line's ``config``, the same for both arms of a workload: its
+    shape, tokens per step, the mean number of distinct experts a step reads
+    (from the routing of the token pool), the L2 note and the parallelism."""
+    D, F = shape.d_model, shape.ffn_hidden
+    gb = U * 3 * D * F * (2 if shape.dtype == "bf16" else 4) / 1e9
+    return {
+        "workload": workload, "d_model": D, "ffn_hidden": F, "n_experts": shape.n_experts,
+        "top_k": shape.top_k, "tokens_per_step": T, "distinct_experts_per_step": U,
+        "l2": (f"inputs larger than L2: each step streams its selected experts' weights "
+               f"({gb:.2f} GB) vs 129 MB L2" if gb > 0.129 else
+               f"inputs smaller than L2 ({gb * 1e3:.1f} MB of selected weights per step)"),
+        "parallelism": "replicas only" if world > 1 else "single GPU",
+    }
+
+
+def oracle_distinct_experts(xs_host, w_r_host, shape):
+    """Mean distinct experts per step of a token pool, from the oracle's
+    routing (equal to the GPU's: routing is bit-exact)."""
+    import oracle
+
+    U = []
+    for x in xs_host:
+        idx, _ = oracle.topk_gates(oracle.router_logits(x, w_r_host, shape.dtype), shape.top_k)
+        U.append(len(set(idx.reshape(-1).tolist())))
+    return float(np.mean(U))
+
+
 def algorithmic_flops(kernel: str, shape: gen.LayerShape, T: int) -> float:
     """Multiply-adds x 2 a GEMM kernel must do per launch."""
     D, F, K = shape.d_model, shape.ffn_hidden, shape.top_k
@@ -310,6 +340,13 @@ class Layer:
         self.d = moe.dims(shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k,
                           torch.bfloat16)
         self.stream = torch.cuda.current_stream(dev)
+        self._host = None
+
+    def host_weights(self):
+        """The expert weights' bytes on the host (copied once, for the oracle)."""
+        if self._host is None:
+            self._host = host_weights(self.shape, self.w)
+        return self._host
 
     def inputs(self, T, pool):
         import torch
@@ -390,12 +427,16 @@ def tensor_roofline(kstats, shape, T, workload):
     avg_s = ms_dom / n_dom / 1e3
     flops = algorithmic_flops(dominant, shape, T)
     peaks, src = measured_peaks()
-    peak = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
+    # the GEMM is timed in a loop of a few tens of milliseconds (its own
+    # launches, event-bracketed): the burst figure is its peak; the
+    # seconds-long sustained figure is reported beside it
+    peak = float(peaks.get("bf16_tflops", BF16_FALLBACK_TFLOPS))
+    sustained = float(peaks.get("bf16_tflops_sustained", BF16_SUSTAINED_FALLBACK_TFLOPS))
     achieved = flops / avg_s / 1e12
     return {"kernel": dominant, "bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
             "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-            "peak_source": f"{src} bf16_tflops_sustained (cuBLAS bf16 GEMM, seconds-long loop)",
-            "frac_of_burst_peak": round(achieved / float(peaks.get("bf16_tflops", 1910.6)), 4),
+            "peak_source": f"{src} bf16_tflops (cuBLAS bf16 8192^3 GEMM, burst)",
+            "frac_of_sustained_peak": round(achieved / sustained, 4),
             "traffic": committed_traffic(dominant, workload),
             "algorithmic_flops_per_launch": flops, "avg_launch_us": round(avg_s * 1e6, 2),
             "timing": "CUDA events around each launch on its stream, over a second pass "
@@ -410,17 +451,19 @@ def eq1_refit(shape, T, U, ms):
     peaks, _ = measured_peaks()
     m = perf_model.gb300_moe_layer_time(
         T, U, float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS)) * 1e9,
-        float(peaks.get("bf16_tflops", 1910.6)) * 1e12, shape.d_model, shape.ffn_hidden,
+        float(peaks.get("bf16_tflops", BF16_FALLBACK_TFLOPS)) * 1e12, shape.d_model,
+        shape.ffn_hidden,
         shape.top_k)
     return {"model_ms": round(m["time"] * 1e3, 4), "bound": m["bound"],
             "measured_over_model": round(ms / (m["time"] * 1e3), 3)}
 
 
-def measure_extra(layer, workload, steps, warmup):
-    """A secondary workload of the same layer: a few timed steps."""
+def measure_extra(layer, workload, steps, warmup, cpu_seconds=None):
+    """A secondary workload of the same layer: a few timed steps, and (with
+    ``cpu_seconds``) the oracle timed on a bounded sample of it."""
     shape, T = WORKLOADS[workload]
     pool = 4 if T >= PREFILL_MIN_TOKENS else 16
-    _, _, xs, w_r, ws, out = layer.inputs(T, pool)
+    xs_host, w_r_host, xs, w_r, ws, out = layer.inputs(T, pool)
     w1, v1, w2 = layer.w
     d, moe = layer.d, layer.moe
 
@@ -445,6 +488,9 @@ def measure_extra(layer, workload, steps, warmup):
         r["achieved_hbm_gbs_step"] = round(step_bytes / (ms / 1e3) / 1e9, 1)
         peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
         r["frac_of_hbm_step"] = round(step_bytes / (ms / 1e3) / 1e9 / peak, 4)
+    if cpu_seconds:
+        r["cpu_baseline"] = cpu_baseline(shape, T, xs_host, w_r_host, layer.host_weights(),
+                                         cpu_seconds)
     return r
 
 
@@ -459,20 +505,15 @@ def measure_stack(moe, dev, n_layers=16, steps=64, batches=(1, 8), graph=True, d
 
     shape = gen.DBRX
     D, F, E, K = shape.d_model, shape.ffn_hidden, shape.n_experts, shape.top_k
-    layers = []
-    for l in range(n_layers):
-        w_r = gen.host_to_torch(gen.host_normal((D, E), gen.W_STD, "bf16", SEED, "stack-w_r", l),
-                                "bf16", dev)
-        layers.append((w_r,) + gen.device_expert_weights(shape, SEED + 1 + l, dev, layer=l))
+    layers = gen.device_stack_layers(shape, n_layers, SEED, dev)
     sw = moe.StackWeights(layers)
     d = moe.dims(D, F, E, K, torch.bfloat16, torch.bfloat16, torch.float32)
     stream = torch.cuda.current_stream(dev)
     res = {"layers": n_layers, "resident_weight_gb": round(n_layers * 3 * E * D * F * 2 / 1e9, 2),
            "steps": steps}
     for T in batches:
-        xs = torch.stack([gen.host_to_torch(gen.host_normal((T, D), 1.0, "bf16", SEED, "stack-x",
-                                                            T, s), "bf16", dev).float()
-                          for s in range(steps)])
+        xs = torch.stack([gen.host_to_torch(gen.stack_batch(shape, T, SEED, s), "bf16",
+                                            dev).float() for s in range(steps)])
         resid = torch.empty((T, D), dtype=torch.float32, device=dev)
         ws = torch.empty(moe.stack_workspace_size(d, T), dtype=torch.uint8, device=dev)
 
@@ -693,6 +734,15 @@ def measure_dense(layer, T, steps=100, warmup=3):
             "kernels": kernel_table(kstats)}
 
 
+def decoder_config(workload, shape, T, prefill, ctx_len=2048):
+    """The ``config`` of a decoder-layer workload, the same for both arms."""
+    return {"workload": workload, "d_model": shape.d_model, "ffn_hidden": shape.ffn_hidden,
+            "n_experts": shape.n_experts, "top_k": shape.top_k, "tokens_per_step": T,
+            "mode": ("prefill of one sequence, causal" if prefill
+                     else f"decode, {T} sequences at context {ctx_len}"),
+            "attention": "48 query / 8 key-value heads of 128 (D_qkv = 8192)"}
+
+
 def run_decoder(args, moe, dev, dist, rank, world):
     """A whole decoder layer as the measured step (device-resident inputs);
     one JSON line with the step time per token and the attention block's
@@ -713,11 +763,7 @@ def run_decoder(args, moe, dev, dist, rank, world):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,0.02^2) bf16 weights, N(0,1) tokens, KV cache "
                 "pre-filled with synthetic entries)",
-        "config": {"workload": args.workload, "d_model": shape.d_model,
-                   "ffn_hidden": shape.ffn_hidden, "n_experts": shape.n_experts,
-                   "top_k": shape.top_k, "tokens_per_step": T,
-                   "mode": r.get("mode", f"decode, {T} sequences at context {r.get('context')}"),
-                   "attention": "48 query / 8 key-value heads of 128 (D_qkv = 8192)"},
+        "config": decoder_config(args.workload, shape, T, prefill),
         "attention_block": r["attention_block"], "kernels": r["kernels"],
         "gpu_launches": int(r["launches_per_step"] * args.steps),
     }
@@ -821,8 +867,11 @@ def run_ours(args):
     # contract): the 2048-token prefill and the decode batch sweep ----
     extra = {}
     if not args.no_extra and args.workload == "dbrx-decode-t1":
-        extra["prefill"] = measure_extra(layer, "dbrx-prefill-t2048", 20, 3)
-        extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5)
+        # the oracle beside every config (a third of the headline's budget
+        # each), on rank 0 of a one-GPU run only
+        cpu_s = None if (args.no_cpu_baseline or world > 1) else args.cpu_seconds / 3
+        extra["prefill"] = measure_extra(layer, "dbrx-prefill-t2048", 20, 3, cpu_s)
+        extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5, cpu_s)
                                  for t in (2, 4, 8, 16, 32, 64)]
         extra["busy_full_loading"] = [measure_dense(layer, t) for t in (1, 8)]
         extra["decoder_layer"] = [measure_decoder_layer(layer, t) for t in (1, 8)]
@@ -851,14 +900,8 @@ def run_ours(args):
         "ms_per_step": round(ms_max, 5), "higher_is_better": hib,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,0.02^2) bf16 weights, N(0,1) tokens, gap-conditioned router)",
-        "config": {
-            "workload": args.workload, "d_model": D, "ffn_hidden": F, "n_experts": E,
-            "top_k": K, "tokens_per_step": T, "accumulate": "f32",
-            "distinct_experts_per_step": U_mean,
-            "l2": "inputs larger than L2: each step streams its selected experts' weights "
-                  f"({U_mean * 3 * D * F * 2 / 1e9:.2f} GB) vs 129 MB L2",
-            "parallelism": "replicas only" if world > 1 else "single GPU",
-        },
+        "config": workload_config(args.workload, shape, T, U_mean, world),
+        "accumulate": "f32",
         "roofline": (tensor_roofline(kstats, shape, T, args.workload) if prefill
                      else hbm_roofline(kstats, shape, T, U_mean, args.workload)),
         "kernels": kernel_table(kstats),
@@ -875,7 +918,7 @@ def run_ours(args):
     if extra:
         line["extra"] = extra
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(shape, T, xs_host, w_r_host, (w1, v1, w2),
+        line["cpu_baseline"] = cpu_baseline(shape, T, xs_host, w_r_host, layer.host_weights(),
                                             args.cpu_seconds)
     print(json.dumps(line), flush=True)
     if dist is not None:
@@ -891,13 +934,14 @@ def host_weights(shape, weights_dev):
     return [gen.torch_to_host(t, shape.dtype) for t in weights_dev]
 
 
-def cpu_baseline(shape, T, xs_host, w_r_host, weights_dev, budget_s):
+def cpu_baseline(shape, T, xs_host, w_r_host, weights_host, budget_s):
     """The oracle, as it stands, on a bounded sample of the same workload:
     whole decode token-steps from the same token pool (prefill: tokens of the
-    first batch), until the time budget is used."""
+    first batch), until the time budget is used.  weights_host: the expert
+    tensors' bytes on the host."""
     import oracle
 
-    w1, v1, w2 = host_weights(shape, weights_dev)
+    w1, v1, w2 = weights_host
     prefill = T >= PREFILL_MIN_TOKENS
     n, t_total = 0, 0.0
     if prefill:
@@ -1016,9 +1060,9 @@ def run_reference(args):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms, 3), "higher_is_better": hib, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": f"synthetic ({src})",
-        "config": {"workload": args.workload, "d_model": shape.d_model,
-                   "ffn_hidden": shape.ffn_hidden, "n_experts": shape.n_experts,
-                   "top_k": shape.top_k, "tokens_per_step": T},
+        "config": (decoder_config(args.workload, shape, T, prefill) if decoder else
+                   workload_config(args.workload, shape, T,
+                                   oracle_distinct_experts(xs_host, w_r_host, shape), world)),
         "cpu_baseline": {"value": value, "unit": unit, "kind": "oracle",
                          "cores": oracle.num_threads(), "sample": sample},
         "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0,

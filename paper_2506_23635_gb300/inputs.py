@@ -301,6 +301,28 @@ def device_expert_weights(shape: LayerShape, seed: int, device, layer: int = 0):
     return w1, v1, w2
 
 
+def stack_router(shape: LayerShape, seed: int, layer: int) -> np.ndarray:
+    """Router W_r [D, E] of layer ``layer`` of a stack of MoE layers."""
+    return host_normal((shape.d_model, shape.n_experts), W_STD, shape.dtype, seed, "stack-w_r",
+                       layer)
+
+
+def device_stack_layers(shape: LayerShape, n_layers: int, seed: int, device):
+    """A stack of independently seeded layers on ``device``: per layer the
+    tuple (W_r, W1, V1, W2), the experts drawn on the device."""
+    layers = []
+    for l in range(n_layers):
+        w_r = host_to_torch(stack_router(shape, seed, l), shape.dtype, device)
+        layers.append((w_r,) + device_expert_weights(shape, seed + 1 + l, device, layer=l))
+    return layers
+
+
+def stack_batch(shape: LayerShape, T: int, seed: int, step: int) -> np.ndarray:
+    """The fresh tokens [T, D] of decode step ``step`` of a stack (reading
+    C10: every step takes new seeded tokens)."""
+    return host_normal((T, shape.d_model), X_STD, shape.dtype, seed, "stack-x", T, step)
+
+
 # --------------------------------------------------------------------------
 # self-attention block of a decoder layer
 # --------------------------------------------------------------------------
