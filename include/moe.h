@@ -330,9 +330,9 @@ int32_t moe_profile_read(moe_kernel_stat *stats, int32_t max_stats);
  *   - causal softmax attention scaled by 1/sqrt(head_dim); no biases;
  *   - the pre-norm residual block  resid += w_o . Attn(RMSNorm0(resid)),
  *     RMSNorm0 as in moe_prenorm (no learned scale).
- * Storage: the normalised input, the cached keys and values and the
- * attention output ctx are bf16; projections accumulate in fp32; the
- * residual stream is fp32.
+ * Storage: the normalised input, the rotated queries (as the attention
+ * reads them), the cached keys and values and the attention output ctx are
+ * bf16; projections accumulate in fp32; the residual stream is fp32.
  *
  * Layouts (row-major): w_qkv [(Hq + 2 Hkv) dh, D] bf16 -- the query rows,
  * then the key rows, then the value rows; w_o [D, Hq dh] bf16; k_cache and
@@ -374,10 +374,14 @@ moe_status moe_sa_qkv(const moe_sa_dims *dims, int32_t T, const void *x_norm,
                       void *v_cache, void *ws, size_t ws_bytes, moe_stream_t stream);
 
 /* moe_sa_attend: ctx[t, h dh .. (h+1) dh) = softmax over positions
- * 0..pos[t] of q[t,h] . K / sqrt(dh), applied to V (bf16 out).  As in
- * moe_sa_forward, every 128 consecutive tokens that are positions
- * p0..p0+127 of one sequence (a prefill chunk) are attended on the tensor
- * cores from q rounded to bf16; the other tokens use q as given. */
+ * 0..pos[t] of bf16(q[t,h]) . K / sqrt(dh), applied to V (bf16 out): the
+ * queries are read rounded to bf16.  As in moe_sa_forward, every 128
+ * consecutive tokens that are positions p0..p0+127 of one sequence (a
+ * prefill chunk) are attended by the tensor-core flash attention, and the
+ * tokens of a call without such a chunk (decode steps) by the tensor-core
+ * decode attention; other tokens by the CUDA-core kernel.
+ * MOE_ATTN_CUDA_CORES=1 in the environment keeps decode steps on the
+ * CUDA-core kernel. */
 moe_status moe_sa_attend(const moe_sa_dims *dims, int32_t T, const float *q,
                          const int32_t *seq, const int32_t *pos, int32_t n_seq,
                          int32_t max_len, const void *k_cache, const void *v_cache,

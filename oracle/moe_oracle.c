@@ -331,8 +331,9 @@ void orc_round_bf16(size_t n, const double *in, double *out)
  *     sequence s attends to cache positions 0..p of s; the keys and values of
  *     all tokens of a call are written to the cache before any token attends.
  *   Block: resid += Wo . ctx, with ctx the attention of RMSNorm0(resid).
- *     With bf16 storage the normalised input, the cached keys and values and
- *     ctx are rounded to bf16: each is stored and read back by the next step.
+ *     With bf16 storage the normalised input, the rotated queries, the
+ *     cached keys and values and ctx are rounded to bf16: each is an
+ *     activation the paper's bf16 inference stores and the next step reads.
  *
  * Cache layout: [n_seq, Hkv, L, dh] (keys and values alike), as doubles
  * holding exactly the stored values. */
@@ -427,6 +428,7 @@ int orc_sa_forward(int T, int D, int Hq, int Hkv, int dh, double base, double ep
     orc_rope(T, Hq, dh, base, pos, q);
     orc_rope(T, Hkv, dh, base, pos, k);
     if (round) {
+        orc_round_bf16((size_t)T * nq, q, q);
         orc_round_bf16((size_t)T * nkv, k, k);
         orc_round_bf16((size_t)T * nkv, v, v);
     }

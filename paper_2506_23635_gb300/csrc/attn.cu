@@ -31,6 +31,7 @@
 //   projection     W_o . ctx (the same two kernels), its partial sums added to
 //                  the residual by k_residual_add.
 #include <math.h>
+#include <stdlib.h>
 
 #include <algorithm>
 
@@ -289,8 +290,12 @@ k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__
     const int chunk = (n + n_split - 1) / n_split;
     const int j0 = min(n, s * chunk), j1 = min(n, j0 + chunk);
     const float scale = 1.0f / sqrtf((float)kHeadDim);
+    // the queries as stored activations: rounded to bf16, as the tensor-core
+    // kernels read them
     for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x)
-        qs[i / kHeadDim][i % kHeadDim] = q[((size_t)t * Hq + g * G) * kHeadDim + i] * scale;
+        qs[i / kHeadDim][i % kHeadDim] =
+            __bfloat162float(__float2bfloat16_rn(q[((size_t)t * Hq + g * G) * kHeadDim + i])) *
+            scale;
     __syncthreads();
 
     float m[G], l[G], acc[G][4];
@@ -685,21 +690,49 @@ cudaError_t qkv_rope(const SaCall &c, const void *xn, const void *w_qkv, const i
                       dim3(kRopeRows * kHeadDim / 2), 0, c.st, args);
 }
 
-// Attention over the caches: per-split partials, then their merge.
+// Whether decode-type calls (no full prefill tile) attend on the tensor
+// cores; MOE_ATTN_CUDA_CORES=1 keeps them on the CUDA-core kernel.
+bool decode_tc() {
+    static const bool off = [] {
+        const char *v = getenv("MOE_ATTN_CUDA_CORES");
+        return v && v[0] == '1';
+    }();
+    return !off && attn_decode_tc_ok();
+}
+
+// Whether a call of T tokens wants the bf16 copy of its queries (one of the
+// tensor-core attention kernels reads it).
+bool wants_q16(int T) { return tc_attention(T) || decode_tc(); }
+
+// Attention over the caches.  A call with 128 or more tokens: full prefill
+// tiles on the tensor cores, the rest on the CUDA-core kernel (one split);
+// a smaller call: the decode kernel on the tensor cores.  Per-split
+// partials, when there are several splits, are merged last.
 cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const int32_t *pos,
                    int n_seq, int L, const void *kc, const void *vc, void *ctx,
                    const bf16 *q16 = nullptr) {
     const int Hq = c.d.n_heads, Hkv = c.d.n_kv_heads, G = Hq / Hkv;
     int ns = n_split_for(c.T, Hkv, L);
     int *tile_ok = nullptr;
-    if (q16) {  // full prefill tiles on the tensor cores, the rest below (one split)
+    float *ml = at<float>(c.ws, c.L.part_ml), *acc = at<float>(c.ws, c.L.part_acc);
+    bf16 *cp = static_cast<bf16 *>(ctx);
+    if (q16 && tc_attention(c.T)) {  // full prefill tiles on the tensor cores, the rest below
         tile_ok = at<int>(c.ws, c.L.tile_ok);
         cudaError_t e = launch_attn_prefill_tc(c.T, Hq, Hkv, n_seq, L, seq, pos, q16, kc, vc, ctx,
                                                tile_ok, c.st);
         if (e != cudaSuccess) return e;
         ns = 1;
+    } else if (q16 && decode_tc()) {
+        ns = attn_decode_tc_splits(c.T, Hkv, L, split_cap(c.T, Hkv));
+        cudaError_t e = launch_attn_decode_tc(c.T, Hq, Hkv, n_seq, L, ns, seq, pos, q16, kc, vc,
+                                              ml, acc, ctx, c.st);
+        if (e != cudaSuccess || ns == 1) return e;
+        const float *mlc = ml, *accc = acc;
+        void *args[] = {&ns, &mlc, &accc, &cp};
+        LaunchScope ls("attn_merge", c.st);
+        return launch_pdl((const void *)k_attn_merge, dim3(c.T * Hq),
+                          dim3(kHeadDim * kMergeGroups), 0, c.st, args);
     }
-    float *ml = at<float>(c.ws, c.L.part_ml), *acc = at<float>(c.ws, c.L.part_acc);
     const void *kern = nullptr;
     switch (G) {
         case 1: kern = (const void *)k_attn_partial<1>; break;
@@ -713,7 +746,6 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     }
     int Hqv = Hq, Hkvv = Hkv, nsq = n_seq, Lv = L;
     const bf16 *kcp = static_cast<const bf16 *>(kc), *vcp = static_cast<const bf16 *>(vc);
-    bf16 *cp = static_cast<bf16 *>(ctx);
     {
         const int *tok = tile_ok;
         void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &seq, &pos, &q, &kcp, &vcp, &ml, &acc, &cp,
@@ -820,7 +852,7 @@ moe_status sa_forward_impl(const moe_sa_dims *dims, int32_t T, const int32_t *se
                              dim3(kNormThreads), 0, c.st, args);
         if (e != cudaSuccess) return MOE_ERR_CUDA;
     }
-    bf16 *q16 = tc_attention(T) ? at<bf16>(ws, c.L.q16) : nullptr;
+    bf16 *q16 = wants_q16(T) ? at<bf16>(ws, c.L.q16) : nullptr;
     cudaError_t e = qkv_rope(c, xn, w_qkv, seq, pos, n_seq, max_len, q, k_cache, v_cache, q16);
     if (e == cudaSuccess) e = attend(c, q, seq, pos, n_seq, max_len, k_cache, v_cache, ctx, q16);
     if (e == cudaSuccess) e = out_proj(c, ctx, w_o, resid, xn_next, eps);
@@ -868,10 +900,10 @@ moe_status moe_sa_attend(const moe_sa_dims *dims, int32_t T, const float *q, con
         return MOE_ERR_INVALID_ARG;
     if ((s = check_ws(dims, T, ws, ws_bytes)) != MOE_OK) return s;
     SaCall c{*dims, T, (cudaStream_t)stream, ws, sa_ws(*dims, T)};
-    // the same kernels as the whole block: full prefill tiles on the tensor
-    // cores, from a bf16 copy of the queries
+    // the same kernels as the whole block: the tensor-core attention
+    // kernels, from a bf16 copy of the queries
     bf16 *q16 = nullptr;
-    if (tc_attention(T)) {
+    if (wants_q16(T)) {
         q16 = at<bf16>(ws, c.L.q16);
         long long n4 = (long long)T * dims->n_heads * dims->head_dim / 4;
         const float *qc = q;

@@ -1,0 +1,480 @@
+// Decode attention on the tcgen05 tensor cores: tokens that attend to a key/
+// value cache one by one (a decode step: one token per sequence).
+//
+// A decode token's grouped-query attention is small in the query dimension
+// (the G <= 8 query heads that share one key/value head) and long in the
+// position dimension, so the positions are the MMA's M and the heads its N:
+//
+//   S^T = K_j Q^T       M = 128 positions, N = 16 (the G heads, zero-
+//                       padded), K = 128 dims; K_j and Q both K-major
+//   O^T += V_j^T P_j^T  M = 128 dims, N = 16 heads, K = 128 positions; V_j
+//                       as it lies in the cache (dims contiguous: an
+//                       MN-major A operand), P_j K-major in shared memory
+//
+// with S^T and O^T in tensor memory (lane = position, resp. dim; column =
+// head).  One CTA per (position split s, token t, key/value head g), over
+// the split's positions [j0, j1) of t's sequence in tiles of 128:
+//
+//   warp 0      TMA: the group's bf16 query rows once, then key and value
+//               tiles into two-stage rings (each 32 KB: two boxes of 64
+//               dims with the 128-byte swizzle);
+//   warp 1      tensor memory (S^T twice, O^T: 48 of 64 columns) and the
+//               MMAs: S_{j+1} is issued as soon as its key tile has landed
+//               and the softmax has read S_{j-1}, O += P_j V_j once P_j is
+//               written;
+//   warps 2-5   softmax, one thread per position of the tile (its tensor-
+//               memory lane): the tile maximum of every head across the
+//               128 positions (a warp maximum, then the four warps' through
+//               shared memory), the base-2 exponent of the 1/sqrt(128)-
+//               scaled scores against a per-head base that moves only when
+//               the maximum passes it by more than 8 (then O^T is rescaled
+//               in tensor memory, each thread its dim's row), bf16
+//               probabilities written into P_j (rows = heads, positions
+//               contiguous, 128-byte swizzle), rows of V_j past the split's
+//               last position zeroed (0 * NaN is NaN; those cache rows may
+//               hold anything).
+//
+// The end: each thread owns dim r of O^T; per head the row sums of the four
+// warps are added, and the CTA writes either ctx (a single split) or the
+// split's (maximum, sum, weighted values) for k_attn_merge, in the form of
+// the CUDA-core kernel's partials.
+//
+// Numerics as the prefill flash attention: bf16 queries and probabilities,
+// fp32 scores and accumulation; the row sum takes the probabilities as
+// stored.  Every wait is bounded (ptx.cuh); once one gives up the thread
+// skips the later waits and the kernel ends.
+#include <math.h>
+
+#include "tc.cuh"
+
+namespace moe {
+namespace {
+
+using namespace tc;
+
+constexpr int kDecPos = 128;   // positions per key/value tile: the MMA's M
+constexpr int kDecN = 16;      // the MMA's N: the group's query heads, zero-padded
+constexpr int kDecMaxG = 8;    // query heads per key/value head
+constexpr int kDecThreads = 6 * 32;
+constexpr uint32_t kDecHalf = kDecPos * 128;  // one 64-dim box of a key/value tile: 16 KB
+constexpr uint32_t kDecTile = 2 * kDecHalf;   // 32 KB
+constexpr uint32_t kDecNHalf = kDecN * 128;   // 16 rows x 64 elements: 2 KB
+constexpr uint32_t kDecQ = 2 * kDecNHalf;     // query rows, 128 dims
+constexpr uint32_t kDecP = 2 * kDecNHalf;     // probabilities, 128 positions
+// shared memory (1024-byte aligned): K[2], V[2], Q, P[2], header
+constexpr uint32_t kDecOffK = 0;
+constexpr uint32_t kDecOffV = kDecOffK + 2 * kDecTile;
+constexpr uint32_t kDecOffQ = kDecOffV + 2 * kDecTile;
+constexpr uint32_t kDecOffP = kDecOffQ + kDecQ;
+constexpr uint32_t kDecOffHdr = kDecOffP + 2 * kDecP;
+constexpr uint32_t kDecHdrBytes = 1024;
+constexpr size_t kDecSmem = 1024 + kDecOffHdr + kDecHdrBytes;
+static_assert(kDecSmem <= 227 * 1024, "shared memory");
+// kind::f16: bf16 A and B, fp32 D, M = 128, N = 16; A and B K-major
+constexpr uint32_t kDecIdescQK = (1u << 4) | (1u << 7) | (1u << 10) |
+                                 ((uint32_t)(kDecN >> 3) << 17) | ((uint32_t)(kDecPos >> 4) << 24);
+// the same with A MN-major (bit 15): O^T += V^T P^T with V as stored
+constexpr uint32_t kDecIdescPV = kDecIdescQK | (1u << 15);
+constexpr uint32_t kDecTmemCols = 64;
+constexpr uint32_t kDecColS = 0, kDecColO = 2 * kDecN;
+// base-2 distance the tile maximum may run ahead of a head's exponent base
+constexpr float kDecRescale = 8.f;
+
+struct DecHeader {
+    uint64_t q_full;
+    uint64_t k_full[2], k_empty[2];  // key tile j in stage j % 2
+    uint64_t v_full[2], v_empty[2];  // value tile j in stage j % 2
+    uint64_t s_full[2];              // S_j written (buffer j % 2)
+    uint64_t s_empty[2];             // S_j read by the four softmax warps
+    uint64_t p_ready[2];             // P_j written (four softmax warps)
+    uint64_t p_empty[2];             // P_j V_j finished
+    uint64_t done;
+    uint32_t tmem_base;
+    float red[2][4][kDecMaxG];  // the warps' tile maxima, by tile parity
+    float lsum[4][kDecMaxG];    // the warps' row sums at the end
+};
+static_assert(sizeof(DecHeader) <= kDecHdrBytes, "decode attention header");
+
+__device__ __forceinline__ bool dec_wait(uint64_t *bar, uint32_t parity, unsigned *err) {
+    return ptx::mbar_try_wait(bar, parity) || ptx::mbar_wait_hint(bar, parity, err);
+}
+
+__device__ __forceinline__ float dec_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// 16 fp32 columns of this warp's 32 tensor-memory lanes.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15]))
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// MN-major operand written by TMA with the 128-byte swizzle (the value tile
+// as A = V^T): a 128-byte row holds 64 consecutive dims of one position, 8
+// positions make a 1024-byte atom (stride offset), the next 64 dims are the
+// second box, 16 KB on (leading offset).
+__device__ __forceinline__ uint64_t dec_desc_mn(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)(kDecHalf >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// S^T = K Q^T: 128 positions x 16 heads over 128 dims.
+__device__ __forceinline__ void dec_issue_qk(uint32_t d_tmem, uint32_t k_smem, uint32_t q_smem) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        const uint64_t ad = smem_desc(k_smem + half * kDecHalf);
+        const uint64_t bd = smem_desc(q_smem + half * kDecNHalf);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+            mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, kDecIdescQK, (half | kk) != 0 ? 1u : 0u);
+    }
+}
+
+// O^T (+)= V^T P^T: 128 dims x 16 heads over 128 positions, 16 a step.
+__device__ __forceinline__ void dec_issue_pv(uint32_t d_tmem, uint32_t v_smem, uint32_t p_smem,
+                                             bool accumulate) {
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+        const uint64_t ad = dec_desc_mn(v_smem + ks * 16 * 128);
+        const uint64_t bd = smem_desc(p_smem + (ks >> 2) * kDecNHalf) + 2 * (ks & 3);
+        mma_bf16(d_tmem, ad, bd, kDecIdescPV, (accumulate || ks != 0) ? 1u : 0u);
+    }
+}
+
+template <int G>
+__global__ void __launch_bounds__(kDecThreads, 1)
+k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, int Hq, int Hkv, int n_seq, int L,
+                 int n_split, const int32_t *__restrict__ seq, const int32_t *__restrict__ pos,
+                 float *__restrict__ part_ml, float *__restrict__ part_acc,
+                 bf16 *__restrict__ ctx, unsigned *err) {
+    static_assert(G >= 1 && G <= kDecMaxG, "query heads per key/value head");
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    DecHeader *hd = reinterpret_cast<DecHeader *>(smem + kDecOffHdr);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int s = blockIdx.x, tg = blockIdx.y;
+    const int t = tg / Hkv, g = tg - t * Hkv;
+
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(&hd->q_full, 1);
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(&hd->k_full[b], 1);
+            ptx::mbar_init(&hd->k_empty[b], 1);
+            ptx::mbar_init(&hd->v_full[b], 1);
+            ptx::mbar_init(&hd->v_empty[b], 1);
+            ptx::mbar_init(&hd->s_full[b], 1);
+            ptx::mbar_init(&hd->s_empty[b], 4);
+            ptx::mbar_init(&hd->p_ready[b], 4);
+            ptx::mbar_init(&hd->p_empty[b], 1);
+        }
+        ptx::mbar_init(&hd->done, 1);
+        ptx::fence_barrier_init();
+        ptx::prefetch_tmap(&tmQ);
+        ptx::prefetch_tmap(&tmK);
+        ptx::prefetch_tmap(&tmV);
+    }
+    if (warp == 1) tmem_alloc(&hd->tmem_base, kDecTmemCols);
+    if (warp >= 2) {
+        // probability rows G..15 stay zero (the MMA's padding heads)
+        uint4 *pz = reinterpret_cast<uint4 *>(smem + kDecOffP);
+        for (int i = threadIdx.x - 64; i < (int)(2 * kDecP / 16); i += 128)
+            pz[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    ptx::grid_dependency_wait();  // queries and caches come from the previous kernel
+    const int sq = seq[t], p = pos[t];
+    const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
+    const int n = ok ? p + 1 : 0;
+    // the split's positions: a multiple of the tile, so only the last tile
+    // of the sequence is partial
+    const int per = ((n + n_split - 1) / n_split + kDecPos - 1) / kDecPos * kDecPos;
+    const int j0 = min(n, s * per), j1 = min(n, j0 + per);
+    const int n_tiles = (j1 - j0 + kDecPos - 1) / kDecPos;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = hd->tmem_base;
+    const uint32_t sbase = ptx::smem_u32(smem);
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0 && n_tiles > 0) {
+            const uint64_t pol_kv = ptx::policy_evict_first();  // read once
+            const uint64_t pol_q = ptx::policy_evict_normal();
+            const int qrow = t * Hq + g * G;
+            const int row0 = (sq * Hkv + g) * L + j0;
+            ptx::mbar_arrive_expect_tx(&hd->q_full, kDecQ);
+            for (int half = 0; half < 2; ++half)
+                ptx::tma_load_2d(smem + kDecOffQ + half * kDecNHalf, &tmQ, half * 64, qrow,
+                                 &hd->q_full, pol_q);
+            int k_issued = 0, v_issued = 0;
+            for (int j = 0; j < n_tiles; ++j) {
+                const int b = j & 1;
+                const uint32_t ph = ((j >> 1) & 1) ^ 1;
+                if (!dec_wait(&hd->k_empty[b], ph, err)) break;
+                ptx::mbar_arrive_expect_tx(&hd->k_full[b], kDecTile);
+                for (int half = 0; half < 2; ++half)
+                    ptx::tma_load_2d(smem + kDecOffK + b * kDecTile + half * kDecHalf, &tmK,
+                                     half * 64, row0 + j * kDecPos, &hd->k_full[b], pol_kv);
+                k_issued = j + 1;
+                if (!dec_wait(&hd->v_empty[b], ph, err)) break;
+                ptx::mbar_arrive_expect_tx(&hd->v_full[b], kDecTile);
+                for (int half = 0; half < 2; ++half)
+                    ptx::tma_load_2d(smem + kDecOffV + b * kDecTile + half * kDecHalf, &tmV,
+                                     half * 64, row0 + j * kDecPos, &hd->v_full[b], pol_kv);
+                v_issued = j + 1;
+            }
+            // copies still in flight land before the block can exit
+            dec_wait(&hd->q_full, 0, err);
+            for (int j = (k_issued > 2 ? k_issued - 2 : 0); j < k_issued; ++j)
+                dec_wait(&hd->k_full[j & 1], (j >> 1) & 1, err);
+            for (int j = (v_issued > 2 ? v_issued - 2 : 0); j < v_issued; ++j)
+                dec_wait(&hd->v_full[j & 1], (j >> 1) & 1, err);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && n_tiles > 0) {
+            bool good = dec_wait(&hd->q_full, 0, err) && dec_wait(&hd->k_full[0], 0, err);
+            if (good) {
+                tc_fence_after();
+                dec_issue_qk(tmem + kDecColS, sbase + kDecOffK, sbase + kDecOffQ);
+                mma_commit(&hd->s_full[0]);
+                mma_commit(&hd->k_empty[0]);
+            }
+            for (int j = 0; j < n_tiles && good; ++j) {
+                if (j + 1 < n_tiles) {
+                    // S_{j+1} into the buffer of S_{j-1}, once the softmax has read it
+                    const int b1 = (j + 1) & 1;
+                    good = dec_wait(&hd->k_full[b1], ((j + 1) >> 1) & 1, err) &&
+                           (j < 1 || dec_wait(&hd->s_empty[b1], ((j - 1) >> 1) & 1, err));
+                    if (!good) break;
+                    tc_fence_after();
+                    dec_issue_qk(tmem + kDecColS + b1 * kDecN, sbase + kDecOffK + b1 * kDecTile,
+                                 sbase + kDecOffQ);
+                    mma_commit(&hd->s_full[b1]);
+                    mma_commit(&hd->k_empty[b1]);
+                }
+                const int b = j & 1;
+                good = dec_wait(&hd->v_full[b], (j >> 1) & 1, err) &&
+                       dec_wait(&hd->p_ready[b], (j >> 1) & 1, err);
+                if (!good) break;
+                tc_fence_after();
+                dec_issue_pv(tmem + kDecColO, sbase + kDecOffV + b * kDecTile,
+                             sbase + kDecOffP + b * kDecP, j != 0);
+                mma_commit(&hd->p_empty[b]);
+                mma_commit(&hd->v_empty[b]);
+            }
+            mma_commit(&hd->done);
+            dec_wait(&hd->done, 0, err);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ softmax
+        const int qd = warp & 3;       // tensor-memory lane quarter
+        const int r = qd * 32 + lane;  // position of the tile; dim of O^T
+        const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+        const float sl2 = 1.4426950408889634f / sqrtf(128.f);
+        float base[G], l[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            base[h] = -INFINITY;
+            l[h] = 0.f;
+        }
+        bool good = true;
+        for (int j = 0; j < n_tiles; ++j) {
+            const int b = j & 1;
+            const int pj = j0 + j * kDecPos + r;
+            const bool valid = pj < j1;
+            // (the load runs on every lane whatever its waits returned: it is
+            // warp-collective; after a failed wait the values are not used)
+            float v[16];
+            good = good && dec_wait(&hd->s_full[b], (j >> 1) & 1, err);
+            tc_fence_after();
+            tmem_ld16(tmem + lane_base + kDecColS + b * kDecN, v);
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&hd->s_empty[b]);
+            // the tile maximum of every head (finite: the tile has a valid position)
+            float x[G];
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                x[h] = valid ? v[h] * sl2 : -INFINITY;
+                float m = x[h];
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+                if (lane == 0) hd->red[b][qd][h] = m;
+            }
+            ptx::named_bar_sync(1, 128);
+            float corr[G];
+            bool bump_any = false;
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float tm = fmaxf(fmaxf(hd->red[b][0][h], hd->red[b][1][h]),
+                                       fmaxf(hd->red[b][2][h], hd->red[b][3][h]));
+                const bool bump = tm > base[h] + kDecRescale;
+                corr[h] = bump ? exp2f(base[h] - tm) : 1.f;  // 0 on the first tile
+                if (bump) base[h] = tm;
+                bump_any |= bump;
+            }
+            // P_j into buffer b, free once P_{j-2} V_{j-2} has finished
+            good = good && (j < 2 || dec_wait(&hd->p_empty[b], ((j - 2) >> 1) & 1, err));
+            unsigned char *pb = smem + kDecOffP + b * kDecP + (r >> 6) * kDecNHalf;
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float pv = valid ? dec_exp2(x[h] - base[h]) : 0.f;
+                const bf16 pq = __float2bfloat16_rn(pv);
+                if (good)
+                    *reinterpret_cast<bf16 *>(pb + swizzle_offset((uint32_t)h, (uint32_t)(r & 63))) =
+                        pq;
+                l[h] = fmaf(l[h], corr[h], __bfloat162float(pq));
+            }
+            // a value tile that runs past the split's last position: its rows
+            // there are zeroed before P_j V_j reads them
+            if (j0 + j * kDecPos + kDecPos > j1) {
+                good = good && dec_wait(&hd->v_full[b], (j >> 1) & 1, err);
+                if (good && !valid) {
+                    unsigned char *vt = smem + kDecOffV + b * kDecTile;
+#pragma unroll
+                    for (int c = 0; c < 128; c += 8)
+                        *reinterpret_cast<uint4 *>(vt + (c >> 6) * kDecHalf +
+                                                   swizzle_offset((uint32_t)r, (uint32_t)(c & 63))) =
+                            make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
+            // a moved base rescales O^T (each thread its dim's row) once
+            // P_{j-1} V_{j-1} has finished; P_j V_j waits for this warp
+            if (j >= 1 && bump_any) {
+                good = good && dec_wait(&hd->p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, err);
+                if (__all_sync(0xffffffffu, good)) {
+                    tc_fence_after();
+                    float o[16];
+                    tmem_ld16(tmem + lane_base + kDecColO, o);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int h = 0; h < G; ++h) o[h] *= corr[h];
+                    tmem_st16(tmem + lane_base + kDecColO, o);
+                }
+            }
+            fence_proxy_async_smem();  // P_j and the zeroed value rows
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&hd->p_ready[b]);
+        }
+        // the split's result: O^T row r (dim r) of every head, the row sums
+        // of the four warps added in warp order
+        bool fin = good && n_tiles > 0;
+        if (fin) fin = dec_wait(&hd->p_empty[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1, err);
+        fin = __all_sync(0xffffffffu, fin);
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            const float ws = warp_sum(l[h]);
+            if (lane == 0) hd->lsum[qd][h] = ws;
+        }
+        ptx::named_bar_sync(1, 128);
+        float o[16];
+#pragma unroll
+        for (int h = 0; h < 16; ++h) o[h] = 0.f;
+        if (fin) {
+            tc_fence_after();
+            tmem_ld16(tmem + lane_base + kDecColO, o);
+            tmem_ld_wait();
+        }
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            const float Ls =
+                fin ? (hd->lsum[0][h] + hd->lsum[1][h]) + (hd->lsum[2][h] + hd->lsum[3][h]) : 0.f;
+            const int head = g * G + h;
+            if (n_split == 1) {
+                ctx[((size_t)t * Hq + head) * 128 + r] =
+                    __float2bfloat16_rn(Ls > 0.f ? o[h] / Ls : 0.f);
+            } else {
+                const size_t oi = ((size_t)t * Hq + head) * n_split + s;
+                if (r == 0) {
+                    // (maximum, sum) in the natural-log form of the merge
+                    part_ml[2 * oi] = fin ? base[h] * 0.6931471805599453f : -INFINITY;
+                    part_ml[2 * oi + 1] = Ls;
+                }
+                part_acc[oi * 128 + r] = fin ? o[h] : 0.f;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, kDecTmemCols);
+}
+
+}  // namespace
+
+bool attn_decode_tc_ok() { return encode_fn() != nullptr; }
+
+int attn_decode_tc_splits(int T, int Hkv, int max_len, int split_cap) {
+    // one wave of one-CTA-per-SM blocks, at least one position tile a split
+    const int tg = std::max(1, T * Hkv);
+    int ns = std::max(1, device_info().sm_count / tg);
+    ns = std::min(ns, (max_len + kDecPos - 1) / kDecPos);
+    return std::max(1, std::min(ns, split_cap));
+}
+
+cudaError_t launch_attn_decode_tc(int T, int Hq, int Hkv, int n_seq, int L, int n_split,
+                                  const int32_t *seq, const int32_t *pos, const void *q16,
+                                  const void *k_cache, const void *v_cache, float *part_ml,
+                                  float *part_acc, void *ctx, cudaStream_t st) {
+    const int G = Hq / Hkv;
+    if (G < 1 || G > kDecMaxG || G * Hkv != Hq || n_split < 1) return cudaErrorInvalidValue;
+    CUtensorMap mq, mk, mv;
+    const uint64_t rows = (uint64_t)n_seq * Hkv * L;
+    if (!make_map(&mq, q16, (uint64_t)T * Hq, 128, kDecN) ||
+        !make_map(&mk, k_cache, rows, 128, kDecPos) || !make_map(&mv, v_cache, rows, 128, kDecPos))
+        return cudaErrorInvalidValue;
+    const void *kern = nullptr;
+    switch (G) {
+        case 1: kern = (const void *)k_attn_decode_tc<1>; break;
+        case 2: kern = (const void *)k_attn_decode_tc<2>; break;
+        case 3: kern = (const void *)k_attn_decode_tc<3>; break;
+        case 4: kern = (const void *)k_attn_decode_tc<4>; break;
+        case 5: kern = (const void *)k_attn_decode_tc<5>; break;
+        case 6: kern = (const void *)k_attn_decode_tc<6>; break;
+        case 7: kern = (const void *)k_attn_decode_tc<7>; break;
+        default: kern = (const void *)k_attn_decode_tc<8>; break;
+    }
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecSmem);
+    if (e != cudaSuccess) return e;
+    unsigned *err = device_info().err;
+    bf16 *cp = static_cast<bf16 *>(ctx);
+    int Hqv = Hq, Hkvv = Hkv, ns = n_seq, Lv = L, nsp = n_split;
+    void *args[] = {&mq, &mk, &mv, &Hqv, &Hkvv, &ns, &Lv, &nsp, &seq, &pos,
+                    &part_ml, &part_acc, &cp, &err};
+    LaunchScope ls("attention_decode_tc", st);
+    return launch_pdl(kern, dim3(n_split, T * Hkv), dim3(kDecThreads), kDecSmem, st, args);
+}
+
+}  // namespace moe

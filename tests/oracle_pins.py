@@ -592,6 +592,43 @@ def pin_sa_bf16_storage(orc):
         assert np.array_equal(gen.to_f64(gen.store(c, "bf16"), "bf16"), c), "cache not bf16"
 
 
+def pin_sa_bf16_block_composition(orc):
+    """With bf16 storage the block is the composition of pin_sa_block_-
+    composition with every stored activation rounded to bf16 by numpy's bit
+    rounding (independent of the oracle's): the normalised input, the rotated
+    queries and keys, the values, and ctx."""
+    from scipy.linalg import expm
+
+    def r16(a):
+        return gen.to_f64(gen.store(a, "bf16"), "bf16")
+
+    rng = np.random.default_rng(71)
+    D, Hq, Hkv, dh, base, eps = 24, 4, 2, 8, 1000.0, 1e-6
+    w_qkv, w_o, kc, vc = _sa_case(rng, D, Hq, Hkv, dh, dt="bf16")
+    n = 5
+    x = rng.normal(size=(n, D)) * 3.0
+    seq = np.array([0, 0, 1, 1, 1], np.int32)
+    pos = np.array([3, 4, 0, 1, 2], np.int32)
+    got, _, _ = orc.sa_forward(x, w_qkv, w_o, "bf16", Hq, Hkv, base, eps, seq, pos, kc, vc)
+    xn = r16(x / np.sqrt(np.mean(x * x, axis=1, keepdims=True) + eps))
+    qkv = xn @ gen.to_f64(w_qkv, "bf16").T
+    q = qkv[:, :Hq * dh].reshape(n, Hq, dh)
+    k = qkv[:, Hq * dh:(Hq + Hkv) * dh].reshape(n, Hkv, dh)
+    v = r16(qkv[:, (Hq + Hkv) * dh:].reshape(n, Hkv, dh))
+    G = _rope_generator(dh, base)
+    R = [expm(p * G) for p in pos]
+    q = r16(np.stack([q[t] @ R[t].T for t in range(n)]))
+    k = r16(np.stack([k[t] @ R[t].T for t in range(n)]))
+    wk, wv = kc.copy(), vc.copy()
+    for t in range(n):
+        wk[seq[t], :, pos[t]] = k[t]
+        wv[seq[t], :, pos[t]] = v[t]
+    ctx = r16(np.stack([_sdpa(q[t][:, None, :], wk[seq[t], :, :pos[t] + 1],
+                              wv[seq[t], :, :pos[t] + 1], False)[:, 0, :] for t in range(n)]))
+    want = x + ctx.reshape(n, Hq * dh) @ gen.to_f64(w_o, "bf16").T
+    _close(got, want, 1e-9, 1e-11, "self-attention block, bf16 storage")
+
+
 def pin_decoder_layer_composition(orc):
     """A decoder layer whose output projection is zero is the MoE stack
     layer alone (pinned above); with it, the layer is the self-attention

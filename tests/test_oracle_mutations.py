@@ -60,6 +60,7 @@ MUTATIONS = [
     ("values_from_keys", "qkv + (size_t)t * nr + nq + nkv, sizeof(double) * nkv);",
      "qkv + (size_t)t * nr + nq, sizeof(double) * nkv);"),
     ("cache_not_rounded", "        orc_round_bf16((size_t)T * nkv, v, v);\n", "\n"),
+    ("queries_not_rounded", "        orc_round_bf16((size_t)T * nq, q, q);\n", "\n"),
 ]
 
 
