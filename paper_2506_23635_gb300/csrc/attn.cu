@@ -160,6 +160,10 @@ k_rope_cache(int T, int Hq, int Hkv, int n_seq, int L, RopeRates rates,
              const float *__restrict__ qkv, int n_part, long long part_stride,
              float *__restrict__ q, bf16 *__restrict__ q16, bf16 *__restrict__ kc,
              bf16 *__restrict__ vc, unsigned *err) {
+    // a decode-type call (no 128-token prefill tile): the tensor-core decode
+    // attention, one CTA per SM on the SMs this small grid leaves free, may
+    // launch now and set itself up while this kernel runs
+    if (T < kAttnTcTile) ptx::launch_dependents();
     ptx::grid_dependency_wait();
     constexpr int H2 = kHeadDim / 2;
     static_assert(kRopeTokens * H2 <= kRopeRows * H2, "one thread per (token, pair)");
@@ -270,153 +274,168 @@ __device__ __forceinline__ void unpack4(uint2 u, float (&o)[4]) {
 // (relative to m).
 template <int G>
 __global__ void __launch_bounds__(kAttnThreads)
-k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, const int32_t *__restrict__ seq,
-               const int32_t *__restrict__ pos, const float *__restrict__ q,
-               const bf16 *__restrict__ kc, const bf16 *__restrict__ vc,
-               float *__restrict__ part_ml, float *__restrict__ part_acc,
-               bf16 *__restrict__ ctx, const int *__restrict__ tile_ok) {
+k_attn_partial(int Hq, int Hkv, int n_seq, int L, int n_split, int n_tg,
+               const int32_t *__restrict__ seq, const int32_t *__restrict__ pos,
+               const float *__restrict__ q, const bf16 *__restrict__ kc,
+               const bf16 *__restrict__ vc, float *__restrict__ part_ml,
+               float *__restrict__ part_acc, bf16 *__restrict__ ctx,
+               const int *__restrict__ tile_ok) {
     ptx::grid_dependency_wait();
     __shared__ __align__(16) float qs[G][kHeadDim];
     __shared__ float sm_m[kAttnWarps][G], sm_l[kAttnWarps][G];
     __shared__ float sm_acc[kAttnWarps][G][kHeadDim];
     __shared__ __align__(16) bf16 vtile[kAttnWarps][32][kHeadDim];  // each warp's value tile
-    const int s = blockIdx.x, tg = blockIdx.y;
-    const int t = tg / Hkv, g = tg - t * Hkv;
-    if (tile_ok && tile_ok[t / kAttnTcTile]) return;  // the tensor-core kernel has it
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int sq = seq[t], p = pos[t];
-    const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
-    const int n = ok ? p + 1 : 0;
-    const int chunk = (n + n_split - 1) / n_split;
-    const int j0 = min(n, s * chunk), j1 = min(n, j0 + chunk);
-    const float scale = 1.0f / sqrtf((float)kHeadDim);
-    // the queries as stored activations: rounded to bf16, as the tensor-core
-    // kernels read them
-    for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x)
-        qs[i / kHeadDim][i % kHeadDim] =
-            __bfloat162float(__float2bfloat16_rn(q[((size_t)t * Hq + g * G) * kHeadDim + i])) *
-            scale;
-    __syncthreads();
-
-    float m[G], l[G], acc[G][4];
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-        m[h] = -INFINITY;
-        l[h] = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc[h][i] = 0.f;
+    __shared__ unsigned char s_ok[kMaxSaTokens / kAttnTcTile];
+    const int s = blockIdx.x;
+    // (token, key/value head) items blockIdx.y, + gridDim.y, ...: a call
+    // whose prefill tiles went to the tensor cores launches a bounded grid
+    // that skips them (their flags read once into shared memory), instead
+    // of a block per item
+    if (tile_ok) {
+        const int n_tiles = (n_tg / Hkv + kAttnTcTile - 1) / kAttnTcTile;
+        for (int i = threadIdx.x; i < n_tiles; i += blockDim.x) s_ok[i] = tile_ok[i] ? 1 : 0;
+        __syncthreads();
     }
-    const size_t base = ok ? ((size_t)sq * Hkv + g) * L * kHeadDim : 0;
-    const bf16 *kb = kc + base;
-    const bf16 *vb = vc + base;
-    for (int jt = j0 + warp * 32; jt < j1; jt += kAttnWarps * 32) {
-        const int jl = jt + lane;  // this lane's position
-        const bool live = jl < j1;
-        const int nt = min(32, j1 - jt);
-        // the tile's value rows land in shared memory while the scores are
-        // computed: lane l copies bytes [8l, 8l+8) of every row
-        __syncwarp();
-        for (int u = 0; u < nt; ++u)
-            cp_async8(&vtile[warp][u][lane * 4], vb + (size_t)(jt + u) * kHeadDim + lane * 4);
-        cp_async_commit();
-        float sc[G];
+    for (int tg = blockIdx.y; tg < n_tg; tg += gridDim.y) {
+        const int t = tg / Hkv, g = tg - t * Hkv;
+        if (tile_ok && s_ok[t / kAttnTcTile]) continue;  // the tensor-core kernel has it
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        const int sq = seq[t], p = pos[t];
+        const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
+        const int n = ok ? p + 1 : 0;
+        const int chunk = (n + n_split - 1) / n_split;
+        const int j0 = min(n, s * chunk), j1 = min(n, j0 + chunk);
+        const float scale = 1.0f / sqrtf((float)kHeadDim);
+        // the queries as stored activations: rounded to bf16, as the
+        // tensor-core kernels read them
+        for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x)
+            qs[i / kHeadDim][i % kHeadDim] =
+                __bfloat162float(
+                    __float2bfloat16_rn(q[((size_t)t * Hq + g * G) * kHeadDim + i])) *
+                scale;
+        __syncthreads();
+
+        float m[G], l[G], acc[G][4];
 #pragma unroll
-        for (int h = 0; h < G; ++h) sc[h] = 0.f;
-        if (live) {
-            const uint4 *kr = reinterpret_cast<const uint4 *>(kb + (size_t)jl * kHeadDim);
+        for (int h = 0; h < G; ++h) {
+            m[h] = -INFINITY;
+            l[h] = 0.f;
 #pragma unroll
-            for (int c = 0; c < kHeadDim / 32; ++c) {  // 32 dims per step
-                uint4 u[4];
+            for (int i = 0; i < 4; ++i) acc[h][i] = 0.f;
+        }
+        const size_t base = ok ? ((size_t)sq * Hkv + g) * L * kHeadDim : 0;
+        const bf16 *kb = kc + base;
+        const bf16 *vb = vc + base;
+        for (int jt = j0 + warp * 32; jt < j1; jt += kAttnWarps * 32) {
+            const int jl = jt + lane;  // this lane's position
+            const bool live = jl < j1;
+            const int nt = min(32, j1 - jt);
+            // the tile's value rows land in shared memory while the scores are
+            // computed: lane l copies bytes [8l, 8l+8) of every row
+            __syncwarp();
+            for (int u = 0; u < nt; ++u)
+                cp_async8(&vtile[warp][u][lane * 4], vb + (size_t)(jt + u) * kHeadDim + lane * 4);
+            cp_async_commit();
+            float sc[G];
 #pragma unroll
-                for (int v = 0; v < 4; ++v) u[v] = __ldg(kr + c * 4 + v);
+            for (int h = 0; h < G; ++h) sc[h] = 0.f;
+            if (live) {
+                const uint4 *kr = reinterpret_cast<const uint4 *>(kb + (size_t)jl * kHeadDim);
 #pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    float k8[8];
-                    unpack_bf16x2(u[v].x, k8[0], k8[1]);
-                    unpack_bf16x2(u[v].y, k8[2], k8[3]);
-                    unpack_bf16x2(u[v].z, k8[4], k8[5]);
-                    unpack_bf16x2(u[v].w, k8[6], k8[7]);
-                    const int d0 = c * 32 + v * 8;
+                for (int c = 0; c < kHeadDim / 32; ++c) {  // 32 dims per step
+                    uint4 u[4];
 #pragma unroll
-                    for (int h = 0; h < G; ++h) {
-                        const float4 qa = *reinterpret_cast<const float4 *>(&qs[h][d0]);
-                        const float4 qb = *reinterpret_cast<const float4 *>(&qs[h][d0 + 4]);
-                        sc[h] = fmaf(qa.x, k8[0], sc[h]);
-                        sc[h] = fmaf(qa.y, k8[1], sc[h]);
-                        sc[h] = fmaf(qa.z, k8[2], sc[h]);
-                        sc[h] = fmaf(qa.w, k8[3], sc[h]);
-                        sc[h] = fmaf(qb.x, k8[4], sc[h]);
-                        sc[h] = fmaf(qb.y, k8[5], sc[h]);
-                        sc[h] = fmaf(qb.z, k8[6], sc[h]);
-                        sc[h] = fmaf(qb.w, k8[7], sc[h]);
+                    for (int v = 0; v < 4; ++v) u[v] = __ldg(kr + c * 4 + v);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        float k8[8];
+                        unpack_bf16x2(u[v].x, k8[0], k8[1]);
+                        unpack_bf16x2(u[v].y, k8[2], k8[3]);
+                        unpack_bf16x2(u[v].z, k8[4], k8[5]);
+                        unpack_bf16x2(u[v].w, k8[6], k8[7]);
+                        const int d0 = c * 32 + v * 8;
+#pragma unroll
+                        for (int h = 0; h < G; ++h) {
+                            const float4 qa = *reinterpret_cast<const float4 *>(&qs[h][d0]);
+                            const float4 qb = *reinterpret_cast<const float4 *>(&qs[h][d0 + 4]);
+                            sc[h] = fmaf(qa.x, k8[0], sc[h]);
+                            sc[h] = fmaf(qa.y, k8[1], sc[h]);
+                            sc[h] = fmaf(qa.z, k8[2], sc[h]);
+                            sc[h] = fmaf(qa.w, k8[3], sc[h]);
+                            sc[h] = fmaf(qb.x, k8[4], sc[h]);
+                            sc[h] = fmaf(qb.y, k8[5], sc[h]);
+                            sc[h] = fmaf(qb.z, k8[6], sc[h]);
+                            sc[h] = fmaf(qb.w, k8[7], sc[h]);
+                        }
                     }
                 }
             }
-        }
-        float w[G];
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            float tm = live ? sc[h] : -INFINITY;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, o));
-            const float mn = fmaxf(m[h], tm);  // finite: the tile has a live lane
-            const float corr = expf(m[h] - mn);  // 0 while m is -inf
-            w[h] = live ? expf(sc[h] - mn) : 0.f;
-            l[h] = l[h] * corr + warp_sum(w[h]);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) acc[h][i] *= corr;
-            m[h] = mn;
-        }
-        cp_async_wait_all();
-        __syncwarp();
-#pragma unroll 4
-        for (int u = 0; u < nt; ++u) {
-            float v4[4];
-            unpack4(*reinterpret_cast<const uint2 *>(&vtile[warp][u][lane * 4]), v4);
+            float w[G];
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                const float wu = __shfl_sync(0xffffffffu, w[h], u);
+                float tm = live ? sc[h] : -INFINITY;
 #pragma unroll
-                for (int i = 0; i < 4; ++i) acc[h][i] = fmaf(wu, v4[i], acc[h][i]);
+                for (int o = 16; o > 0; o >>= 1)
+                    tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, o));
+                const float mn = fmaxf(m[h], tm);  // finite: the tile has a live lane
+                const float corr = expf(m[h] - mn);  // 0 while m is -inf
+                w[h] = live ? expf(sc[h] - mn) : 0.f;
+                l[h] = l[h] * corr + warp_sum(w[h]);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[h][i] *= corr;
+                m[h] = mn;
+            }
+            cp_async_wait_all();
+            __syncwarp();
+#pragma unroll 4
+            for (int u = 0; u < nt; ++u) {
+                float v4[4];
+                unpack4(*reinterpret_cast<const uint2 *>(&vtile[warp][u][lane * 4]), v4);
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float wu = __shfl_sync(0xffffffffu, w[h], u);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) acc[h][i] = fmaf(wu, v4[i], acc[h][i]);
+                }
             }
         }
-    }
 #pragma unroll
-    for (int h = 0; h < G; ++h) {
-        if (lane == 0) {
-            sm_m[warp][h] = m[h];
-            sm_l[warp][h] = l[h];
+        for (int h = 0; h < G; ++h) {
+            if (lane == 0) {
+                sm_m[warp][h] = m[h];
+                sm_l[warp][h] = l[h];
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) sm_acc[warp][h][lane * 4 + i] = acc[h][i];
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) sm_acc[warp][h][lane * 4 + i] = acc[h][i];
-    }
-    __syncthreads();
-    const int d = threadIdx.x;
+        __syncthreads();
+        const int d = threadIdx.x;
 #pragma unroll 1
-    for (int h = 0; h < G; ++h) {
-        float M = -INFINITY;
+        for (int h = 0; h < G; ++h) {
+            float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < kAttnWarps; ++w) M = fmaxf(M, sm_m[w][h]);
-        float Ls = 0.f, A = 0.f;
-        if (M != -INFINITY) {
+            for (int w = 0; w < kAttnWarps; ++w) M = fmaxf(M, sm_m[w][h]);
+            float Ls = 0.f, A = 0.f;
+            if (M != -INFINITY) {
 #pragma unroll
-            for (int w = 0; w < kAttnWarps; ++w) {
-                const float c = expf(sm_m[w][h] - M);
-                Ls = fmaf(sm_l[w][h], c, Ls);
-                A = fmaf(sm_acc[w][h][d], c, A);
+                for (int w = 0; w < kAttnWarps; ++w) {
+                    const float c = expf(sm_m[w][h] - M);
+                    Ls = fmaf(sm_l[w][h], c, Ls);
+                    A = fmaf(sm_acc[w][h][d], c, A);
+                }
             }
+            if (n_split == 1) {  // the only split: this is the result
+                ctx[((size_t)t * Hq + g * G + h) * kHeadDim + d] =
+                    __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
+                continue;
+            }
+            const size_t o = ((size_t)t * Hq + g * G + h) * n_split + s;
+            if (d == 0) {
+                part_ml[2 * o] = M;
+                part_ml[2 * o + 1] = Ls;
+            }
+            part_acc[o * kHeadDim + d] = A;
         }
-        if (n_split == 1) {  // the only split: this is the result
-            ctx[((size_t)t * Hq + g * G + h) * kHeadDim + d] =
-                __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
-            continue;
-        }
-        const size_t o = ((size_t)t * Hq + g * G + h) * n_split + s;
-        if (d == 0) {
-            part_ml[2 * o] = M;
-            part_ml[2 * o + 1] = Ls;
-        }
-        part_acc[o * kHeadDim + d] = A;
     }
 }
 
@@ -723,15 +742,9 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
         if (e != cudaSuccess) return e;
         ns = 1;
     } else if (q16 && decode_tc()) {
-        ns = attn_decode_tc_splits(c.T, Hkv, L, split_cap(c.T, Hkv));
-        cudaError_t e = launch_attn_decode_tc(c.T, Hq, Hkv, n_seq, L, ns, seq, pos, q16, kc, vc,
-                                              ml, acc, ctx, c.st);
-        if (e != cudaSuccess || ns == 1) return e;
-        const float *mlc = ml, *accc = acc;
-        void *args[] = {&ns, &mlc, &accc, &cp};
-        LaunchScope ls("attn_merge", c.st);
-        return launch_pdl((const void *)k_attn_merge, dim3(c.T * Hq),
-                          dim3(kHeadDim * kMergeGroups), 0, c.st, args);
+        // splits merged inside the kernel (a cluster per token and key/value head)
+        return launch_attn_decode_tc(c.T, Hq, Hkv, n_seq, L, attn_decode_tc_splits(c.T, Hkv, L),
+                                     seq, pos, q16, kc, vc, ctx, c.st);
     }
     const void *kern = nullptr;
     switch (G) {
@@ -748,10 +761,12 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     const bf16 *kcp = static_cast<const bf16 *>(kc), *vcp = static_cast<const bf16 *>(vc);
     {
         const int *tok = tile_ok;
-        void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &seq, &pos, &q, &kcp, &vcp, &ml, &acc, &cp,
-                        &tok};
+        int n_tg = c.T * Hkv;
+        const int gy = tile_ok ? std::min(n_tg, 8 * device_info().sm_count) : n_tg;
+        void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &n_tg, &seq, &pos, &q, &kcp, &vcp, &ml,
+                        &acc, &cp, &tok};
         LaunchScope ls("attention", c.st);
-        cudaError_t e = launch_pdl(kern, dim3(ns, c.T * Hkv), dim3(kAttnThreads), 0, c.st, args);
+        cudaError_t e = launch_pdl(kern, dim3(ns, gy), dim3(kAttnThreads), 0, c.st, args);
         if (e != cudaSuccess || ns == 1) return e;
     }
     const float *mlc = ml, *accc = acc;

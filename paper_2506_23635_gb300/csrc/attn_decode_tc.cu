@@ -16,7 +16,7 @@
 // the split's positions [j0, j1) of t's sequence in tiles of 128:
 //
 //   warp 0      TMA: the group's bf16 query rows once, then key and value
-//               tiles into two-stage rings (each 32 KB: two boxes of 64
+//               tiles into three-stage rings (each 32 KB: two boxes of 64
 //               dims with the 128-byte swizzle);
 //   warp 1      tensor memory (S^T twice, O^T: 48 of 64 columns) and the
 //               MMAs: S_{j+1} is issued as soon as its key tile has landed
@@ -35,15 +35,24 @@
 //               hold anything).
 //
 // The end: each thread owns dim r of O^T; per head the row sums of the four
-// warps are added, and the CTA writes either ctx (a single split) or the
-// split's (maximum, sum, weighted values) for k_attn_merge, in the form of
-// the CUDA-core kernel's partials.
+// warps are added.  A single split writes ctx.  Several splits of one
+// (token, key/value head) are the CTAs of one thread-block cluster (at most
+// 8), and CTA c owns the heads h = c, c + n_split, ...: every CTA stores its
+// (base, sum) and O^T row of each head straight into the owner's shared
+// memory (distributed shared memory stores need no round trip), then
+// arrives on the owner's merge barrier with release semantics; the owner
+// waits for all n_split arrivals, combines its heads and writes their ctx.
+// (The stores wait until every CTA of the cluster has initialised its
+// barriers: each arrives on the cluster barrier at its start and waits on it
+// before storing, by when the wait is long satisfied.)
 //
 // Numerics as the prefill flash attention: bf16 queries and probabilities,
 // fp32 scores and accumulation; the row sum takes the probabilities as
 // stored.  Every wait is bounded (ptx.cuh); once one gives up the thread
 // skips the later waits and the kernel ends.
 #include <math.h>
+
+#include <algorithm>
 
 #include "tc.cuh"
 
@@ -56,18 +65,25 @@ constexpr int kDecPos = 128;   // positions per key/value tile: the MMA's M
 constexpr int kDecN = 16;      // the MMA's N: the group's query heads, zero-padded
 constexpr int kDecMaxG = 8;    // query heads per key/value head
 constexpr int kDecThreads = 6 * 32;
+constexpr int kDecStages = 3;     // key and value tiles in flight
+constexpr int kDecMaxSplit = 8;   // splits of one (token, key/value head): a portable cluster
 constexpr uint32_t kDecHalf = kDecPos * 128;  // one 64-dim box of a key/value tile: 16 KB
 constexpr uint32_t kDecTile = 2 * kDecHalf;   // 32 KB
 constexpr uint32_t kDecNHalf = kDecN * 128;   // 16 rows x 64 elements: 2 KB
 constexpr uint32_t kDecQ = 2 * kDecNHalf;     // query rows, 128 dims
 constexpr uint32_t kDecP = 2 * kDecNHalf;     // probabilities, 128 positions
-// shared memory (1024-byte aligned): K[2], V[2], Q, P[2], header
+// shared memory (1024-byte aligned): K[3], V[3], Q, P[2], the O^T rows the
+// splits store for the heads this CTA merges, header
 constexpr uint32_t kDecOffK = 0;
-constexpr uint32_t kDecOffV = kDecOffK + 2 * kDecTile;
-constexpr uint32_t kDecOffQ = kDecOffV + 2 * kDecTile;
+constexpr uint32_t kDecOffV = kDecOffK + kDecStages * kDecTile;
+constexpr uint32_t kDecOffQ = kDecOffV + kDecStages * kDecTile;
 constexpr uint32_t kDecOffP = kDecOffQ + kDecQ;
-constexpr uint32_t kDecOffHdr = kDecOffP + 2 * kDecP;
-constexpr uint32_t kDecHdrBytes = 1024;
+constexpr uint32_t kDecOffX = kDecOffP + 2 * kDecP;
+// [heads this CTA owns <= ceil(8 / n_split)][n_split][128] floats: at most
+// 14 rows (8 heads over 7 splits)
+constexpr uint32_t kDecXBytes = 14 * 128 * 4;
+constexpr uint32_t kDecOffHdr = kDecOffX + kDecXBytes;
+constexpr uint32_t kDecHdrBytes = 2048;
 constexpr size_t kDecSmem = 1024 + kDecOffHdr + kDecHdrBytes;
 static_assert(kDecSmem <= 227 * 1024, "shared memory");
 // kind::f16: bf16 A and B, fp32 D, M = 128, N = 16; A and B K-major
@@ -82,21 +98,45 @@ constexpr float kDecRescale = 8.f;
 
 struct DecHeader {
     uint64_t q_full;
-    uint64_t k_full[2], k_empty[2];  // key tile j in stage j % 2
-    uint64_t v_full[2], v_empty[2];  // value tile j in stage j % 2
+    uint64_t k_full[kDecStages], k_empty[kDecStages];  // key tile j in stage j % 3
+    uint64_t v_full[kDecStages], v_empty[kDecStages];  // value tile j in stage j % 3
     uint64_t s_full[2];              // S_j written (buffer j % 2)
     uint64_t s_empty[2];             // S_j read by the four softmax warps
     uint64_t p_ready[2];             // P_j written (four softmax warps)
     uint64_t p_empty[2];             // P_j V_j finished
     uint64_t done;
+    uint64_t merge_full;             // every split's partials stored here (n_split arrivals)
     uint32_t tmem_base;
     float red[2][4][kDecMaxG];  // the warps' tile maxima, by tile parity
     float lsum[4][kDecMaxG];    // the warps' row sums at the end
+    float ml[kDecMaxG][kDecMaxSplit][2];  // (base, sum) of the owned heads, by split
 };
 static_assert(sizeof(DecHeader) <= kDecHdrBytes, "decode attention header");
 
+// Waits spin on the non-blocking test (bounded by the wall-time limit of
+// ptx.cuh): the pipeline is a chain of short steps, and a thread that
+// suspends in try_wait resumes later than the phase completes.
+__device__ __forceinline__ bool dec_test(uint64_t *bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(ptx::smem_u32(bar)), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
 __device__ __forceinline__ bool dec_wait(uint64_t *bar, uint32_t parity, unsigned *err) {
-    return ptx::mbar_try_wait(bar, parity) || ptx::mbar_wait_hint(bar, parity, err);
+    if (dec_test(bar, parity)) return true;
+    const uint64_t t0 = ptx::globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (dec_test(bar, parity)) return true;
+        if ((it & 255u) == 0 && ptx::globaltimer() - t0 > ptx::kWaitLimitNs) {
+            set_error(err, kErrTimeout);
+            return false;
+        }
+    }
 }
 
 __device__ __forceinline__ float dec_exp2(float x) {
@@ -132,6 +172,22 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) 
         "r"(__float_as_uint(v[15]))
         : "memory");
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Store a float into CTA `rank`'s shared memory (distributed shared memory
+// of the cluster), at the address this CTA's `p` has in its own.
+__device__ __forceinline__ void st_cluster_f32(float *p, uint32_t rank, float v) {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(
+                     ptx::map_rank(ptx::smem_u32(p), rank)),
+                 "f"(v)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
 }
 
 // MN-major operand written by TMA with the 128-byte swizzle (the value tile
@@ -171,7 +227,6 @@ __global__ void __launch_bounds__(kDecThreads, 1)
 k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                  const __grid_constant__ CUtensorMap tmV, int Hq, int Hkv, int n_seq, int L,
                  int n_split, const int32_t *__restrict__ seq, const int32_t *__restrict__ pos,
-                 float *__restrict__ part_ml, float *__restrict__ part_acc,
                  bf16 *__restrict__ ctx, unsigned *err) {
     static_assert(G >= 1 && G <= kDecMaxG, "query heads per key/value head");
     extern __shared__ unsigned char smem_raw[];
@@ -184,29 +239,42 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 
     if (threadIdx.x == 0) {
         ptx::mbar_init(&hd->q_full, 1);
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kDecStages; ++b) {
             ptx::mbar_init(&hd->k_full[b], 1);
             ptx::mbar_init(&hd->k_empty[b], 1);
             ptx::mbar_init(&hd->v_full[b], 1);
             ptx::mbar_init(&hd->v_empty[b], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(&hd->s_full[b], 1);
             ptx::mbar_init(&hd->s_empty[b], 4);
             ptx::mbar_init(&hd->p_ready[b], 4);
             ptx::mbar_init(&hd->p_empty[b], 1);
         }
         ptx::mbar_init(&hd->done, 1);
+        ptx::mbar_init(&hd->merge_full, n_split);
         ptx::fence_barrier_init();
         ptx::prefetch_tmap(&tmQ);
         ptx::prefetch_tmap(&tmK);
         ptx::prefetch_tmap(&tmV);
     }
     if (warp == 1) tmem_alloc(&hd->tmem_base, kDecTmemCols);
+    if (n_split > 1) {
+        // this CTA's barriers are initialised (thread 0, fenced at cluster
+        // scope): the cluster's other CTAs may store into it once they pass
+        // the matching wait
+        __syncthreads();
+        cluster_arrive_relaxed();
+    }
     if (warp >= 2) {
         // probability rows G..15 stay zero (the MMA's padding heads)
         uint4 *pz = reinterpret_cast<uint4 *>(smem + kDecOffP);
         for (int i = threadIdx.x - 64; i < (int)(2 * kDecP / 16); i += 128)
             pz[i] = make_uint4(0u, 0u, 0u, 0u);
     }
+    // the output projection may launch now: it streams its weights into the
+    // SMs this grid leaves free while the attention runs
+    ptx::launch_dependents();
     ptx::grid_dependency_wait();  // queries and caches come from the previous kernel
     const int sq = seq[t], p = pos[t];
     const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
@@ -235,8 +303,8 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                                  &hd->q_full, pol_q);
             int k_issued = 0, v_issued = 0;
             for (int j = 0; j < n_tiles; ++j) {
-                const int b = j & 1;
-                const uint32_t ph = ((j >> 1) & 1) ^ 1;
+                const int b = j % kDecStages;
+                const uint32_t ph = ((j / kDecStages) & 1) ^ 1;
                 if (!dec_wait(&hd->k_empty[b], ph, err)) break;
                 ptx::mbar_arrive_expect_tx(&hd->k_full[b], kDecTile);
                 for (int half = 0; half < 2; ++half)
@@ -252,10 +320,10 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             }
             // copies still in flight land before the block can exit
             dec_wait(&hd->q_full, 0, err);
-            for (int j = (k_issued > 2 ? k_issued - 2 : 0); j < k_issued; ++j)
-                dec_wait(&hd->k_full[j & 1], (j >> 1) & 1, err);
-            for (int j = (v_issued > 2 ? v_issued - 2 : 0); j < v_issued; ++j)
-                dec_wait(&hd->v_full[j & 1], (j >> 1) & 1, err);
+            for (int j = std::max(0, k_issued - kDecStages); j < k_issued; ++j)
+                dec_wait(&hd->k_full[j % kDecStages], (j / kDecStages) & 1, err);
+            for (int j = std::max(0, v_issued - kDecStages); j < v_issued; ++j)
+                dec_wait(&hd->v_full[j % kDecStages], (j / kDecStages) & 1, err);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -270,25 +338,25 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             for (int j = 0; j < n_tiles && good; ++j) {
                 if (j + 1 < n_tiles) {
                     // S_{j+1} into the buffer of S_{j-1}, once the softmax has read it
-                    const int b1 = (j + 1) & 1;
-                    good = dec_wait(&hd->k_full[b1], ((j + 1) >> 1) & 1, err) &&
-                           (j < 1 || dec_wait(&hd->s_empty[b1], ((j - 1) >> 1) & 1, err));
+                    const int sb1 = (j + 1) & 1, kb1 = (j + 1) % kDecStages;
+                    good = dec_wait(&hd->k_full[kb1], ((j + 1) / kDecStages) & 1, err) &&
+                           (j < 1 || dec_wait(&hd->s_empty[sb1], ((j - 1) >> 1) & 1, err));
                     if (!good) break;
                     tc_fence_after();
-                    dec_issue_qk(tmem + kDecColS + b1 * kDecN, sbase + kDecOffK + b1 * kDecTile,
+                    dec_issue_qk(tmem + kDecColS + sb1 * kDecN, sbase + kDecOffK + kb1 * kDecTile,
                                  sbase + kDecOffQ);
-                    mma_commit(&hd->s_full[b1]);
-                    mma_commit(&hd->k_empty[b1]);
+                    mma_commit(&hd->s_full[sb1]);
+                    mma_commit(&hd->k_empty[kb1]);
                 }
-                const int b = j & 1;
-                good = dec_wait(&hd->v_full[b], (j >> 1) & 1, err) &&
-                       dec_wait(&hd->p_ready[b], (j >> 1) & 1, err);
+                const int pb = j & 1, vb = j % kDecStages;
+                good = dec_wait(&hd->v_full[vb], (j / kDecStages) & 1, err) &&
+                       dec_wait(&hd->p_ready[pb], (j >> 1) & 1, err);
                 if (!good) break;
                 tc_fence_after();
-                dec_issue_pv(tmem + kDecColO, sbase + kDecOffV + b * kDecTile,
-                             sbase + kDecOffP + b * kDecP, j != 0);
-                mma_commit(&hd->p_empty[b]);
-                mma_commit(&hd->v_empty[b]);
+                dec_issue_pv(tmem + kDecColO, sbase + kDecOffV + vb * kDecTile,
+                             sbase + kDecOffP + pb * kDecP, j != 0);
+                mma_commit(&hd->p_empty[pb]);
+                mma_commit(&hd->v_empty[vb]);
             }
             mma_commit(&hd->done);
             dec_wait(&hd->done, 0, err);
@@ -351,20 +419,22 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 const float pv = valid ? dec_exp2(x[h] - base[h]) : 0.f;
                 const bf16 pq = __float2bfloat16_rn(pv);
                 if (good)
-                    *reinterpret_cast<bf16 *>(pb + swizzle_offset((uint32_t)h, (uint32_t)(r & 63))) =
-                        pq;
+                    *reinterpret_cast<bf16 *>(pb + swizzle_offset((uint32_t)h,
+                                                                  (uint32_t)(r & 63))) = pq;
                 l[h] = fmaf(l[h], corr[h], __bfloat162float(pq));
             }
             // a value tile that runs past the split's last position: its rows
             // there are zeroed before P_j V_j reads them
             if (j0 + j * kDecPos + kDecPos > j1) {
-                good = good && dec_wait(&hd->v_full[b], (j >> 1) & 1, err);
+                const int vb = j % kDecStages;
+                good = good && dec_wait(&hd->v_full[vb], (j / kDecStages) & 1, err);
                 if (good && !valid) {
-                    unsigned char *vt = smem + kDecOffV + b * kDecTile;
+                    unsigned char *vt = smem + kDecOffV + vb * kDecTile;
 #pragma unroll
                     for (int c = 0; c < 128; c += 8)
-                        *reinterpret_cast<uint4 *>(vt + (c >> 6) * kDecHalf +
-                                                   swizzle_offset((uint32_t)r, (uint32_t)(c & 63))) =
+                        *reinterpret_cast<uint4 *>(
+                            vt + (c >> 6) * kDecHalf +
+                            swizzle_offset((uint32_t)r, (uint32_t)(c & 63))) =
                             make_uint4(0u, 0u, 0u, 0u);
                 }
             }
@@ -406,25 +476,61 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             tmem_ld16(tmem + lane_base + kDecColO, o);
             tmem_ld_wait();
         }
+        if (n_split == 1) {
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-            const float Ls =
-                fin ? (hd->lsum[0][h] + hd->lsum[1][h]) + (hd->lsum[2][h] + hd->lsum[3][h]) : 0.f;
-            const int head = g * G + h;
-            if (n_split == 1) {
-                ctx[((size_t)t * Hq + head) * 128 + r] =
+            for (int h = 0; h < G; ++h) {
+                const float Ls = fin ? (hd->lsum[0][h] + hd->lsum[1][h]) +
+                                           (hd->lsum[2][h] + hd->lsum[3][h])
+                                     : 0.f;
+                ctx[((size_t)t * Hq + g * G + h) * 128 + r] =
                     __float2bfloat16_rn(Ls > 0.f ? o[h] / Ls : 0.f);
-            } else {
-                const size_t oi = ((size_t)t * Hq + head) * n_split + s;
+            }
+        } else {
+            // every CTA of the cluster has initialised its barriers
+            cluster_wait();
+            const uint32_t c = ptx::cluster_ctarank();
+            float *xo = reinterpret_cast<float *>(smem + kDecOffX);
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                // head h belongs to CTA h % n_split, row slot h / n_split
+                const uint32_t owner = (uint32_t)(h % n_split);
+                const int slot = h / n_split;
+                st_cluster_f32(&xo[((size_t)slot * n_split + c) * 128 + r], owner,
+                               fin ? o[h] : 0.f);
                 if (r == 0) {
-                    // (maximum, sum) in the natural-log form of the merge
-                    part_ml[2 * oi] = fin ? base[h] * 0.6931471805599453f : -INFINITY;
-                    part_ml[2 * oi + 1] = Ls;
+                    const float Ls = fin ? (hd->lsum[0][h] + hd->lsum[1][h]) +
+                                               (hd->lsum[2][h] + hd->lsum[3][h])
+                                         : 0.f;
+                    st_cluster_f32(&hd->ml[slot][c][0], owner, fin ? base[h] : -INFINITY);
+                    st_cluster_f32(&hd->ml[slot][c][1], owner, Ls);
                 }
-                part_acc[oi * 128 + r] = fin ? o[h] : 0.f;
+            }
+            // all four warps' stores issued, then one release arrival on
+            // every CTA's merge barrier (ordered after them)
+            ptx::named_bar_sync(1, 128);
+            if (threadIdx.x == 64)
+                for (int q = 0; q < n_split; ++q)
+                    ptx::mbar_arrive_cluster(
+                        ptx::map_rank(ptx::smem_u32(&hd->merge_full), (uint32_t)q));
+            // the heads this CTA owns (base 2: split weight 2^(base_s - M))
+            const bool got = ptx::mbar_wait_cluster(&hd->merge_full, 0, err);
+            for (int h = (int)c, slot = 0; h < G && got; h += n_split, ++slot) {
+                float M = -INFINITY;
+                for (int q = 0; q < n_split; ++q) M = fmaxf(M, hd->ml[slot][q][0]);
+                float A = 0.f, Ls = 0.f;
+                if (M != -INFINITY) {
+                    for (int q = 0; q < n_split; ++q) {
+                        const float w = exp2f(hd->ml[slot][q][0] - M);
+                        Ls = fmaf(w, hd->ml[slot][q][1], Ls);
+                        A = fmaf(w, xo[((size_t)slot * n_split + q) * 128 + r], A);
+                    }
+                }
+                ctx[((size_t)t * Hq + g * G + h) * 128 + r] =
+                    __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
             }
         }
     }
+    if (n_split > 1 && warp < 2) cluster_wait();  // (the aligned wait of every thread)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -435,20 +541,22 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 
 bool attn_decode_tc_ok() { return encode_fn() != nullptr; }
 
-int attn_decode_tc_splits(int T, int Hkv, int max_len, int split_cap) {
-    // one wave of one-CTA-per-SM blocks, at least one position tile a split
+int attn_decode_tc_splits(int T, int Hkv, int max_len) {
+    // one wave of one-CTA-per-SM blocks, at least one position tile a
+    // split, at most a portable cluster of splits
     const int tg = std::max(1, T * Hkv);
     int ns = std::max(1, device_info().sm_count / tg);
     ns = std::min(ns, (max_len + kDecPos - 1) / kDecPos);
-    return std::max(1, std::min(ns, split_cap));
+    return std::max(1, std::min(ns, kDecMaxSplit));
 }
 
 cudaError_t launch_attn_decode_tc(int T, int Hq, int Hkv, int n_seq, int L, int n_split,
                                   const int32_t *seq, const int32_t *pos, const void *q16,
-                                  const void *k_cache, const void *v_cache, float *part_ml,
-                                  float *part_acc, void *ctx, cudaStream_t st) {
+                                  const void *k_cache, const void *v_cache, void *ctx,
+                                  cudaStream_t st) {
     const int G = Hq / Hkv;
-    if (G < 1 || G > kDecMaxG || G * Hkv != Hq || n_split < 1) return cudaErrorInvalidValue;
+    if (G < 1 || G > kDecMaxG || G * Hkv != Hq || n_split < 1 || n_split > kDecMaxSplit)
+        return cudaErrorInvalidValue;
     CUtensorMap mq, mk, mv;
     const uint64_t rows = (uint64_t)n_seq * Hkv * L;
     if (!make_map(&mq, q16, (uint64_t)T * Hq, 128, kDecN) ||
@@ -471,10 +579,24 @@ cudaError_t launch_attn_decode_tc(int T, int Hq, int Hkv, int n_seq, int L, int 
     unsigned *err = device_info().err;
     bf16 *cp = static_cast<bf16 *>(ctx);
     int Hqv = Hq, Hkvv = Hkv, ns = n_seq, Lv = L, nsp = n_split;
-    void *args[] = {&mq, &mk, &mv, &Hqv, &Hkvv, &ns, &Lv, &nsp, &seq, &pos,
-                    &part_ml, &part_acc, &cp, &err};
+    void *args[] = {&mq, &mk, &mv, &Hqv, &Hkvv, &ns, &Lv, &nsp, &seq, &pos, &cp, &err};
+    // the splits of a (token, key/value head) form one cluster
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n_split, T * Hkv);
+    cfg.blockDim = dim3(kDecThreads);
+    cfg.dynamicSmemBytes = kDecSmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = n_split;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
     LaunchScope ls("attention_decode_tc", st);
-    return launch_pdl(kern, dim3(n_split, T * Hkv), dim3(kDecThreads), kDecSmem, st, args);
+    return cudaLaunchKernelExC(&cfg, kern, args);
 }
 
 }  // namespace moe

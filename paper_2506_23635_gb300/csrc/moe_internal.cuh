@@ -273,18 +273,17 @@ cudaError_t launch_attn_prefill_tc(int T, int Hq, int Hkv, int n_seq, int L, con
                                    const int32_t *pos, const void *q16, const void *k_cache,
                                    const void *v_cache, void *ctx, int *tile_ok, cudaStream_t st);
 // Decode attention on the tensor cores (attn_decode_tc.cu): every token of
-// the call over positions 0..pos[t] of its sequence, in n_split position
-// splits per (token, key/value head); a single split writes ctx, several
-// write the per-split (maximum, sum, weighted values) partials that
-// k_attn_merge combines.  Queries as above; query heads per key/value head
-// <= 8.  attn_decode_tc_splits: the split count for one wave of CTAs (at
-// most split_cap).
+// the call over positions 0..pos[t] of its sequence, in n_split (<= 8)
+// position splits per (token, key/value head) that form a cluster and merge
+// through distributed shared memory; ctx written.  Queries as above; query
+// heads per key/value head <= 8.  attn_decode_tc_splits: the split count for
+// one wave of CTAs.
 bool attn_decode_tc_ok();
-int attn_decode_tc_splits(int T, int Hkv, int max_len, int split_cap);
+int attn_decode_tc_splits(int T, int Hkv, int max_len);
 cudaError_t launch_attn_decode_tc(int T, int Hq, int Hkv, int n_seq, int L, int n_split,
                                   const int32_t *seq, const int32_t *pos, const void *q16,
-                                  const void *k_cache, const void *v_cache, float *part_ml,
-                                  float *part_acc, void *ctx, cudaStream_t st);
+                                  const void *k_cache, const void *v_cache, void *ctx,
+                                  cudaStream_t st);
 
 // name: the profiling name of the launch (default "gemm_down_tc").  y_tail
 // (optional, [T*K, D]): the stream-K schedule's second output; the result is

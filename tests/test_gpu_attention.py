@@ -370,3 +370,56 @@ def test_prefill_head_groups(Hq, Hkv):
     want = oracle.attention(q.reshape(T, Hq, dh).astype(np.float64), gen.to_f64(kc, "bf16"),
                             gen.to_f64(vc, "bf16"), seq, pos)
     assert_parity(to_numpy(ctx), want.reshape(T, -1), "bf16", f"prefill Hq={Hq} Hkv={Hkv}", True)
+
+
+def _decode_path_child():
+    """(run in a child process) A DBRX decode step, 8 sequences at context
+    2048, through moe_sa_forward: which attention kernel ran, and the block
+    against the oracle."""
+    import os
+    m = moe()
+    shape = gen.DBRX_ATTN
+    T, L = 8, 2048
+    w_qkv, w_o = gen.host_attn_weights(shape, 37)
+    kc, vc = gen.host_kv_cache(shape, T, L, 37)
+    seq = np.arange(T, dtype=np.int32)
+    pos = np.full(T, L - 1, np.int32)
+    pos[0] = 700  # a shorter context: a partial last tile, an empty split
+    x = np.random.default_rng(41).normal(size=(T, shape.d_model)).astype(np.float32)
+    want, _, _ = oracle.sa_forward(x.astype(np.float64), w_qkv, w_o, "bf16", 48, 8,
+                                   shape.rope_base, EPS, seq, pos, gen.to_f64(kc, "bf16"),
+                                   gen.to_f64(vc, "bf16"))
+    resid = torch.from_numpy(x).cuda()
+    m.profile_reset()
+    m.profile_enable(True)
+    m.sa_forward(_sa(m, shape), resid, dev(w_qkv, "bf16"), dev(w_o, "bf16"),
+                 torch.from_numpy(seq).cuda(), torch.from_numpy(pos).cuda(), dev(kc, "bf16"),
+                 dev(vc, "bf16"), eps=EPS)
+    assert m.get_last_error() == 0
+    m.profile_enable(False)
+    ran = {k for k, v in m.profile_read().items() if v[0] > 0}
+    expect = "attention" if os.environ.get("MOE_ATTN_CUDA_CORES") == "1" else "attention_decode_tc"
+    assert expect in ran, f"{expect} did not run: {sorted(ran)}"
+    assert_parity(to_numpy(resid) - x, want - x, "bf16", f"decode block on {expect}")
+    print("decode path ok:", expect)
+
+
+@pytest.mark.parametrize("cuda_cores", [False, True], ids=["tensor_cores", "cuda_cores"])
+def test_dbrx_decode_on_both_attention_kernels(cuda_cores):
+    """Decode steps attend on the tensor-core decode kernel by default and on
+    the CUDA-core kernel with MOE_ATTN_CUDA_CORES=1; both meet the block
+    bound (a fresh process each: the switch is read once)."""
+    need_gpu()
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ)
+    env.pop("MOE_ATTN_CUDA_CORES", None)
+    if cuda_cores:
+        env["MOE_ATTN_CUDA_CORES"] = "1"
+    p = subprocess.run([sys.executable, "-c",
+                        "import tests.test_gpu_attention as t; t._decode_path_child()"],
+                       cwd=root, env=env, capture_output=True, text=True, timeout=600)
+    assert p.returncode == 0, (p.stdout + p.stderr)[-3000:]
+    assert "decode path ok" in p.stdout
