@@ -25,7 +25,8 @@
 //    columns per run rather than up to 127 rows of a fixed 128-slot tile.
 // Units are numbered expert by expert, weight tile outer and slot tile inner
 // (units running at the same time share weight tiles in L2); CTA (pair) b of
-// G takes units b, b+G, ...
+// G takes units b, b+G, ... in full rounds, and a piece of one of the last
+// round's units (wm_item).
 //
 // Per CTA, 6 warps:
 //   warp 0     TMA producer (one lane): the A tile and the run's slot rows
@@ -158,6 +159,41 @@ __device__ __forceinline__ WmTile wm_tile(const int *tprefix, const int32_t *off
     return t;
 }
 
+// The work of pair (or CTA) `pair` of n_pairs, item i: units pair,
+// pair + n_pairs, ... in full rounds; the units of a last, partial round are
+// cut into pieces along their slot run (granules of `gran` slots) so that
+// the pairs the round would leave idle share them -- each piece keeps the
+// whole reduction, so every output element is still computed once, by one
+// MMA chain.  (768 down-projection units on 76 pairs of a 2048-token
+// prefill: the eleventh round held 8 units, now 64 pieces of 32 slots.)
+// False once the pair has no item i.  Items of zero width are skipped by
+// the caller (cnt == 0).
+__device__ __forceinline__ bool wm_item(const int *tprefix, const int32_t *offsets, int E,
+                                        int n_units, int pair, int n_pairs, int i, int gran,
+                                        WmTile &t) {
+    const int rounds = n_units / n_pairs, full = rounds * n_pairs;
+    if (i < rounds) {
+        t = wm_tile(tprefix, offsets, E, pair + i * n_pairs, gran);
+        return true;
+    }
+    const int rem = n_units - full;
+    if (i > rounds || rem == 0) return false;
+    // the tail round: pair -> (tail unit, piece)
+    const int max_pieces = kWmMaxN / gran;
+    const int P = max(1, min(max_pieces, n_pairs / rem));
+    const int tu = pair / P, q = pair - tu * P;
+    if (tu >= rem) return false;
+    t = wm_tile(tprefix, offsets, E, full + tu, gran);
+    const int g = t.n / gran;                      // granules of the run
+    const int a = g * q / P, b = g * (q + 1) / P;  // this piece's granules
+    const int s_a = a * gran;
+    t.s0 += s_a;
+    t.cnt = max(0, min(t.cnt, b * gran) - s_a);
+    t.n = (b - a) * gran;
+    if (t.n == 0) t.cnt = 0;
+    return true;
+}
+
 // A tensor copy that completes on the mbarrier at cluster address `bar` --
 // this CTA's or, in a CTA pair, the peer's (cta_group::2).
 template <int CG>
@@ -260,8 +296,11 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
             const uint64_t pol_x = ptx::policy_evict_last();
             uint32_t it = 0;
             bool ok = true;
-            for (int u = unit0; ok && u < n_units; u += ustride) {
-                const WmTile t = wm_tile(hd->tprefix, offsets, E, u, C::kGran);
+            WmTile t;
+            for (int i = 0; ok && wm_item(hd->tprefix, offsets, E, n_units, unit0, ustride, i,
+                                          C::kGran, t);
+                 ++i) {
+                if (t.cnt == 0) continue;
                 const uint32_t rows_b = (uint32_t)(t.n / CG);  // a multiple of 16, <= kRowsB
                 const int brow = t.s0 + (int)(rank * rows_b);
                 const int arow = t.e * Nw + (t.wt * CG + (int)rank) * C::kOutPerCta;
@@ -301,9 +340,13 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
             if (lane == 0) {
                 uint32_t it = 0, tl = 0;
                 bool ok = true;
-                for (int u = unit0; ok && u < n_units; u += ustride, ++tl) {
-                    const WmTile t = wm_tile(hd->tprefix, offsets, E, u, C::kGran);
+                WmTile t;
+                for (int i = 0; ok && wm_item(hd->tprefix, offsets, E, n_units, unit0, ustride,
+                                              i, C::kGran, t);
+                     ++i) {
+                    if (t.cnt == 0) continue;
                     const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
+                    ++tl;
                     // released by both CTAs' epilogues
                     if (!(ok = CG == 2 ? ptx::mbar_wait_cluster(&hd->tempty[acc], aph ^ 1, err)
                                        : ptx::mbar_wait(&hd->tempty[acc], aph ^ 1, err)))
@@ -348,9 +391,12 @@ k_gemm_wm(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUte
         uint32_t tl = 0, chunk = 0;
         const uint32_t tempty_issuer0 =
             CG == 2 ? ptx::map_rank(ptx::smem_u32(&hd->tempty[0]), 0) : 0u;
-        for (int u = unit0; u < n_units; u += ustride, ++tl) {
-            const WmTile t = wm_tile(hd->tprefix, offsets, E, u, C::kGran);
+        WmTile t;
+        for (int i = 0; wm_item(hd->tprefix, offsets, E, n_units, unit0, ustride, i, C::kGran, t);
+             ++i) {
+            if (t.cnt == 0) continue;
             const uint32_t acc = tl & 1, aph = (tl >> 1) & 1;
+            ++tl;
             if (!dead && !ptx::mbar_wait_hint(&hd->tfull[acc], aph, err)) dead = true;
             tc_fence_after();
             const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + acc * 256;

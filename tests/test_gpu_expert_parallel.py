@@ -153,7 +153,9 @@ def test_two_ranks_gloo_on_one_gpu(case):
     L = gen.host_layer(sh, T, 31)
     res = gen.to_f64(gen.host_normal((T, D), 1.0, "f32", 31, "residual"), "f32")
     want, _, _ = oracle.layer_tokens(L.x, L.w_r, L.w1, L.v1, L.w2, "bf16", K, residual=res)
-    out = mp.Manager().dict()
+    # the shared dict's manager process is spawned too: nothing is forked
+    # after this process has initialised CUDA
+    out = mp.get_context("spawn").Manager().dict()
     mp.start_processes(_ep_rank, args=(2, _free_port(), case, out), nprocs=2, join=True,
                        start_method="spawn")
     for r in range(2):
