@@ -734,6 +734,48 @@ def measure_dense(layer, T, steps=100, warmup=3):
             "kernels": kernel_table(kstats)}
 
 
+def measure_expert_share(layer, T, n_nodes, steps=100, warmup=3):
+    """One node's share of the expert-parallel layer (Sec. 4.3): the whole
+    routing and experts [0, E/P) of a P-node split, on this GPU, through
+    moe_layer_forward_experts -- the per-node MoE compute of Eq. 1, without
+    the all-reduce of the partials.  Also the distinct experts of the share
+    a step reads (its weight bytes)."""
+    import torch
+
+    shape = layer.shape
+    E = shape.n_experts
+    e_end = E // n_nodes
+    pool = 4 if T >= PREFILL_MIN_TOKENS else 16
+    xs_host, w_r_host, xs, w_r, ws, _ = layer.inputs(T, pool)
+    w1, v1, w2 = layer.w
+    d, moe = layer.d, layer.moe
+    part = torch.empty((T, shape.d_model), dtype=torch.float32, device=layer.dev)
+
+    def step(i):
+        moe.layer_forward_experts(d, xs[i % pool], w_r, 0, e_end, w1[:e_end], v1[:e_end],
+                                  w2[:e_end], out=part, ws=ws, stream=layer.stream)
+
+    for i in range(warmup):
+        step(i)
+    ms, _, kstats = layer.time_steps(step, steps)
+    U = []
+    for i in range(pool):
+        idx, _, _ = moe.route(d, xs[i], w_r)
+        U.append(len({e for e in idx.cpu().numpy().reshape(-1).tolist() if e < e_end}))
+    u_mean = float(np.mean(U))
+    share_bytes = u_mean * 3 * shape.d_model * shape.ffn_hidden * 2
+    peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
+    r = {"nodes": n_nodes, "experts": [0, e_end], "tokens_per_step": T,
+         "ms_per_step": round(ms, 4), "distinct_experts_of_share": u_mean,
+         "kernels": kernel_table(kstats)}
+    if T < PREFILL_MIN_TOKENS:
+        r["frac_of_hbm_step"] = round(share_bytes / (ms / 1e3) / 1e9 / peak, 4)
+    else:
+        flops = 2.0 * T * shape.top_k * 3 * shape.d_model * shape.ffn_hidden / n_nodes
+        r["tflops"] = round(flops / (ms / 1e3) / 1e12, 1)
+    return r
+
+
 def decoder_config(workload, shape, T, prefill, ctx_len=2048):
     """The ``config`` of a decoder-layer workload, the same for both arms."""
     return {"workload": workload, "d_model": shape.d_model, "ffn_hidden": shape.ffn_hidden,
@@ -874,6 +916,8 @@ def run_ours(args):
         extra["decode_sweep"] = [measure_extra(layer, f"dbrx-decode-t{t}", 200, 5, cpu_s)
                                  for t in (2, 4, 8, 16, 32, 64)]
         extra["busy_full_loading"] = [measure_dense(layer, t) for t in (1, 8)]
+        extra["expert_parallel_share"] = [measure_expert_share(layer, t, p)
+                                          for p in (2, 4) for t in (1, 8, 2048)]
         extra["decoder_layer"] = [measure_decoder_layer(layer, t) for t in (1, 8)]
         extra["decoder_prefill"] = [measure_decoder_layer(layer, t, steps=20, warmup=3,
                                                           prefill=True) for t in (128, 2048)]
