@@ -762,7 +762,9 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
     {
         const int *tok = tile_ok;
         int n_tg = c.T * Hkv;
-        const int gy = tile_ok ? std::min(n_tg, 8 * device_info().sm_count) : n_tg;
+        // (a prefill call usually leaves no token: one wave of CTAs that
+        // read the tile flags and find nothing to do)
+        const int gy = tile_ok ? std::min(n_tg, 2 * device_info().sm_count) : n_tg;
         void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &n_tg, &seq, &pos, &q, &kcp, &vcp, &ml,
                         &acc, &cp, &tok};
         LaunchScope ls("attention", c.st);
