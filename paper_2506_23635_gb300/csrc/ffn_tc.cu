@@ -528,12 +528,17 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
 
 __global__ void __launch_bounds__(256)
 k_gather_rows(int S, int D, int K, const bf16 *__restrict__ x, const int32_t *__restrict__ perm,
-              bf16 *__restrict__ xs, unsigned *err) {
+              bf16 *__restrict__ xs, const int32_t *__restrict__ range, int n_range,
+              unsigned *err) {
     ptx::grid_dependency_wait();
     const int nv = D >> 3;  // 16-byte vectors per row
-    const long long total = (long long)S * nv;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
+    // sorted positions [range[0], range[n_range]) only, when a range of
+    // experts is given (one node's share of an expert-parallel layer)
+    const int j_lo = range ? max(0, min(S, range[0])) : 0;
+    const int j_hi = range ? max(j_lo, min(S, range[n_range])) : S;
+    const long long total = (long long)j_hi * nv;
+    for (long long i = (long long)j_lo * nv + (long long)blockIdx.x * blockDim.x + threadIdx.x;
+         i < total; i += (long long)gridDim.x * blockDim.x) {
         const int j = (int)(i / nv), v = (int)(i - (long long)j * nv);
         int slot = perm[j];
         if (slot < 0 || slot >= S) {
@@ -600,7 +605,8 @@ bool tc_path_ok(const moe_dims &d) {
 }
 
 cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const int32_t *perm,
-                               void *x_sorted, cudaStream_t st) {
+                               void *x_sorted, cudaStream_t st, const int32_t *range,
+                               int n_range) {
     const int S = T * d.top_k;
     const long long total = (long long)S * (d.d_model / 8);
     const long long cap = (long long)device_info().sm_count * 8;
@@ -609,7 +615,7 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
     const bf16 *xp = static_cast<const bf16 *>(x);
     bf16 *xs = static_cast<bf16 *>(x_sorted);
     unsigned *err = device_info().err;
-    void *args[] = {&Sv, &D, &K, &xp, &perm, &xs, &err};
+    void *args[] = {&Sv, &D, &K, &xp, &perm, &xs, &range, &n_range, &err};
     LaunchScope ls("gather_rows", st);
     return launch_pdl((const void *)k_gather_rows, dim3(grid), dim3(256), 0, st, args);
 }

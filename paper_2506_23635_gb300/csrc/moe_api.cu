@@ -1437,7 +1437,7 @@ moe_status moe_layer_forward_experts(const moe_dims *dims, int32_t T, const void
         void *xs = at<void>(ws, L.xs);
         float *y = at<float>(ws, L.y);
         float *y_tail = T <= kStreamKMaxTokens ? at<float>(ws, L.y_tail) : nullptr;
-        e = launch_gather_rows(d, T, x, perm, xs, st);
+        e = launch_gather_rows(d, T, x, perm, xs, st, loff, dl.n_experts);
         if (e == cudaSuccess) e = launch_gemm_up_tc(dl, T, xs, loff, w1_local, v1_local, h, st);
         if (e == cudaSuccess)
             e = launch_gemm_down_tc(dl, T, h, loff, w2_local, y, st, nullptr, y_tail);

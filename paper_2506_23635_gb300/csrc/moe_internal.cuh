@@ -248,7 +248,8 @@ constexpr int kFusedCombineMaxTokens = 64;
 // tcgen05 grouped GEMMs (ffn_tc.cu), bf16 only; h is bf16, y_sorted fp32.
 bool tc_path_ok(const moe_dims &d);
 cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const int32_t *perm,
-                               void *x_sorted, cudaStream_t st);
+                               void *x_sorted, cudaStream_t st, const int32_t *range = nullptr,
+                               int n_range = 0);
 cudaError_t launch_gemm_up_tc(const moe_dims &d, int T, const void *x_sorted,
                               const int32_t *offsets, const void *w1, const void *v1, void *h,
                               cudaStream_t st);
