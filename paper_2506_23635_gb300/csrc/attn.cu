@@ -763,8 +763,9 @@ cudaError_t attend(const SaCall &c, const float *q, const int32_t *seq, const in
         const int *tok = tile_ok;
         int n_tg = c.T * Hkv;
         // (a prefill call usually leaves no token: one wave of CTAs that
-        // read the tile flags and find nothing to do)
-        const int gy = tile_ok ? std::min(n_tg, 2 * device_info().sm_count) : n_tg;
+        // read the tile flags and find nothing to do; otherwise a block per
+        // item up to the grid's y limit, the kernel looping past it)
+        const int gy = std::min(n_tg, tile_ok ? 2 * device_info().sm_count : 65535);
         void *args[] = {&Hqv, &Hkvv, &nsq, &Lv, &ns, &n_tg, &seq, &pos, &q, &kcp, &vcp, &ml,
                         &acc, &cp, &tok};
         LaunchScope ls("attention", c.st);
