@@ -33,21 +33,28 @@ def expert_range(n_experts: int, world_size: int, rank: int) -> tuple:
     return begin, begin + base + (1 if rank < extra else 0)
 
 
-def all_reduce_partials(partial, group=None):
+def all_reduce_partials(partial, group=None, stream=None):
     """Sum a rank's partial output [T, D] (fp32) over the group, in place;
-    returns it.  One collective per layer; without an initialised process
-    group (one node) the partial is already the sum."""
+    returns it.  One collective per layer, ordered after the work on
+    ``stream`` (default: torch's current stream) that wrote the partial;
+    without an initialised process group (one node) the partial is already
+    the sum."""
+    import contextlib
+
     import torch
     import torch.distributed as dist
 
     if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size(group) == 1:
         return partial
-    if partial.is_cuda and dist.get_backend(group) == "gloo":
-        host = partial.cpu()
-        dist.all_reduce(host, op=dist.ReduceOp.SUM, group=group)
-        partial.copy_(host)
-        return partial
-    dist.all_reduce(partial, op=dist.ReduceOp.SUM, group=group)
+    on = torch.cuda.stream(stream) if (partial.is_cuda and stream is not None) \
+        else contextlib.nullcontext()
+    with on:
+        if partial.is_cuda and dist.get_backend(group) == "gloo":
+            host = partial.cpu()
+            dist.all_reduce(host, op=dist.ReduceOp.SUM, group=group)
+            partial.copy_(host)
+            return partial
+        dist.all_reduce(partial, op=dist.ReduceOp.SUM, group=group)
     return partial
 
 
@@ -87,4 +94,4 @@ def layer_forward(d, x, shard: ExpertShard, residual=None, group=None, ws=None, 
                                         shard.w1, shard.v1, shard.w2,
                                         residual=residual if add_residual else None, ws=ws,
                                         stream=stream)
-    return all_reduce_partials(partial, group)
+    return all_reduce_partials(partial, group, stream)
