@@ -676,13 +676,13 @@ def measure_decoder_layer(layer, T, ctx_len=2048, steps=200, warmup=5, prefill=F
         step(i)
     ms, launches, kstats = layer.time_steps(step, steps)
     sa_names = ("sa_prenorm", "qkv_rows_tc", "qkv_gemm_tc", "rope_cache", "attention_tc",
-                "attention", "attn_merge", "o_rows_tc", "o_gemm_tc", "residual_add",
-                "residual_prenorm")
+                "attention_decode_tc", "attention", "attn_merge", "o_rows_tc", "o_gemm_tc",
+                "residual_add", "residual_prenorm")
     sa_ms = sum(v[1] for k, v in kstats.items() if k in sa_names) / steps
     b = sa_bytes(a, T, ctx_len)
     peak = float(measured_peaks()[0].get("hbm_gbs", HBM_FALLBACK_GBS))
     kv = T * ctx_len * a.n_kv_heads * a.head_dim * 4
-    att = kstats.get("attention")
+    att = kstats.get("attention_decode_tc") or kstats.get("attention")
     if prefill:  # tensor work: projections 2*T*(8192 + 6144)*6144, attention ~2*2*T^2/2*48*128
         sa_flops = 2.0 * T * (a_shape.qkv_rows + a.d_model) * a.d_model \
             + 2.0 * T * (T + 1) * a.n_heads * a.head_dim

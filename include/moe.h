@@ -345,7 +345,10 @@ int32_t moe_profile_read(moe_kernel_stat *stats, int32_t max_stats);
  * 0..pos[t] of its sequence: a prefill passes consecutive positions of one
  * sequence, a decode step one token per sequence.  The caller keeps the
  * (seq, pos) pairs of a call distinct and the positions below pos[t]
- * filled by earlier calls.  A token whose seq or pos lies outside the cache
+ * filled by earlier calls.  seq and pos are complete before the call in
+ * stream order (written by a copy, or by a kernel that lets the next launch
+ * start only when it ends: the decode attention reads them before it waits
+ * for the kernel ahead of it).  A token whose seq or pos lies outside the cache
  * is recorded as MOE_ERR_DEVICE_INDEX, writes nothing to the cache and gets a
  * zero ctx.
  *

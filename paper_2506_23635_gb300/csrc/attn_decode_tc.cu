@@ -12,12 +12,18 @@
 //                       MN-major A operand), P_j K-major in shared memory
 //
 // with S^T and O^T in tensor memory (lane = position, resp. dim; column =
-// head).  One CTA per (position split s, token t, key/value head g), over
-// the split's positions [j0, j1) of t's sequence in tiles of 128:
+// head).  One CTA per (position split c, token t, key/value head g); the
+// splits of (t, g) share the position tiles of t's sequence (128 positions
+// each): split c takes tiles c, c + n_split, c + 2 n_split first, then one
+// at a time from a counter in the cluster's CTA 0, so a split whose share
+// of the memory bandwidth runs ahead takes more tiles.  A CTA's j-th tile
+// goes to its stages in order and is published in a ring of tile indices
+// (-1 after its last):
 //
 //   warp 0      TMA: the group's bf16 query rows once, then key and value
 //               tiles into three-stage rings (each 32 KB: two boxes of 64
-//               dims with the 128-byte swizzle);
+//               dims with the 128-byte swizzle), the first three before the
+//               block-wide barrier of the set-up;
 //   warp 1      tensor memory (S^T twice, O^T: 48 of 64 columns) and the
 //               MMAs: S_{j+1} is issued as soon as its key tile has landed
 //               and the softmax has read S_{j-1}, O += P_j V_j once P_j is
@@ -30,21 +36,23 @@
 //               the maximum passes it by more than 8 (then O^T is rescaled
 //               in tensor memory, each thread its dim's row), bf16
 //               probabilities written into P_j (rows = heads, positions
-//               contiguous, 128-byte swizzle), rows of V_j past the split's
-//               last position zeroed (0 * NaN is NaN; those cache rows may
-//               hold anything).
+//               contiguous, 128-byte swizzle), rows of V_j past the
+//               sequence's last position zeroed (0 * NaN is NaN; those cache
+//               rows may hold anything).
 //
 // The end: each thread owns dim r of O^T; per head the row sums of the four
 // warps are added.  A single split writes ctx.  Several splits of one
 // (token, key/value head) are the CTAs of one thread-block cluster (at most
 // 8), and CTA c owns the heads h = c, c + n_split, ...: every CTA stores its
 // (base, sum) and O^T row of each head straight into the owner's shared
-// memory (distributed shared memory stores need no round trip), then
-// arrives on the owner's merge barrier with release semantics; the owner
-// waits for all n_split arrivals, combines its heads and writes their ctx.
-// (The stores wait until every CTA of the cluster has initialised its
-// barriers: each arrives on the cluster barrier at its start and waits on it
-// before storing, by when the wait is long satisfied.)
+// memory with asynchronous stores that count their bytes on the owner's
+// merge barrier (the owner expects all splits' bytes from its start), so
+// no sender waits for its stores or fences them; the owner's acquire wait
+// on the barrier sees every split's partials, then it combines its heads
+// and writes their ctx.  (The stores wait until every CTA of the cluster
+// has initialised its barriers: each arrives on the cluster barrier at its
+// start and waits on it before storing, by when the wait is long
+// satisfied.)
 //
 // Numerics as the prefill flash attention: bf16 queries and probabilities,
 // fp32 scores and accumulation; the row sum takes the probabilities as
@@ -67,6 +75,11 @@ constexpr int kDecMaxG = 8;    // query heads per key/value head
 constexpr int kDecThreads = 6 * 32;
 constexpr int kDecStages = 3;     // key and value tiles in flight
 constexpr int kDecMaxSplit = 8;   // splits of one (token, key/value head): a portable cluster
+// the position tiles of a CTA are published in a ring: the producer
+// publishes its tile j once S_{j-3} has been computed (after the softmax
+// took S_{j-5}, so after it read tile j-5), so a slot is rewritten long
+// after both its readers (issuer, softmax) took it
+constexpr int kDecRing = 8;
 constexpr uint32_t kDecHalf = kDecPos * 128;  // one 64-dim box of a key/value tile: 16 KB
 constexpr uint32_t kDecTile = 2 * kDecHalf;   // 32 KB
 constexpr uint32_t kDecNHalf = kDecN * 128;   // 16 rows x 64 elements: 2 KB
@@ -104,12 +117,15 @@ struct DecHeader {
     uint64_t s_empty[2];             // S_j read by the four softmax warps
     uint64_t p_ready[2];             // P_j written (four softmax warps)
     uint64_t p_empty[2];             // P_j V_j finished
+    uint64_t t_full[kDecRing];       // tile index j of this CTA published (producer)
     uint64_t done;
-    uint64_t merge_full;             // every split's partials stored here (n_split arrivals)
+    uint64_t merge_full;             // every split's partials stored here (their bytes)
     uint32_t tmem_base;
+    uint32_t next_tile;              // the cluster's tile counter (in CTA 0)
+    int tidx[kDecRing];              // position tile of this CTA's j-th tile, -1 past the last
     float red[2][4][kDecMaxG];  // the warps' tile maxima, by tile parity
     float lsum[4][kDecMaxG];    // the warps' row sums at the end
-    float ml[kDecMaxG][kDecMaxSplit][2];  // (base, sum) of the owned heads, by split
+    alignas(8) float ml[kDecMaxG][kDecMaxSplit][2];  // (base, sum) of the owned heads, by split
 };
 static_assert(sizeof(DecHeader) <= kDecHdrBytes, "decode attention header");
 
@@ -174,17 +190,36 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) 
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// Store a float into CTA `rank`'s shared memory (distributed shared memory
-// of the cluster), at the address this CTA's `p` has in its own.
-__device__ __forceinline__ void st_cluster_f32(float *p, uint32_t rank, float v) {
-    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(
-                     ptx::map_rank(ptx::smem_u32(p), rank)),
-                 "f"(v)
-                 : "memory");
+// Asynchronous stores into CTA `rank`'s shared memory that count their bytes
+// on that CTA's barrier `bar` (complete-tx, released at cluster scope): the
+// receiver's acquire wait on `bar` sees them, and the sender waits for
+// nothing.
+__device__ __forceinline__ void st_async_f32(float *p, uint32_t rank, uint64_t *bar, float v) {
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.f32 [%0], %1, [%2];" ::"r"(
+            ptx::map_rank(ptx::smem_u32(p), rank)),
+        "f"(v), "r"(ptx::map_rank(ptx::smem_u32(bar), rank))
+        : "memory");
 }
 
-__device__ __forceinline__ void cluster_arrive_relaxed() {
-    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+__device__ __forceinline__ void st_async_v2f32(float *p, uint32_t rank, uint64_t *bar, float a,
+                                               float b) {
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(
+            ptx::map_rank(ptx::smem_u32(p), rank)),
+        "f"(a), "f"(b), "r"(ptx::map_rank(ptx::smem_u32(bar), rank))
+        : "memory");
+}
+
+__device__ __forceinline__ void cluster_arrive_release() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+// Take the next value of a counter in a cluster CTA's shared memory.
+__device__ __forceinline__ uint32_t dec_take(uint32_t cluster_addr) {
+    uint32_t old;
+    asm volatile("atom.shared::cluster.add.u32 %0, [%1], 1;" : "=r"(old) : "r"(cluster_addr)
+                 : "memory");
+    return old;
 }
 __device__ __forceinline__ void cluster_wait() {
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
@@ -236,6 +271,12 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int s = blockIdx.x, tg = blockIdx.y;
     const int t = tg / Hkv, g = tg - t * Hkv;
+    // the token's sequence and position are inputs of the call, complete
+    // before it in stream order (no kernel of the library writes them): read
+    // first, their latency behind the set-up
+    const int sq = seq[t], p = pos[t];
+
+    const int c = s;  // rank in the cluster (the splits of one pair)
 
     if (threadIdx.x == 0) {
         ptx::mbar_init(&hd->q_full, 1);
@@ -251,39 +292,75 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             ptx::mbar_init(&hd->p_ready[b], 4);
             ptx::mbar_init(&hd->p_empty[b], 1);
         }
+        for (int b = 0; b < kDecRing; ++b) ptx::mbar_init(&hd->t_full[b], 1);
         ptx::mbar_init(&hd->done, 1);
-        ptx::mbar_init(&hd->merge_full, n_split);
+        ptx::mbar_init(&hd->merge_full, 1);
+        hd->next_tile = 0u;
+        if (n_split > 1) {
+            // the bytes every split stores here: an O^T row and (base, sum)
+            // for each head this CTA merges
+            const int owned = c < G ? (G - 1 - c) / n_split + 1 : 0;
+            ptx::mbar_arrive_expect_tx(&hd->merge_full,
+                                       (uint32_t)(n_split * owned * (kDecPos * 4 + 8)));
+        }
         ptx::fence_barrier_init();
         ptx::prefetch_tmap(&tmQ);
         ptx::prefetch_tmap(&tmK);
         ptx::prefetch_tmap(&tmV);
     }
-    if (warp == 1) tmem_alloc(&hd->tmem_base, kDecTmemCols);
     if (n_split > 1) {
-        // this CTA's barriers are initialised (thread 0, fenced at cluster
-        // scope): the cluster's other CTAs may store into it once they pass
-        // the matching wait
+        // this CTA's barriers and tile counter are initialised: the
+        // cluster's other CTAs may use them once they pass the matching wait
+        // (the arrival releases thread 0's stores at cluster scope)
         __syncthreads();
-        cluster_arrive_relaxed();
+        cluster_arrive_release();
     }
-    if (warp >= 2) {
-        // probability rows G..15 stay zero (the MMA's padding heads)
-        uint4 *pz = reinterpret_cast<uint4 *>(smem + kDecOffP);
-        for (int i = threadIdx.x - 64; i < (int)(2 * kDecP / 16); i += 128)
-            pz[i] = make_uint4(0u, 0u, 0u, 0u);
-    }
+    if (warp == 1) tmem_alloc(&hd->tmem_base, kDecTmemCols);
     // the output projection may launch now: it streams its weights into the
     // SMs this grid leaves free while the attention runs
     ptx::launch_dependents();
     ptx::grid_dependency_wait();  // queries and caches come from the previous kernel
-    const int sq = seq[t], p = pos[t];
     const bool ok = sq >= 0 && sq < n_seq && p >= 0 && p < L;
+    // the position tiles of the sequence: the splits share them, the first
+    // kDecStages of each split fixed (tile c + i n_split for split c), the
+    // rest taken one by one from a counter in CTA 0 of the cluster by
+    // whichever split frees a stage first (the splits' shares of the memory
+    // bandwidth differ); only the last tile of the sequence is partial
     const int n = ok ? p + 1 : 0;
-    // the split's positions: a multiple of the tile, so only the last tile
-    // of the sequence is partial
-    const int per = ((n + n_split - 1) / n_split + kDecPos - 1) / kDecPos * kDecPos;
-    const int j0 = min(n, s * per), j1 = min(n, j0 + per);
-    const int n_tiles = (j1 - j0 + kDecPos - 1) / kDecPos;
+    const int n_all = (n + kDecPos - 1) / kDecPos;
+    const int row0 = (sq * Hkv + g) * L;
+    int n_first = 0;  // fixed tiles of this split that exist
+    for (int i = 0; i < kDecStages; ++i) n_first += c + i * n_split < n_all ? 1 : 0;
+    // the producer (thread 0, which initialised the barriers) sends the
+    // query rows and the fixed tiles before the block-wide barrier: their
+    // stages are empty yet
+    if (threadIdx.x == 0) {
+        if (n_first > 0) {
+            const uint64_t pol_kv = ptx::policy_evict_first();  // read once
+            ptx::mbar_arrive_expect_tx(&hd->q_full, kDecQ);
+            for (int half = 0; half < 2; ++half)
+                ptx::tma_load_2d(smem + kDecOffQ + half * kDecNHalf, &tmQ, half * 64,
+                                 t * Hq + g * G, &hd->q_full, ptx::policy_evict_normal());
+            for (int j = 0; j < n_first; ++j) {
+                const int row = row0 + (c + j * n_split) * kDecPos;
+                ptx::mbar_arrive_expect_tx(&hd->k_full[j], kDecTile);
+                for (int half = 0; half < 2; ++half)
+                    ptx::tma_load_2d(smem + kDecOffK + j * kDecTile + half * kDecHalf, &tmK,
+                                     half * 64, row, &hd->k_full[j], pol_kv);
+                ptx::mbar_arrive_expect_tx(&hd->v_full[j], kDecTile);
+                for (int half = 0; half < 2; ++half)
+                    ptx::tma_load_2d(smem + kDecOffV + j * kDecTile + half * kDecHalf, &tmV,
+                                     half * 64, row, &hd->v_full[j], pol_kv);
+                hd->tidx[j] = c + j * n_split;
+                ptx::mbar_arrive(&hd->t_full[j]);
+            }
+        }
+        if (n_first < kDecStages) {
+            // no tile past these: the end is published now
+            hd->tidx[n_first] = -1;
+            ptx::mbar_arrive(&hd->t_full[n_first]);
+        }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -292,30 +369,44 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
-        if (lane == 0 && n_tiles > 0) {
-            const uint64_t pol_kv = ptx::policy_evict_first();  // read once
-            const uint64_t pol_q = ptx::policy_evict_normal();
-            const int qrow = t * Hq + g * G;
-            const int row0 = (sq * Hkv + g) * L + j0;
-            ptx::mbar_arrive_expect_tx(&hd->q_full, kDecQ);
-            for (int half = 0; half < 2; ++half)
-                ptx::tma_load_2d(smem + kDecOffQ + half * kDecNHalf, &tmQ, half * 64, qrow,
-                                 &hd->q_full, pol_q);
-            int k_issued = 0, v_issued = 0;
-            for (int j = 0; j < n_tiles; ++j) {
+        // (CTA 0's counter is initialised before the first take)
+        if (n_split > 1) cluster_wait();
+        if (lane == 0 && n_first == kDecStages) {
+            const uint64_t pol_kv = ptx::policy_evict_first();
+            const uint32_t counter = ptx::map_rank(ptx::smem_u32(&hd->next_tile), 0u);
+            // the next tile is taken one ahead: its counter round trip runs
+            // while the stage it goes to frees
+            int taken = 0;  // (a single split counts alone)
+            auto take = [&]() -> int {
+                return kDecStages * n_split +
+                       (n_split > 1 ? (int)dec_take(counter) : taken++);
+            };
+            int nxt = take();
+            int k_issued = kDecStages, v_issued = kDecStages;
+            for (int j = kDecStages;; ++j) {
+                const int tile = nxt;
+                if (tile >= n_all) {
+                    hd->tidx[j % kDecRing] = -1;
+                    ptx::mbar_arrive(&hd->t_full[j % kDecRing]);
+                    break;
+                }
+                nxt = take();
                 const int b = j % kDecStages;
                 const uint32_t ph = ((j / kDecStages) & 1) ^ 1;
+                const int row = row0 + tile * kDecPos;
                 if (!dec_wait(&hd->k_empty[b], ph, err)) break;
                 ptx::mbar_arrive_expect_tx(&hd->k_full[b], kDecTile);
                 for (int half = 0; half < 2; ++half)
                     ptx::tma_load_2d(smem + kDecOffK + b * kDecTile + half * kDecHalf, &tmK,
-                                     half * 64, row0 + j * kDecPos, &hd->k_full[b], pol_kv);
+                                     half * 64, row, &hd->k_full[b], pol_kv);
                 k_issued = j + 1;
+                hd->tidx[j % kDecRing] = tile;
+                ptx::mbar_arrive(&hd->t_full[j % kDecRing]);
                 if (!dec_wait(&hd->v_empty[b], ph, err)) break;
                 ptx::mbar_arrive_expect_tx(&hd->v_full[b], kDecTile);
                 for (int half = 0; half < 2; ++half)
                     ptx::tma_load_2d(smem + kDecOffV + b * kDecTile + half * kDecHalf, &tmV,
-                                     half * 64, row0 + j * kDecPos, &hd->v_full[b], pol_kv);
+                                     half * 64, row, &hd->v_full[b], pol_kv);
                 v_issued = j + 1;
             }
             // copies still in flight land before the block can exit
@@ -324,10 +415,17 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 dec_wait(&hd->k_full[j % kDecStages], (j / kDecStages) & 1, err);
             for (int j = std::max(0, v_issued - kDecStages); j < v_issued; ++j)
                 dec_wait(&hd->v_full[j % kDecStages], (j / kDecStages) & 1, err);
+        } else if (lane == 0 && n_first > 0) {
+            dec_wait(&hd->q_full, 0, err);
+            for (int j = 0; j < n_first; ++j) {
+                dec_wait(&hd->k_full[j], 0, err);
+                dec_wait(&hd->v_full[j], 0, err);
+            }
         }
+        __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0 && n_tiles > 0) {
+        if (lane == 0 && n_first > 0) {
             bool good = dec_wait(&hd->q_full, 0, err) && dec_wait(&hd->k_full[0], 0, err);
             if (good) {
                 tc_fence_after();
@@ -335,8 +433,12 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                 mma_commit(&hd->s_full[0]);
                 mma_commit(&hd->k_empty[0]);
             }
-            for (int j = 0; j < n_tiles && good; ++j) {
-                if (j + 1 < n_tiles) {
+            for (int j = 0; good; ++j) {
+                // is there a tile j + 1 (published by the producer)?
+                const int r1 = (j + 1) % kDecRing;
+                if (!(good = dec_wait(&hd->t_full[r1], ((j + 1) / kDecRing) & 1, err))) break;
+                const bool more = hd->tidx[r1] >= 0;
+                if (more) {
                     // S_{j+1} into the buffer of S_{j-1}, once the softmax has read it
                     const int sb1 = (j + 1) & 1, kb1 = (j + 1) % kDecStages;
                     good = dec_wait(&hd->k_full[kb1], ((j + 1) / kDecStages) & 1, err) &&
@@ -357,6 +459,7 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                              sbase + kDecOffP + pb * kDecP, j != 0);
                 mma_commit(&hd->p_empty[pb]);
                 mma_commit(&hd->v_empty[vb]);
+                if (!more) break;
             }
             mma_commit(&hd->done);
             dec_wait(&hd->done, 0, err);
@@ -364,6 +467,20 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax
+        {
+            // probability rows G..15 of both buffers stay zero (the MMA's
+            // padding heads; no thread writes them later, and each thread's
+            // proxy fence before it releases P_0 covers its zeros)
+            constexpr int kPadRow = G * 8;  // 16-byte chunks before row G of a half
+            constexpr int kPad = 16 * 8 - kPadRow;
+            for (int i = threadIdx.x - 64; i < 4 * kPad; i += 128) {
+                uint4 *half = reinterpret_cast<uint4 *>(smem + kDecOffP) + (i / kPad) * (kDecNHalf / 16);
+                half[kPadRow + i % kPad] = make_uint4(0u, 0u, 0u, 0u);
+            }
+        }
+        // every CTA of the cluster has initialised its barriers before this
+        // one's merge stores (waited here, long before they are needed)
+        if (n_split > 1) cluster_wait();
         const int qd = warp & 3;       // tensor-memory lane quarter
         const int r = qd * 32 + lane;  // position of the tile; dim of O^T
         const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
@@ -375,10 +492,17 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             l[h] = 0.f;
         }
         bool good = true;
-        for (int j = 0; j < n_tiles; ++j) {
+        int m = 0;  // tiles this split has had
+        for (int j = 0;; ++j) {
             const int b = j & 1;
-            const int pj = j0 + j * kDecPos + r;
-            const bool valid = pj < j1;
+            good = good && dec_wait(&hd->t_full[j % kDecRing], (j / kDecRing) & 1, err);
+            // (lane 0's reading steers the warp: its loop stays converged)
+            const int tile =
+                __shfl_sync(0xffffffffu, good ? hd->tidx[j % kDecRing] : -1, 0);
+            if (tile < 0) break;
+            m = j + 1;
+            const int pj = tile * kDecPos + r;
+            const bool valid = pj < n;
             // (the load runs on every lane whatever its waits returned: it is
             // warp-collective; after a failed wait the values are not used)
             float v[16];
@@ -425,7 +549,7 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             }
             // a value tile that runs past the split's last position: its rows
             // there are zeroed before P_j V_j reads them
-            if (j0 + j * kDecPos + kDecPos > j1) {
+            if (tile * kDecPos + kDecPos > n) {
                 const int vb = j % kDecStages;
                 good = good && dec_wait(&hd->v_full[vb], (j / kDecStages) & 1, err);
                 if (good && !valid) {
@@ -459,8 +583,8 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         }
         // the split's result: O^T row r (dim r) of every head, the row sums
         // of the four warps added in warp order
-        bool fin = good && n_tiles > 0;
-        if (fin) fin = dec_wait(&hd->p_empty[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1, err);
+        bool fin = good && m > 0;
+        if (fin) fin = dec_wait(&hd->p_empty[(m - 1) & 1], ((m - 1) >> 1) & 1, err);
         fin = __all_sync(0xffffffffu, fin);
 #pragma unroll
         for (int h = 0; h < G; ++h) {
@@ -483,54 +607,63 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                                            (hd->lsum[2][h] + hd->lsum[3][h])
                                      : 0.f;
                 ctx[((size_t)t * Hq + g * G + h) * 128 + r] =
-                    __float2bfloat16_rn(Ls > 0.f ? o[h] / Ls : 0.f);
+                    __float2bfloat16_rn(Ls > 0.f ? __fdividef(o[h], Ls) : 0.f);
             }
         } else {
-            // every CTA of the cluster has initialised its barriers
-            cluster_wait();
-            const uint32_t c = ptx::cluster_ctarank();
             float *xo = reinterpret_cast<float *>(smem + kDecOffX);
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                // head h belongs to CTA h % n_split, row slot h / n_split
+                // head h belongs to CTA h % n_split, row slot h / n_split;
+                // the stores count their bytes on the owner's merge barrier
                 const uint32_t owner = (uint32_t)(h % n_split);
                 const int slot = h / n_split;
-                st_cluster_f32(&xo[((size_t)slot * n_split + c) * 128 + r], owner,
-                               fin ? o[h] : 0.f);
+                st_async_f32(&xo[((size_t)slot * n_split + c) * 128 + r], owner, &hd->merge_full,
+                             fin ? o[h] : 0.f);
                 if (r == 0) {
                     const float Ls = fin ? (hd->lsum[0][h] + hd->lsum[1][h]) +
                                                (hd->lsum[2][h] + hd->lsum[3][h])
                                          : 0.f;
-                    st_cluster_f32(&hd->ml[slot][c][0], owner, fin ? base[h] : -INFINITY);
-                    st_cluster_f32(&hd->ml[slot][c][1], owner, Ls);
+                    st_async_v2f32(&hd->ml[slot][c][0], owner, &hd->merge_full,
+                                   fin ? base[h] : -INFINITY, Ls);
                 }
             }
-            // all four warps' stores issued, then one release arrival on
-            // every CTA's merge barrier (ordered after them)
-            ptx::named_bar_sync(1, 128);
-            if (threadIdx.x == 64)
-                for (int q = 0; q < n_split; ++q)
-                    ptx::mbar_arrive_cluster(
-                        ptx::map_rank(ptx::smem_u32(&hd->merge_full), (uint32_t)q));
-            // the heads this CTA owns (base 2: split weight 2^(base_s - M))
+            // the heads this CTA owns (base 2: split weight 2^(base_s - M)),
+            // once every split's bytes have landed
             const bool got = ptx::mbar_wait_cluster(&hd->merge_full, 0, err);
-            for (int h = (int)c, slot = 0; h < G && got; h += n_split, ++slot) {
-                float M = -INFINITY;
-                for (int q = 0; q < n_split; ++q) M = fmaxf(M, hd->ml[slot][q][0]);
+            // (unrolled to the bounds and predicated, so that the heads' and
+            // the splits' loads go out together: n_split >= 2 leaves at most
+            // (G + 1) / 2 heads to a CTA)
+#pragma unroll
+            for (int slot = 0; slot < (G + 1) / 2; ++slot) {
+                const int h = (int)c + slot * n_split;
+                if (!got || h >= G) continue;
+                float bq[kDecMaxSplit], M = -INFINITY;
+#pragma unroll
+                for (int q = 0; q < kDecMaxSplit; ++q) {
+                    bq[q] = q < n_split ? hd->ml[slot][q][0] : -INFINITY;
+                    M = fmaxf(M, bq[q]);
+                }
                 float A = 0.f, Ls = 0.f;
                 if (M != -INFINITY) {
-                    for (int q = 0; q < n_split; ++q) {
-                        const float w = exp2f(hd->ml[slot][q][0] - M);
-                        Ls = fmaf(w, hd->ml[slot][q][1], Ls);
-                        A = fmaf(w, xo[((size_t)slot * n_split + q) * 128 + r], A);
+#pragma unroll
+                    for (int q = 0; q < kDecMaxSplit; ++q) {
+                        if (q < n_split) {
+                            const float w = dec_exp2(bq[q] - M);
+                            Ls = fmaf(w, hd->ml[slot][q][1], Ls);
+                            A = fmaf(w, xo[(slot * n_split + q) * 128 + r], A);
+                        }
                     }
                 }
+                // (Ls is a sum of probabilities of at most 2^8 each: far
+                // inside the fast division's range)
                 ctx[((size_t)t * Hq + g * G + h) * 128 + r] =
-                    __float2bfloat16_rn(Ls > 0.f ? A / Ls : 0.f);
+                    __float2bfloat16_rn(Ls > 0.f ? __fdividef(A, Ls) : 0.f);
             }
         }
     }
-    if (n_split > 1 && warp < 2) cluster_wait();  // (the aligned wait of every thread)
+    // (the aligned wait of every thread: producer and softmax warps waited
+    // at their start)
+    if (n_split > 1 && warp == 1) cluster_wait();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();

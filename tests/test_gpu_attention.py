@@ -423,3 +423,38 @@ def test_dbrx_decode_on_both_attention_kernels(cuda_cores):
                        cwd=root, env=env, capture_output=True, text=True, timeout=600)
     assert p.returncode == 0, (p.stdout + p.stderr)[-3000:]
     assert "decode path ok" in p.stdout
+
+
+# (Hq, Hkv, sequences = decode tokens, max_len): the tensor-core decode
+# kernel's position tiles shared between the splits of one (token, key/value
+# head): one split that takes all its tiles after the first three (192 pairs),
+# three splits over up to 20 tiles (50 pairs), eight splits over up to 40
+# tiles (2 pairs), and short sequences whose splits have fewer than three
+# tiles or none; positions random, with 0 and max_len - 1 present.
+SHARED_TILES = [(16, 8, 24, 1000), (6, 1, 50, 2500), (8, 1, 2, 5000), (6, 2, 9, 300)]
+
+
+@pytest.mark.parametrize("Hq,Hkv,n_seq,L", SHARED_TILES,
+                         ids=["one-split", "three-splits", "eight-splits", "short"])
+def test_decode_splits_share_position_tiles(Hq, Hkv, n_seq, L):
+    m = moe()
+    rng = np.random.default_rng(11)
+    shape = gen.AttnShape(Hq * 128, Hq, Hkv, 128, 10000.0, "bf16")
+    kc, vc = gen.host_kv_cache(shape, n_seq, L, 11)
+    seq = np.arange(n_seq, dtype=np.int32)
+    pos = rng.integers(0, L, size=n_seq).astype(np.int32)
+    pos[0], pos[-1] = 0, L - 1
+    q = rng.normal(size=(n_seq, Hq, 128)).astype(np.float32)
+    a = m.sa_dims(shape.d_model, Hq, Hkv, 128, shape.rope_base)
+    m.profile_enable(True)
+    m.profile_reset()
+    ctx = m.sa_attend(a, torch.from_numpy(q).cuda(), torch.from_numpy(seq).cuda(),
+                      torch.from_numpy(pos).cuda(), dev(kc, "bf16"), dev(vc, "bf16"))
+    torch.cuda.synchronize()
+    ran = {k for k, v in m.profile_read().items() if v[0] > 0}
+    m.profile_enable(False)
+    assert m.get_last_error() == 0
+    assert "attention_decode_tc" in ran, sorted(ran)
+    want = oracle.attention(oracle.round_bf16(q.astype(np.float64)), gen.to_f64(kc, "bf16"),
+                            gen.to_f64(vc, "bf16"), seq, pos)
+    assert_parity(to_numpy(ctx), want.reshape(n_seq, Hq * 128), "bf16", "attention ctx", True)
