@@ -527,26 +527,42 @@ k_gemm_swap(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
 // ---- gather of the A operand: x_sorted[j, :] = x[perm[j] / K, :] ----------------
 
 __global__ void __launch_bounds__(256)
-k_gather_rows(int S, int D, int K, const bf16 *__restrict__ x, const int32_t *__restrict__ perm,
-              bf16 *__restrict__ xs, const int32_t *__restrict__ range, int n_range,
-              unsigned *err) {
+k_gather_rows(int S, int D, int K, int n_chunk, const bf16 *__restrict__ x,
+              const int32_t *__restrict__ perm, bf16 *__restrict__ xs,
+              const int32_t *__restrict__ range, int n_range, unsigned *err) {
     ptx::grid_dependency_wait();
     const int nv = D >> 3;  // 16-byte vectors per row
     // sorted positions [range[0], range[n_range]) only, when a range of
     // experts is given (one node's share of an expert-parallel layer)
     const int j_lo = range ? max(0, min(S, range[0])) : 0;
     const int j_hi = range ? max(j_lo, min(S, range[n_range])) : S;
-    const long long total = (long long)j_hi * nv;
-    for (long long i = (long long)j_lo * nv + (long long)blockIdx.x * blockDim.x + threadIdx.x;
-         i < total; i += (long long)gridDim.x * blockDim.x) {
-        const int j = (int)(i / nv), v = (int)(i - (long long)j * nv);
+    // a warp per (sorted row, chunk of the row): n_chunk chunks a row, so
+    // that few rows still spread over the SMs; four 16-byte loads of each
+    // lane in flight
+    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+    const int per = (nv + n_chunk - 1) / n_chunk;
+    const long long n_items = (long long)(j_hi - j_lo) * n_chunk;
+    for (long long i = (long long)blockIdx.x * wpb + (threadIdx.x >> 5); i < n_items;
+         i += (long long)gridDim.x * wpb) {
+        const int j = j_lo + (int)(i / n_chunk), c = (int)(i % n_chunk);
         int slot = perm[j];
         if (slot < 0 || slot >= S) {
-            set_error(err, kErrIndex);
+            if (lane == 0) set_error(err, kErrIndex);
             slot = 0;
         }
-        const uint4 val = __ldg(reinterpret_cast<const uint4 *>(x + (size_t)(slot / K) * D) + v);
-        reinterpret_cast<uint4 *>(xs + (size_t)j * D)[v] = val;
+        const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)(slot / K) * D);
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + (size_t)j * D);
+        const int v1 = min(nv, (c + 1) * per);
+        int v = c * per + lane;
+        for (; v + 96 < v1; v += 128) {
+            const uint4 a0 = __ldg(src + v), a1 = __ldg(src + v + 32);
+            const uint4 a2 = __ldg(src + v + 64), a3 = __ldg(src + v + 96);
+            dst[v] = a0;
+            dst[v + 32] = a1;
+            dst[v + 64] = a2;
+            dst[v + 96] = a3;
+        }
+        for (; v < v1; v += 32) dst[v] = __ldg(src + v);
     }
 }
 
@@ -608,14 +624,17 @@ cudaError_t launch_gather_rows(const moe_dims &d, int T, const void *x, const in
                                void *x_sorted, cudaStream_t st, const int32_t *range,
                                int n_range) {
     const int S = T * d.top_k;
-    const long long total = (long long)S * (d.d_model / 8);
-    const long long cap = (long long)device_info().sm_count * 8;
-    const int grid = (int)std::max(1LL, std::min((total + 255) / 256, cap));
+    // 8 warps a block, at most 8 blocks per SM; a row in chunks of at least
+    // 32 vectors when there are fewer rows than 64 warps per SM
+    const int warps = device_info().sm_count * 64;
+    int n_chunk = std::max(1, std::min(d.d_model / 8 / 32, warps / std::max(1, S)));
+    const long long items = (long long)S * n_chunk;
+    const int grid = (int)std::max(1LL, std::min((items + 7) / 8, (long long)warps / 8));
     int Sv = S, D = d.d_model, K = d.top_k;
     const bf16 *xp = static_cast<const bf16 *>(x);
     bf16 *xs = static_cast<bf16 *>(x_sorted);
     unsigned *err = device_info().err;
-    void *args[] = {&Sv, &D, &K, &xp, &perm, &xs, &range, &n_range, &err};
+    void *args[] = {&Sv, &D, &K, &n_chunk, &xp, &perm, &xs, &range, &n_range, &err};
     LaunchScope ls("gather_rows", st);
     return launch_pdl((const void *)k_gather_rows, dim3(grid), dim3(256), 0, st, args);
 }
