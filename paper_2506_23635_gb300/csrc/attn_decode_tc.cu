@@ -492,7 +492,7 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             l[h] = 0.f;
         }
         bool good = true;
-        int m = 0;  // tiles this split has had
+        int had = 0;  // tiles this split has had
         for (int j = 0;; ++j) {
             const int b = j & 1;
             good = good && dec_wait(&hd->t_full[j % kDecRing], (j / kDecRing) & 1, err);
@@ -500,7 +500,7 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
             const int tile =
                 __shfl_sync(0xffffffffu, good ? hd->tidx[j % kDecRing] : -1, 0);
             if (tile < 0) break;
-            m = j + 1;
+            had = j + 1;
             const int pj = tile * kDecPos + r;
             const bool valid = pj < n;
             // (the load runs on every lane whatever its waits returned: it is
@@ -547,8 +547,8 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
                                                                   (uint32_t)(r & 63))) = pq;
                 l[h] = fmaf(l[h], corr[h], __bfloat162float(pq));
             }
-            // a value tile that runs past the split's last position: its rows
-            // there are zeroed before P_j V_j reads them
+            // a value tile that runs past the sequence's last position: its
+            // rows there are zeroed before P_j V_j reads them
             if (tile * kDecPos + kDecPos > n) {
                 const int vb = j % kDecStages;
                 good = good && dec_wait(&hd->v_full[vb], (j / kDecStages) & 1, err);
@@ -583,8 +583,8 @@ k_attn_decode_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant_
         }
         // the split's result: O^T row r (dim r) of every head, the row sums
         // of the four warps added in warp order
-        bool fin = good && m > 0;
-        if (fin) fin = dec_wait(&hd->p_empty[(m - 1) & 1], ((m - 1) >> 1) & 1, err);
+        bool fin = good && had > 0;
+        if (fin) fin = dec_wait(&hd->p_empty[(had - 1) & 1], ((had - 1) >> 1) & 1, err);
         fin = __all_sync(0xffffffffu, fin);
 #pragma unroll
         for (int h = 0; h < G; ++h) {
