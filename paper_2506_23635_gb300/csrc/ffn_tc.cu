@@ -537,8 +537,8 @@ k_gather_rows(int S, int D, int K, int n_chunk, const bf16 *__restrict__ x,
     const int j_lo = range ? max(0, min(S, range[0])) : 0;
     const int j_hi = range ? max(j_lo, min(S, range[n_range])) : S;
     // a warp per (sorted row, chunk of the row): n_chunk chunks a row, so
-    // that few rows still spread over the SMs; four 16-byte loads of each
-    // lane in flight
+    // that few rows still spread over the SMs; eight 16-byte loads of each
+    // lane in flight (2048-token prefill: 31 -> 27.5 us against four)
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
     const int per = (nv + n_chunk - 1) / n_chunk;
     const long long n_items = (long long)(j_hi - j_lo) * n_chunk;
@@ -554,6 +554,13 @@ k_gather_rows(int S, int D, int K, int n_chunk, const bf16 *__restrict__ x,
         uint4 *dst = reinterpret_cast<uint4 *>(xs + (size_t)j * D);
         const int v1 = min(nv, (c + 1) * per);
         int v = c * per + lane;
+        for (; v + 224 < v1; v += 256) {
+            uint4 a[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) a[u] = __ldg(src + v + 32 * u);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) dst[v + 32 * u] = a[u];
+        }
         for (; v + 96 < v1; v += 128) {
             const uint4 a0 = __ldg(src + v), a1 = __ldg(src + v + 32);
             const uint4 a2 = __ldg(src + v + 64), a3 = __ldg(src + v + 96);
