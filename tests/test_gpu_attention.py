@@ -458,3 +458,42 @@ def test_decode_splits_share_position_tiles(Hq, Hkv, n_seq, L):
     want = oracle.attention(oracle.round_bf16(q.astype(np.float64)), gen.to_f64(kc, "bf16"),
                             gen.to_f64(vc, "bf16"), seq, pos)
     assert_parity(to_numpy(ctx), want.reshape(n_seq, Hq * 128), "bf16", "attention ctx", True)
+
+
+def _random_decode_configs(n=12, seed=2024):
+    """Seeded decode calls over the tensor-core kernel's launch shapes: head
+    groups of 1-8, one to eight position splits per (token, key/value head)
+    (SMs / pairs, at most the cache's tiles), caches of 1-40 tiles with
+    ragged ends, and tokens at random positions (some at 0, some at the last
+    cache row)."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n):
+        G = int(rng.integers(1, 9))
+        Hkv = int(rng.choice([1, 2, 4, 8]))
+        n_seq = int(rng.integers(1, 25))
+        L = int(rng.integers(1, 5121))
+        n_seq = max(1, min(n_seq, 120_000 // (Hkv * L)))  # caches of at most ~30 MB
+        out.append((G * Hkv, Hkv, n_seq, L, int(rng.integers(0, 1 << 30))))
+    return out
+
+
+@pytest.mark.parametrize("Hq,Hkv,n_seq,L,s", _random_decode_configs())
+def test_decode_random_launch_shapes(Hq, Hkv, n_seq, L, s):
+    m = moe()
+    rng = np.random.default_rng(s)
+    shape = gen.AttnShape(Hq * 128, Hq, Hkv, 128, 10000.0, "bf16")
+    kc, vc = gen.host_kv_cache(shape, n_seq, L, s % 1000)
+    seq = rng.permutation(n_seq).astype(np.int32)
+    pos = rng.integers(0, L, size=n_seq).astype(np.int32)
+    pos[rng.random(n_seq) < 0.15] = 0
+    pos[rng.random(n_seq) < 0.15] = L - 1
+    q = rng.normal(size=(n_seq, Hq, 128)).astype(np.float32)
+    a = m.sa_dims(shape.d_model, Hq, Hkv, 128, shape.rope_base)
+    ctx = m.sa_attend(a, torch.from_numpy(q).cuda(), torch.from_numpy(seq).cuda(),
+                      torch.from_numpy(pos).cuda(), dev(kc, "bf16"), dev(vc, "bf16"))
+    torch.cuda.synchronize()
+    assert m.get_last_error() == 0
+    want = oracle.attention(oracle.round_bf16(q.astype(np.float64)), gen.to_f64(kc, "bf16"),
+                            gen.to_f64(vc, "bf16"), seq, pos)
+    assert_parity(to_numpy(ctx), want.reshape(n_seq, Hq * 128), "bf16", "attention ctx", True)
