@@ -40,6 +40,27 @@ SMALL = [
 ]
 
 
+def _random_cases(n=16, seed=77):
+    """Seeded layer shapes over the validated ranges (D, F multiples of 8 up
+    to 768, E up to 32, K up to min(E, 8), T from 1 to 600, a quarter fp32):
+    every kernel path of the layer (one-token streaming, decode-batch
+    tiles, prefill CTA pairs, CUDA-core GEMV) on shapes no table lists."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        D = 8 * int(rng.integers(1, 97))
+        F = 8 * int(rng.integers(1, 97))
+        E = int(rng.integers(1, 33))
+        K = int(rng.integers(1, min(E, 8) + 1))
+        T = int(rng.choice([int(rng.integers(1, 17)), int(rng.integers(17, 81)),
+                            int(rng.integers(81, 601))]))
+        out.append((D, F, E, K, T, "f32" if rng.random() < 0.25 else "bf16"))
+    return out
+
+
+RANDOM = _random_cases()
+
+
 def _host(case, seed=3, skew=None):
     D, F, E, K, T, dt = case
     shape = gen.LayerShape(D, F, E, K, dt)
@@ -57,7 +78,7 @@ def _devlayer(L):
     return [dev(a, dt) for a in (L.x, L.w_r, L.w1, L.v1, L.w2)]
 
 
-@pytest.mark.parametrize("case", SMALL, ids=lambda c: "D{}F{}E{}K{}T{}{}".format(*c))
+@pytest.mark.parametrize("case", SMALL + RANDOM, ids=lambda c: "D{}F{}E{}K{}T{}{}".format(*c))
 def test_steps_and_layer(case):
     m = moe()
     L = _host(case)
@@ -81,11 +102,14 @@ def test_steps_and_layer(case):
     y = m.expert_ffn(d, x, perm, offsets, w1, v1, w2)
     assert_parity(to_numpy(y), ref["y_sorted"], sh.dtype, "expert_ffn y_sorted")
 
+    # a bf16 output carries its storage rounding on top of the bound (reading
+    # C22): few-term outputs (small F) have elements far above their RMS
+    stored = sh.dtype == "bf16"
     out = m.combine(d, y, inv, gate)
-    assert_parity(to_numpy(out), ref["out"], sh.dtype, "combine")
+    assert_parity(to_numpy(out), ref["out"], sh.dtype, "combine", stored)
 
     out2 = m.layer_forward(d, x, w_r, w1, v1, w2)
-    assert_parity(to_numpy(out2), ref["out"], sh.dtype, "layer_forward")
+    assert_parity(to_numpy(out2), ref["out"], sh.dtype, "layer_forward", stored)
     assert m.get_last_error() == 0
 
 
