@@ -9,7 +9,7 @@ import torch
 
 import oracle
 from paper_2506_23635_gb300 import inputs as gen
-from tests.gpu_util import assert_parity, dev, need_gpu, to_numpy
+from tests.gpu_util import assert_parity, h_rounding_allowance, dev, need_gpu, to_numpy
 
 pytestmark = pytest.mark.gpu
 
@@ -99,12 +99,20 @@ def test_steps_and_layer(case):
     assert np.array_equal(perm.cpu().numpy(), ref["perm"])
     assert np.array_equal(inv.cpu().numpy(), ref["inv_perm"])
 
-    y = m.expert_ffn(d, x, perm, offsets, w1, v1, w2)
-    assert_parity(to_numpy(y), ref["y_sorted"], sh.dtype, "expert_ffn y_sorted")
-
-    # a bf16 output carries its storage rounding on top of the bound (reading
-    # C22): few-term outputs (small F) have elements far above their RMS
+    # bf16: the ungated expert outputs (an intermediate) come from the GLU
+    # hidden vector stored in bf16 (reading C7): where few terms are summed
+    # (small F) an element far above the RMS can carry more of that rounding
+    # than the RMS bound, so each element of y_sorted gets the rounding's
+    # worst case as an allowance.  The layer output keeps the layer bound,
+    # plus its own bf16 storage rounding (reading C22).
+    extra_y = None
     stored = sh.dtype == "bf16"
+    if stored:
+        extra_y = h_rounding_allowance(ref["h_sorted"], gen.to_f64(L.w2, "bf16"),
+                                       ref["offsets"])
+    y = m.expert_ffn(d, x, perm, offsets, w1, v1, w2)
+    assert_parity(to_numpy(y), ref["y_sorted"], sh.dtype, "expert_ffn y_sorted", extra=extra_y)
+
     out = m.combine(d, y, inv, gate)
     assert_parity(to_numpy(out), ref["out"], sh.dtype, "combine", stored)
 
