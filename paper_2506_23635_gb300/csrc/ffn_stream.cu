@@ -93,10 +93,12 @@ k_up_glu_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ x,
     const int W = n_stages;  // consumer warps; warp W is the producer
 
     if (threadIdx.x == 0) init_header(hd, n_stages);
-    // one CTA per SM, all resident: the next kernel's CTAs can only take an
-    // SM this grid has left, so let them launch (and wait on the device) now
-    ptx::launch_dependents();
     ptx::grid_dependency_wait();  // perm/offsets come from the previous kernel
+    // the next kernel's CTAs may launch now (they take the SMs this grid
+    // leaves); triggered after the wait, so a CTA of it that starts finds
+    // the kernels before this one complete (the down projection reads the
+    // dispatch offsets before its own wait)
+    ptx::launch_dependents();
     if (warp == 0) chunk_prefix<NS>(offsets, E, S, hd->prefix, err);
     __syncthreads();
 
@@ -223,7 +225,10 @@ k_down_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ h,
 
     if (threadIdx.x == 0) init_header(hd, n_stages);
     ptx::launch_dependents();  // as in k_up_glu_stream
-    ptx::grid_dependency_wait();
+    // the dispatch offsets come from a kernel before the previous one (the
+    // up projection lets this grid launch only after its own dependency
+    // wait), W2 from none: the first stages' weight rows go out before the
+    // wait for the hidden vectors
     if (warp == 0) chunk_prefix<NS>(offsets, E, S, hd->prefix, err);
     __syncthreads();
 
@@ -231,8 +236,24 @@ k_down_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ h,
     const int r0 = (int)((long long)D * blockIdx.x / gridDim.x);
     const int r1 = (int)((long long)D * (blockIdx.x + 1) / gridDim.x);
     const int R = r1 - r0;
-    if (R <= 0) return;
     const uint32_t row_bytes = (uint32_t)F * 2u;
+    long long n_pre = 0;  // tasks whose weight row was sent before the wait
+    if (warp == W && lane == 0 && R > 0) {
+        const uint64_t pol_w = ptx::policy_evict_first();
+        for (int q = 0; q < Q && n_pre < n_stages; ++q) {
+            int e, j0, ns;
+            chunk_info<NS>(hd->prefix, offsets, E, q, e, j0, ns);
+            for (int r = 0; r < R && n_pre < n_stages; ++r, ++n_pre) {
+                const int st = (int)n_pre;
+                hd->tag[st] = n_pre;
+                ptx::mbar_arrive_expect_tx(&hd->full[st], row_bytes);
+                ptx::bulk_g2s(ring + (size_t)st * F, w2 + ((size_t)e * D + r0 + r) * F, row_bytes,
+                              &hd->full[st], pol_w);
+            }
+        }
+    }
+    ptx::grid_dependency_wait();  // h comes from the previous kernel
+    if (R <= 0) return;
 
     if (warp == W) {
         if (lane != 0) return;
@@ -249,6 +270,7 @@ k_down_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ h,
             ptx::bulk_g2s(hbuf + (size_t)b * NS * F, h + (size_t)j0 * F, (uint32_t)ns * row_bytes,
                           &hd->vfull[b], pol_h);
             for (int r = 0; r < R; ++r, ++i) {
+                if (i < n_pre) continue;  // sent before the dependency wait
                 const int st = (int)(i % n_stages);
                 if (!(ok = ptx::mbar_wait(&hd->empty[st], (uint32_t)((i / n_stages) & 1) ^ 1, err)))
                     break;
