@@ -43,6 +43,8 @@ struct Header {
     uint64_t vempty[2];
     long long tag[kMaxStages];  // task number of the data in each stage
     int prefix[257];
+    // one token, rows shared out: each chunk's expert and h row
+    int q_e[kStreamMaxSlots], q_j[kStreamMaxSlots];
 };
 static_assert(sizeof(Header) <= kHeaderBytes, "header too large");
 
@@ -83,7 +85,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 k_up_glu_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ x,
                 const int32_t *__restrict__ perm, const int32_t *__restrict__ offsets,
                 const bf16 *__restrict__ w1, const bf16 *__restrict__ v1, bf16 *__restrict__ h,
-                int n_stages, unsigned *err) {
+                int n_stages, int *ctr, unsigned *err) {
     extern __shared__ __align__(1024) unsigned char smem[];
     Header *hd = reinterpret_cast<Header *>(smem);
     bf16 *xbuf = reinterpret_cast<bf16 *>(smem + kHeaderBytes);  // [2][NS][D]
@@ -104,6 +106,92 @@ k_up_glu_stream(int D, int F, int E, int K, int T, const bf16 *__restrict__ x,
 
     const int Q = hd->prefix[E];
     const long long N = (long long)Q * F;
+    if (NS == 1 && T == 1 && ctr != nullptr && Q <= kStreamMaxSlots) {
+        // one token, rows shared out as they go: task g = (chunk g / F, row
+        // g % F) in batches of n_stages consecutive tasks taken from a
+        // counter (zeroed by the routing kernel), the next batch taken while
+        // the current one streams -- each SM's share of the memory bandwidth
+        // differs by a few percent, and equal static shares left the last
+        // SM ~10 us behind the first.  Every chunk holds the same token.
+        const uint32_t row_bytes = (uint32_t)D * 2u;
+        for (int q = threadIdx.x; q < Q; q += blockDim.x) {
+            const int e = chunk_expert(hd->prefix, E, q);
+            hd->q_e[q] = e;
+            hd->q_j[q] = offsets[e];
+        }
+        __syncthreads();
+        if (warp == W) {
+            if (lane != 0) return;
+            const uint64_t pol_w = ptx::policy_evict_first();
+            ptx::mbar_arrive_expect_tx(&hd->vfull[0], row_bytes);
+            ptx::bulk_g2s(xbuf, x, row_bytes, &hd->vfull[0], ptx::policy_evict_last());
+            long long i = 0;
+            bool ok = true;
+            int nxt = atomicAdd(ctr, 1);
+            for (;;) {
+                const long long g0 = (long long)nxt * n_stages;
+                if (g0 >= N) break;
+                nxt = atomicAdd(ctr, 1);
+                for (int u = 0; u < n_stages && g0 + u < N && ok; ++u, ++i) {
+                    const int st = (int)(i % n_stages);
+                    if (!(ok = ptx::mbar_wait(&hd->empty[st],
+                                              (uint32_t)((i / n_stages) & 1) ^ 1, err)))
+                        break;
+                    const long long g = g0 + u;
+                    const int q = (int)(g / F), f = (int)(g - (long long)q * F);
+                    const int e = hd->q_e[q];
+                    bf16 *dst = ring + (size_t)st * 2 * D;
+                    hd->tag[st] = g;
+                    ptx::mbar_arrive_expect_tx(&hd->full[st], 2 * row_bytes);
+                    ptx::bulk_g2s(dst, w1 + ((size_t)e * F + f) * D, row_bytes, &hd->full[st],
+                                  pol_w);
+                    ptx::bulk_g2s(dst + D, v1 + ((size_t)e * F + f) * D, row_bytes,
+                                  &hd->full[st], pol_w);
+                }
+                if (!ok) break;
+            }
+            // the end, one marker for each consumer warp (its next task)
+            for (int w = 0; w < W && ok; ++w, ++i) {
+                const int st = (int)(i % n_stages);
+                if (!(ok = ptx::mbar_wait(&hd->empty[st], (uint32_t)((i / n_stages) & 1) ^ 1,
+                                          err)))
+                    break;
+                hd->tag[st] = -1;
+                ptx::mbar_arrive(&hd->full[st]);
+            }
+            ptx::mbar_wait(&hd->vfull[0], 0, err);
+            return;
+        }
+        if (!ptx::mbar_wait(&hd->vfull[0], 0, err)) return;
+        const int nv = D >> 3;
+        for (long long i = warp;; i += W) {
+            const int st = warp;
+            if (!ptx::mbar_wait(&hd->full[st], (uint32_t)((i / n_stages) & 1), err)) return;
+            const long long g = hd->tag[st];
+            if (g < 0) return;
+            const int q = (int)(g / F), f = (int)(g - (long long)q * F);
+            const int jq = hd->q_j[q];
+            const bf16 *wr = ring + (size_t)st * 2 * D;
+            const bf16 *vr = wr + D;
+            float a = 0.f, bb = 0.f;
+#pragma unroll 2
+            for (int v = lane; v < nv; v += 32) {
+                float wv[8], vv[8], xv[8];
+                sm8(wr + v * 8, wv);
+                sm8(vr + v * 8, vv);
+                sm8(xbuf + v * 8, xv);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    a = fmaf(wv[k], xv[k], a);
+                    bb = fmaf(vv[k], xv[k], bb);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&hd->empty[st]);
+            const float as = warp_sum(a), bs = warp_sum(bb);
+            if (lane == 0) h[(size_t)jq * F + f] = __float2bfloat16_rn(silu(as) * bs);
+        }
+    }
     const long long lo = N * blockIdx.x / gridDim.x;
     const long long hi = N * (blockIdx.x + 1) / gridDim.x;
     if (lo >= hi) return;
@@ -418,7 +506,7 @@ bool stream_path_ok(const moe_dims &d, int T) {
 
 cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
                                  const int32_t *offsets, const void *w1, const void *v1, void *h,
-                                 cudaStream_t st) {
+                                 cudaStream_t st, int *ctr) {
     UpPlan p;
     if (!plan_up(d, T, p)) return cudaErrorInvalidValue;
     const void *kern = (const void *)k_up_glu_stream<kNs>;
@@ -431,7 +519,8 @@ cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const 
     const bf16 *v1p = static_cast<const bf16 *>(v1);
     bf16 *hp = static_cast<bf16 *>(h);
     unsigned *err = device_info().err;
-    void *args[] = {&D, &F, &E, &K, &Tv, &xp, &perm, &offsets, &w1p, &v1p, &hp, &ns, &err};
+    int *cp = T == 1 ? ctr : nullptr;
+    void *args[] = {&D, &F, &E, &K, &Tv, &xp, &perm, &offsets, &w1p, &v1p, &hp, &ns, &cp, &err};
     LaunchScope ls("up_glu_stream", st);
     return launch_pdl(kern, dim3(device_info().sm_count), dim3((p.n_stages + 1) * 32), p.smem, st,
                       args);

@@ -231,7 +231,7 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
                        int32_t *__restrict__ topk_idx, float *__restrict__ topk_gate,
                        int32_t *__restrict__ counts, int32_t *__restrict__ offsets,
                        int32_t *__restrict__ perm, int32_t *__restrict__ inv_perm, int staged,
-                       unsigned *err) {
+                       int *__restrict__ ctr, unsigned *err) {
     extern __shared__ __align__(128) unsigned char wsm[];  // W_r when staged
     __shared__ float part[kStagedWarps][256];
     __shared__ float lg[kStagedWarps][256];
@@ -267,6 +267,12 @@ k_route_dispatch_small(int T, int D, int E, int K, const TX *__restrict__ x,
             select_topk(E, K, warp, lg[warp], pk[warp], logits_opt, topk_idx, topk_gate,
                         sidx + warp * K);
         __syncthreads();
+    }
+    // the next kernels' work counters, for this call (the kernels that used
+    // them last finished before this one's dependency wait returned)
+    if (ctr && threadIdx.x == 0) {
+        ctr[0] = 0;
+        ctr[1] = 0;
     }
     if (warp != 0) return;
     const int S = T * K;
@@ -974,6 +980,9 @@ WsLayout ws_layout(const moe_dims &d, int64_t T) {
     L.y = o; o += (bf || T > kFusedCombineMaxTokens) ? up(S * d.d_model * 4) : 0;
     // the stream-K down projection's tails (bf16 decode batches)
     L.y_tail = o; o += (bf && T <= kStreamKMaxTokens) ? up(S * d.d_model * 4) : 0;
+    // work counters of the one-token streaming kernels (zeroed by the
+    // routing kernel of the same call)
+    L.ctr = o; o += up(4 * sizeof(int));
     L.total = o;
     return L;
 }
@@ -1029,7 +1038,7 @@ template <typename TX, typename TW>
 cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x, const void *wr,
                                         int32_t *idx, float *gate, int32_t *counts,
                                         int32_t *offsets, int32_t *perm, int32_t *inv,
-                                        cudaStream_t st) {
+                                        cudaStream_t st, int *ctr) {
     int Tv = T, D = d.d_model, E = d.n_experts, K = d.top_k;
     const TX *xp = static_cast<const TX *>(x);
     const TW *wp = static_cast<const TW *>(wr);
@@ -1044,7 +1053,7 @@ cudaError_t launch_route_dispatch_small(const moe_dims &d, int T, const void *x,
         if (e != cudaSuccess) return e;
     }
     void *args[] = {&Tv, &D, &E, &K, &xp, &wp, &logits, &idx, &gate, &counts, &offsets, &perm, &inv,
-                    &staged, &err};
+                    &staged, &ctr, &err};
     LaunchScope ls("route_dispatch_small", st);
     return launch_pdl(kern, dim3(1), dim3(kStagedThreads), staged ? wrb : 0, st, args);
 }
@@ -1113,12 +1122,13 @@ bool small_route_ok(const moe_dims &d, int T) {
 
 cudaError_t route_dispatch_small_any(const moe_dims &d, int T, const void *x, const void *wr,
                                      int32_t *idx, float *gate, int32_t *counts, int32_t *offsets,
-                                     int32_t *perm, int32_t *inv, cudaStream_t st) {
+                                     int32_t *perm, int32_t *inv, cudaStream_t st,
+                                     int *ctr = nullptr) {
     if (d.w_dtype == MOE_BF16)
         return launch_route_dispatch_small<bf16, bf16>(d, T, x, wr, idx, gate, counts, offsets,
-                                                       perm, inv, st);
+                                                       perm, inv, st, ctr);
     return launch_route_dispatch_small<float, float>(d, T, x, wr, idx, gate, counts, offsets, perm,
-                                                     inv, st);
+                                                     inv, st, ctr);
 }
 
 // scratch (optional, scratch_bytes): room for the tensor-core router's
@@ -1212,6 +1222,13 @@ template <typename P> P *at(void *ws, size_t off) {
     return reinterpret_cast<P *>(static_cast<char *>(ws) + off);
 }
 
+// The one-token streaming kernels' work counters, when the routing of the
+// same call zeroes them (route_dispatch_ws on its one-token path), else null
+// (equal static shares).
+int *stream_ctr(const moe_dims &d, int T, const WsLayout &L, void *ws) {
+    return T == 1 && small_route_ok(d, T) ? at<int>(ws, L.ctr) : nullptr;
+}
+
 // Routing and dispatch of the whole layer into the workspace regions of L:
 // the fused one-CTA or one-cluster kernels for decode batches, else the
 // router (on the tensor cores for large batches, with the GLU hidden
@@ -1227,7 +1244,7 @@ cudaError_t route_dispatch_ws(const moe_dims &d, int T, const void *x, const voi
     int32_t *inv = at<int32_t>(ws, L.inv_perm);
     if (T == 1 && small_route_ok(d, T))
         return route_dispatch_small_any(d, T, x, w_router, idx, gate, counts, offsets, perm, inv,
-                                        st);
+                                        st, stream_ctr(d, T, L, ws));
     if (cluster_route_ok(d, T))
         return route_dispatch_cluster_any(d, T, x, w_router, idx, gate, counts, offsets, perm,
                                           inv, st);
@@ -1361,7 +1378,7 @@ moe_status moe_layer_forward(const moe_dims *dims, int32_t T, const void *x, con
     if (use_stream_path(d, T)) {
         // decode, bf16: bulk-copy pipelined kernels, combine fused into the
         // down projection
-        e = launch_up_glu_stream(d, T, x, perm, offsets, w1, v1, h, st);
+        e = launch_up_glu_stream(d, T, x, perm, offsets, w1, v1, h, st, stream_ctr(d, T, L, ws));
         if (e == cudaSuccess)
             e = launch_down_stream(d, T, h, offsets, inv, w2, gate, residual_opt, out, nullptr,
                                    true, st);
@@ -1430,7 +1447,8 @@ moe_status moe_layer_forward_experts(const moe_dims *dims, int32_t T, const void
     dl.out_dtype = MOE_F32;
     const int32_t *loff = offsets + e_begin;
     if (use_stream_path(d, T)) {
-        e = launch_up_glu_stream(dl, T, x, perm, loff, w1_local, v1_local, h, st);
+        e = launch_up_glu_stream(dl, T, x, perm, loff, w1_local, v1_local, h, st,
+                                 stream_ctr(d, T, L, ws));
         if (e == cudaSuccess)
             e = launch_down_stream(dl, T, h, loff, inv, w2_local, gate, residual_opt, partial_out,
                                    nullptr, true, st);

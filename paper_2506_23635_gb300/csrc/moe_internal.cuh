@@ -207,7 +207,7 @@ struct LaunchScope {
 
 // Workspace layout of moe_layer_forward / moe_expert_ffn for T tokens.
 struct WsLayout {
-    size_t idx, gate, counts, offsets, perm, inv_perm, h, xs, y, y_tail, total;
+    size_t idx, gate, counts, offsets, perm, inv_perm, h, xs, y, y_tail, ctr, total;
 };
 // Decode batches of up to this many tokens take the stream-K down projection
 // (a second [T*K, D] fp32 output, added by the combine).
@@ -325,9 +325,12 @@ cudaError_t launch_route_tc(const moe_dims &d, int T, const void *x, const void 
 constexpr int kStreamMaxSlots = 64;
 constexpr int kStreamMaxTokens = 1;
 bool stream_path_ok(const moe_dims &d, int T);
+// ctr (optional, one token only): a counter the routing kernel zeroed; the
+// rows are then shared out as the SMs free their stages instead of in equal
+// static shares.
 cudaError_t launch_up_glu_stream(const moe_dims &d, int T, const void *x, const int32_t *perm,
                                  const int32_t *offsets, const void *w1, const void *v1, void *h,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int *ctr = nullptr);
 cudaError_t launch_down_stream(const moe_dims &d, int T, const void *h, const int32_t *offsets,
                                const int32_t *inv_perm, const void *w2, const float *gate,
                                const void *residual, void *out, float *y_sorted, bool fused,
