@@ -31,7 +31,9 @@
  * Conventions shared by every entry point:
  *   - Tensor pointers are DEVICE pointers owned by the caller, 16-byte
  *     aligned.  The library allocates no device memory; scratch space is the
- *     caller's workspace (moe_workspace_size).
+ *     caller's workspace (moe_workspace_size), which also holds the work
+ *     counters the one-token kernels share out rows with: calls that run at
+ *     the same time on the GPU need workspaces of their own.
  *   - Calls are asynchronous on `stream` and never synchronise with the host
  *     (except moe_get_last_error and moe_profile_read).
  *   - Arguments are validated before anything is launched; on a validation
